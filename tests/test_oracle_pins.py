@@ -1,0 +1,249 @@
+"""Pins the oracle to things other than itself (CPU only).
+
+* Candidate search (Eq. 1 + longest-suffix n-gram): an independent brute force
+  that finds n-gram occurrences with ``bytes.find`` over a fixed-width byte
+  encoding of the tokens, run exhaustively on tiny contexts.
+* Hidden ranking (Eq. 3): ``scipy.spatial.distance.cosine`` on random rows, and
+  the planted-source statistic (source + N(0, 0.1^2) noise has cosine
+  1/sqrt(1.01) ~ 0.995; unrelated N(0,1) rows have |cos| < 0.1 at d = 4096).
+* Attention ranking (Eq. 2): ``numpy`` max/sum over the selected rows.
+* Verification (Sec. 4.4): ``numpy.argmax`` (documented first occurrence) and
+  the accept-length invariants.
+"""
+import itertools
+
+import numpy as np
+import pytest
+from scipy.spatial.distance import cosine as scipy_cosine
+
+
+# ----------------------------------------------------------------------------
+# candidate search
+# ----------------------------------------------------------------------------
+def _occurrences_by_bytes(seq, L, nmin, nmax):
+    """Longest-suffix n-gram occurrences, found by substring search on bytes."""
+    t = L - 1
+    if t < 1:
+        return [], 0
+    enc = b"".join(int(v).to_bytes(4, "big", signed=True) for v in seq[:L])
+    for n in range(nmax, nmin - 1, -1):
+        if t - n + 1 < 0:
+            continue
+        needle = enc[4 * (t - n + 1): 4 * (t + 1)]
+        hay = enc[: 4 * t]            # the n-gram must END before t, i.e. j < t
+        found, start = [], 0
+        while True:
+            k = hay.find(needle, start)
+            if k < 0:
+                break
+            if k % 4 == 0:            # token-aligned hit; it ends at position j
+                found.append(k // 4 + n - 1)
+            start = k + 1
+        if found:
+            return sorted(found), n
+    return [], 0
+
+
+def test_find_exhaustive_binary_alphabet(orc):
+    # every binary context of length 1..9 (1022 contexts), several n ranges
+    ctx, lens = [], []
+    for L in range(1, 10):
+        for bits in itertools.product([0, 1], repeat=L):
+            ctx.append(list(bits) + [0] * (9 - L))
+            lens.append(L)
+    ids = np.array(ctx, np.int32)
+    for nmin, nmax in [(1, 1), (1, 2), (1, 3), (2, 3), (3, 3), (1, 4)]:
+        cand, cnt, ml, st = orc.find_candidates(ids, lens, nmin, nmax, 16)
+        for b, L in enumerate(lens):
+            want, n = _occurrences_by_bytes(ids[b], L, nmin, nmax)
+            assert cnt[b] == len(want) and ml[b] == n, (ids[b, :L], nmin, nmax)
+            assert cand[b, :len(want)].tolist() == want
+            assert st[b] == 0
+
+
+@pytest.mark.parametrize("V,T", [(3, 40), (5, 200), (50, 300)])
+def test_find_random_vs_bytes_search(orc, V, T):
+    rng = np.random.default_rng(V * 1000 + T)
+    B = 64
+    ids = rng.integers(0, V, size=(B, T)).astype(np.int32)
+    lens = rng.integers(0, T + 1, size=B)
+    cand, cnt, ml, st = orc.find_candidates(ids, lens, 1, 3, T)
+    for b in range(B):
+        want, n = _occurrences_by_bytes(ids[b], lens[b], 1, 3)
+        assert cnt[b] == len(want) and ml[b] == n
+        assert cand[b, :len(want)].tolist() == want
+
+
+def test_find_unigram_is_eq1(orc):
+    rng = np.random.default_rng(7)
+    ids = rng.integers(0, 6, size=(32, 50)).astype(np.int32)
+    lens = rng.integers(2, 51, size=32)
+    cand, cnt, ml, _ = orc.find_candidates(ids, lens, 1, 1, 50)
+    for b in range(32):
+        t = lens[b] - 1
+        eq1 = [j for j in range(t) if ids[b, j] == ids[b, t]]        # Eq. 1 literally
+        assert cand[b, :cnt[b]].tolist() == eq1
+        assert ml[b] == (1 if eq1 else 0)
+
+
+def test_find_overflow_keeps_first_ascending(orc):
+    ids = np.zeros((1, 100), np.int32)
+    cand, cnt, ml, st = orc.find_candidates(ids, [100], 1, 3, 10)
+    assert cnt[0] == 97 and ml[0] == 3            # j = 2..98
+    assert cand[0].tolist() == list(range(2, 12))
+    assert st[0] == orc.ST_CAND_OVERFLOW
+
+
+# ----------------------------------------------------------------------------
+# hidden-state ranking
+# ----------------------------------------------------------------------------
+def test_rank_hidden_matches_scipy(orc):
+    rng = np.random.default_rng(11)
+    B, T, d = 4, 30, 257
+    H = rng.standard_normal((B, T, d)).astype(np.float32)
+    lens = np.array([30, 17, 5, 30], np.int32)
+    cands = np.tile(np.arange(0, 29, dtype=np.int32), (B, 1))
+    cnt = np.array([29, 16, 4, 29], np.int32)
+    scores, best, bs = orc.rank_hidden(H, lens, cands, cnt)
+    for b in range(B):
+        t = lens[b] - 1
+        ref = [-np.inf] + [1.0 - scipy_cosine(H[b, j - 1].astype(np.float64),
+                                              H[b, t - 1].astype(np.float64)) for j in range(1, cnt[b])]
+        np.testing.assert_allclose(scores[b, :cnt[b]], ref, rtol=0, atol=1e-12)
+        jb = int(np.argmax(ref))
+        assert best[b] == jb and abs(bs[b] - ref[jb]) < 1e-12
+
+
+def test_rank_hidden_bf16_is_exact_widening(orc):
+    rng = np.random.default_rng(12)
+    H32 = rng.standard_normal((2, 20, 64)).astype(np.float32)
+    bits = orc.bf16_bits(H32)
+    exact = orc.bf16_to_f32(bits)
+    cands = np.tile(np.arange(1, 19, dtype=np.int32), (2, 1))
+    s_bf, b_bf, _ = orc.rank_hidden(bits, [20, 20], cands, [18, 18])
+    s_32, b_32, _ = orc.rank_hidden(exact, [20, 20], cands, [18, 18])
+    assert np.array_equal(s_bf, s_32) and np.array_equal(b_bf, b_32)
+
+
+def test_rank_hidden_planted_source_wins(orc):
+    """Sec. 4.2.2 premise: the row before the true copy source resembles the query row.
+    Query H_{t-1} = H_{s-1} + N(0, 0.1^2); the source s must win, with the
+    expected cosine ~ 1/sqrt(1.01); wrong query/candidate rows would not."""
+    rng = np.random.default_rng(13)
+    B, T, d = 8, 64, 4096
+    H = rng.standard_normal((B, T, d)).astype(np.float32)
+    lens = np.full(B, T, np.int32)
+    t = T - 1
+    srcs = rng.integers(1, t - 2, size=B)
+    for b in range(B):
+        H[b, t - 1] = H[b, srcs[b] - 1] + 0.1 * rng.standard_normal(d).astype(np.float32)
+    cands = np.tile(np.arange(1, t, dtype=np.int32), (B, 1))
+    scores, best, bs = orc.rank_hidden(H, lens, cands, np.full(B, t - 1, np.int32))
+    assert best.tolist() == srcs.tolist()
+    assert np.all(np.abs(bs - 1 / np.sqrt(1.01)) < 0.005)
+    others = np.array([[scores[b, i] for i in range(t - 1) if i + 1 != srcs[b] and i + 2 != t]
+                       for b in range(B)])
+    assert np.abs(others).max() < 0.1
+
+
+def test_rank_hidden_zero_norm_threshold_ineligible(orc):
+    H = np.zeros((1, 6, 8), np.float32)
+    H[0, 4] = 1.0                                   # query row H_{t-1}, t = 5
+    H[0, 2] = -1.0
+    cands = np.array([[0, 1, 3]], np.int32)         # j=0 ineligible, j=1 -> H_0 = 0, j=3 -> H_2
+    scores, best, bs = orc.rank_hidden(H, [6], cands, [3])
+    assert scores[0, 0] == -np.inf and scores[0, 1] == 0.0 and scores[0, 2] == -1.0
+    assert best[0] == 1 and bs[0] == 0.0
+    _, best, bs = orc.rank_hidden(H, [6], cands, [3], threshold=0.0)     # strict: 0 > 0 fails
+    assert best[0] == -1 and bs[0] == -np.inf
+
+
+# ----------------------------------------------------------------------------
+# attention ranking
+# ----------------------------------------------------------------------------
+@pytest.mark.parametrize("agg", ["max", "sum"])
+def test_rank_attention_matches_numpy(orc, agg):
+    rng = np.random.default_rng(21)
+    B, R, T = 5, 12, 40
+    A = rng.random((B, R, T)).astype(np.float32)
+    lens = rng.integers(2, T + 1, size=B).astype(np.int32)
+    C = 16
+    cands = np.stack([np.sort(rng.choice(T, C, replace=False)) for _ in range(B)]).astype(np.int32)
+    cnt = rng.integers(0, C + 1, size=B).astype(np.int32)
+    rows = np.array([3, 0, 7, 11], np.int32)
+    code = orc.AGG_MAX if agg == "max" else orc.AGG_SUM
+    scores, best, bs = orc.rank_attention(A, lens, cands, cnt, row_idx=rows, agg=code)
+    for b in range(B):
+        sel = A[b][rows].astype(np.float64)
+        red = sel.max(axis=0) if agg == "max" else sel.sum(axis=0)
+        want = [red[j] if j < lens[b] - 1 else -np.inf for j in cands[b, :cnt[b]]]
+        np.testing.assert_allclose(scores[b, :cnt[b]], want, rtol=0, atol=1e-12)
+        valid = [(w, -j) for w, j in zip(want, cands[b, :cnt[b]]) if np.isfinite(w)]
+        assert best[b] == (-max(valid)[1] if valid else -1)
+
+
+def test_rank_attention_planted_key_is_candidate_itself(orc):
+    """Reading of Eq. 2: the induction row of query t-1 peaks at key j (the copied
+    token), so planting mass at key s selects s, not s+1 or s-1."""
+    rng = np.random.default_rng(22)
+    B, R, T = 6, 8, 50
+    logits = rng.standard_normal((B, R, T))
+    srcs = rng.integers(5, 40, size=B)
+    for b in range(B):
+        logits[b, :3, srcs[b]] += 6.0
+    A = np.exp(logits) / np.exp(logits).sum(-1, keepdims=True)
+    cands = np.tile(np.arange(0, T - 1, dtype=np.int32), (B, 1))
+    _, best, _ = orc.rank_attention(A.astype(np.float32), np.full(B, T, np.int32), cands,
+                                    np.full(B, T - 1, np.int32))
+    assert best.tolist() == srcs.tolist()
+
+
+# ----------------------------------------------------------------------------
+# draft + verify
+# ----------------------------------------------------------------------------
+def test_extract_draft_is_following_span(orc):
+    rng = np.random.default_rng(31)
+    B, T, K = 40, 30, 7
+    ids = rng.integers(0, 1000, size=(B, T)).astype(np.int32)
+    lens = rng.integers(0, T + 1, size=B).astype(np.int32)
+    best = rng.integers(-1, T, size=B).astype(np.int32)
+    draft, dl = orc.extract_draft(ids, lens, best, K)
+    for b in range(B):
+        t = lens[b] - 1
+        span = list(ids[b, best[b] + 1: t + 1][:K]) if 0 <= best[b] < t else []
+        assert dl[b] == len(span)
+        assert draft[b].tolist() == span + [-1] * (K - len(span))
+
+
+@pytest.mark.parametrize("bf16", [False, True])
+def test_verify_matches_numpy_argmax_and_invariants(orc, bf16):
+    rng = np.random.default_rng(41 + bf16)
+    B, K, V = 64, 6, 37
+    logits = rng.integers(-3, 4, size=(B, K + 1, V)).astype(np.float32)   # many exact ties
+    logits[logits == 0] = np.where(rng.random((logits == 0).sum()) < 0.5, -0.0, 0.0)
+    am = logits.argmax(-1)                                                 # first occurrence
+    draft = np.where(rng.random((B, K)) < 0.8, am[:, :K], rng.integers(0, V, size=(B, K)))
+    dlen = rng.integers(0, K + 1, size=B)
+    draft = np.where(np.arange(K)[None] < dlen[:, None], draft, -1).astype(np.int32)
+    T_cap = 20
+    ids = rng.integers(0, V, size=(B, T_cap)).astype(np.int32)
+    lens = rng.integers(1, T_cap + 1, size=B).astype(np.int32)
+    ids0, lens0 = ids.copy(), lens.copy()
+    x = orc.bf16_bits(logits) if bf16 else logits
+    out = orc.verify_greedy(x, draft, dlen, ids=ids, seq_len=lens, kv_keep=True)
+    assert np.array_equal(out["argmax"], am)
+    for b in range(B):
+        d = dlen[b]
+        mism = [i for i in range(d) if draft[b, i] != am[b, i]]
+        n = mism[0] if mism else d
+        assert 0 <= out["accept_len"][b] <= d <= K
+        assert out["accept_len"][b] == n and out["next_token"][b] == am[b, n]
+        assert out["kv_keep_len"][b] == lens0[b] + n
+        if lens0[b] + n + 1 <= T_cap:
+            assert lens[b] == lens0[b] + n + 1 and out["status"][b] == 0
+            emitted = list(draft[b, :n]) + [am[b, n]]
+            assert ids[b, lens0[b]:lens[b]].tolist() == emitted
+            assert np.array_equal(ids[b, :lens0[b]], ids0[b, :lens0[b]])
+        else:
+            assert lens[b] == lens0[b] and out["status"][b] == orc.ST_CAPACITY
+            assert np.array_equal(ids[b], ids0[b])
