@@ -1,0 +1,238 @@
+/*
+ * pldp.h -- C ABI of the GB300 (sm_103a) PLD+ drafting and greedy
+ * verification library.
+ *
+ * PLD+ (arXiv 2412.01447) speeds up decoding of input-guided tasks by
+ * drafting a span copied from the context and verifying it with one forward
+ * pass of the target model.  Per decode step and per sequence this library:
+ *
+ *   1. finds the earlier occurrences P of the last token (Eq. 1), narrowed to
+ *      the longest suffix n-gram that occurs earlier     -> pldp_find_candidates
+ *   2. ranks P with a model artifact: the cosine between hidden states
+ *      H_{j-1} and H_{t-1} (Eq. 3)                        -> pldp_rank_hidden
+ *      or the max attention of query t-1 over selected
+ *      (layer, head) rows (Eq. 2)                         -> pldp_rank_attention
+ *   3. drafts the K tokens after the best occurrence j*
+ *      (Sec. 4.3)                                         -> pldp_extract_draft
+ *   4. verifies the draft greedily against the target
+ *      model's K+1 next-token distributions (Sec. 4.4)    -> pldp_verify_greedy
+ *
+ * Conventions shared by every call
+ *  - Every pointer argument is a DEVICE pointer owned by the caller; the
+ *    library allocates nothing and keeps no state between calls, except the
+ *    caller-provided verification workspace described at pldp_verify_greedy.
+ *  - All work is enqueued asynchronously on `stream` (a cudaStream_t; NULL is
+ *    the legacy default stream).  No call synchronises the device or reads
+ *    device memory on the host, so every call may be captured in a CUDA graph.
+ *  - Positions are 0-based int32.  Sequence b holds seq_len[b] tokens in
+ *    ids[b*ids_stride + 0 .. seq_len[b]-1]; its last token is x_t with
+ *    t = seq_len[b] - 1.  Model artifacts exist for positions 0..t-1 only.
+ *  - Host-side argument checks run before anything is enqueued; a failed
+ *    check returns PLDP_ERR_INVALID_ARG (or PLDP_ERR_UNSUPPORTED) and
+ *    enqueues nothing.  A CUDA launch failure returns PLDP_ERR_CUDA.
+ *    pldp_last_error() then gives a message (per host thread).
+ *  - Data-dependent problems found on the device never trap: they set bits in
+ *    the optional per-sequence status word (uint32 status[B], OR-ed in; the
+ *    caller clears it) and the call produces the documented fallback.
+ *  - dtype PLDP_BF16 data is raw bfloat16; PLDP_F32 is IEEE float.  Inputs
+ *    must be finite (NaN is not supported).
+ *  - Calls that overlap on the device must not share output buffers.
+ */
+#ifndef PLDP_H
+#define PLDP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(_WIN32)
+#define PLDP_API
+#else
+#define PLDP_API __attribute__((visibility("default")))
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    PLDP_OK = 0,
+    PLDP_ERR_INVALID_ARG = 1, /* null/misaligned pointer, bad size or stride  */
+    PLDP_ERR_UNSUPPORTED = 2, /* dtype or size the kernels do not handle      */
+    PLDP_ERR_CUDA = 3,        /* launch failed; see pldp_last_error()         */
+    PLDP_ERR_TIMEOUT = 4      /* reserved: no call waits on the host          */
+} pldp_status;
+
+typedef enum { PLDP_F32 = 0, PLDP_BF16 = 1 } pldp_dtype;
+
+typedef enum { PLDP_AGG_MAX = 0, PLDP_AGG_SUM = 1 } pldp_agg;
+
+/* Per-sequence device status bits. */
+#define PLDP_ST_CAND_OVERFLOW 1u  /* |P| > C_cap: the first C_cap positions are listed   */
+#define PLDP_ST_TOKEN_RANGE   2u  /* a draft token outside [0, V)                        */
+#define PLDP_ST_CAPACITY      4u  /* the append would pass T_cap: nothing appended       */
+#define PLDP_ST_SEQ_LEN       8u  /* seq_len outside its valid range: sequence skipped   */
+#define PLDP_ST_DRAFT_LEN    16u  /* draft_len outside [0, K]: clamped into it           */
+#define PLDP_ST_ROW_INDEX    32u  /* a row_idx entry outside [0, R): that row ignored    */
+#define PLDP_ST_TIMEOUT      64u  /* an on-chip copy did not complete in time: no result */
+
+#define PLDP_MAX_NGRAM 8          /* largest ngram_max accepted                          */
+
+/*
+ * Candidate search -- Eq. 1 (Sec. 4.2):  P = { j | x_j = x_t, j < t },
+ * narrowed by the longest-suffix n-gram rule of prompt lookup (Sec. 2, Fig. 2
+ * caption): for n = ngram_max down to ngram_min, the first non-empty
+ *   P_n = { j < t : j-n+1 >= 0 and x_{j-k} = x_{t-k} for k = 0..n-1 }
+ * is P and n is match_len[b].  ngram_min = ngram_max = 1 is Eq. 1 itself.
+ *
+ *  ids        int32 [B, ids_stride]; row b holds the context of sequence b.
+ *  ids_stride elements between rows (>= T_cap).
+ *  seq_len    int32 [B]; valid range [0, T_cap] (else SEQ_LEN, nothing found).
+ *  T_cap      row capacity: positions >= T_cap are never read.
+ *  ngram_min, ngram_max   1 <= ngram_min <= ngram_max <= PLDP_MAX_NGRAM.
+ *  cand_pos   int32 [B, C_cap] out: P in ascending order; slots past
+ *             min(|P|, C_cap) are left untouched.
+ *  C_cap      >= 0.  |P| > C_cap lists the first C_cap and sets CAND_OVERFLOW.
+ *  cand_count int32 [B] out: the true |P| (even when it exceeds C_cap).
+ *  match_len  int32 [B] out: the n of P, 0 when P is empty.
+ *  status     uint32 [B] or NULL.
+ * Fast path when ids is 16-byte aligned and ids_stride % 4 == 0.
+ */
+PLDP_API pldp_status pldp_find_candidates(const int32_t* ids, int64_t ids_stride,
+                                          const int32_t* seq_len, int B, int64_t T_cap,
+                                          int ngram_min, int ngram_max,
+                                          int32_t* cand_pos, int C_cap,
+                                          int32_t* cand_count, int32_t* match_len,
+                                          uint32_t* status, void* stream);
+
+/*
+ * Ranking by hidden states -- Eq. 3 (Sec. 4.2.2):
+ *   score_j = cos(H_{j-1}, H_{t-1}),  j* = argmax_{j in P} score_j,
+ * with the optional threshold of App. B.3 (j kept only if score_j > threshold;
+ * pass -INFINITY for none).  The caller passes the chosen layer l only.
+ *
+ *  H          [B, seq_stride] elements of dtype; row p of sequence b is
+ *             H + b*seq_stride + p*d (rows are contiguous, d elements each).
+ *  d          hidden width, 1 <= d and d * sizeof(dtype) <= 196608.
+ *  seq_stride elements between sequences (>= T_cap * d).
+ *  seq_len    int32 [B]; valid range [0, T_cap] (else SEQ_LEN, no result).
+ *  T_cap      row capacity of H: rows >= T_cap are never read.
+ *  cand_pos, cand_count, C_cap   as written by pldp_find_candidates; entries
+ *             past min(cand_count, C_cap) are ignored.
+ *  scores     float [B, C_cap] out or NULL: score of the i-th listed candidate.
+ *             j = 0 (no H_{-1}) and positions outside [0, t) score -INFINITY
+ *             and are never chosen.  A zero-norm row gives score 0.
+ *  best_pos   int32 [B] out: j*, or -1 when no candidate is eligible.
+ *  best_score float [B] out or NULL: score of j* (-INFINITY when none).
+ *  status     uint32 [B] or NULL.
+ * Scores are accumulated in fp32.  Ties go to the smaller position j; the
+ * choice is deterministic for given inputs.  When H rows are 16-byte aligned
+ * (H aligned, d*sizeof(dtype) and seq_stride*sizeof(dtype) multiples of 16)
+ * the query row is staged in shared memory by a bulk asynchronous copy.
+ */
+PLDP_API pldp_status pldp_rank_hidden(const void* H, pldp_dtype dtype, int64_t d,
+                                      int64_t seq_stride, const int32_t* seq_len, int B,
+                                      int64_t T_cap, const int32_t* cand_pos,
+                                      const int32_t* cand_count, int C_cap, float threshold,
+                                      float* scores, int32_t* best_pos, float* best_score,
+                                      uint32_t* status, void* stream);
+
+/*
+ * Ranking by attentions -- Eq. 2 (Sec. 4.2.1):
+ *   score_j = max over the selected (layer, head) rows of A^{(l,g)}_{t-1}[j],
+ *   j* = argmax_{j in P} score_j;  agg = PLDP_AGG_SUM sums the rows instead
+ *   (the aggregation variant of Sec. 7.1).
+ * The key index of Eq. 2 is read as the candidate j itself (the position an
+ * induction head at query t-1 attends to is the token it copies).
+ *
+ *  A          dtype; for sequence b and row r the attention probabilities of
+ *             query t-1 over keys: A + b*seq_stride + r*row_stride + key.
+ *  R          rows per sequence (>= 1); row_stride >= T_cap; seq_stride >=
+ *             R * row_stride.
+ *  row_idx    int32 [n_sel] device, or NULL for all R rows: the selected
+ *             (layer, head) rows L* x G*.  Entries outside [0, R) are ignored
+ *             and set ROW_INDEX.
+ *  seq_len, T_cap, cand_pos, cand_count, C_cap, status   as pldp_rank_hidden.
+ *  scores     float [B, C_cap] out or NULL.  Positions outside [0, t) score
+ *             -INFINITY and are never chosen.
+ *  best_pos, best_score   as pldp_rank_hidden.  Ties go to the smaller j.
+ * MAX is exact; SUM accumulates in fp32 in a fixed order.
+ */
+PLDP_API pldp_status pldp_rank_attention(const void* A, pldp_dtype dtype, int R,
+                                         int64_t row_stride, int64_t seq_stride,
+                                         const int32_t* row_idx, int n_sel, pldp_agg agg,
+                                         const int32_t* seq_len, int B, int64_t T_cap,
+                                         const int32_t* cand_pos, const int32_t* cand_count,
+                                         int C_cap, float* scores, int32_t* best_pos,
+                                         float* best_score, uint32_t* status, void* stream);
+
+/*
+ * Draft prediction -- Sec. 4.3:  xhat_i = x_{j*+i}, i = 1..K.
+ * The span stops at the last token x_t: draft_len[b] = min(K, t - j*) tokens,
+ * the rest of draft[b, :] is -1.  best_pos[b] = -1 (or outside [0, t), or an
+ * invalid seq_len) gives draft_len 0.
+ *
+ *  ids, ids_stride, seq_len, T_cap   as pldp_find_candidates.
+ *  best_pos   int32 [B].
+ *  K          draft length, >= 1.
+ *  draft      int32 [B, K] out;  draft_len  int32 [B] out.
+ */
+PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
+                                        const int32_t* seq_len, int64_t T_cap,
+                                        const int32_t* best_pos, int B, int K,
+                                        int32_t* draft, int32_t* draft_len, void* stream);
+
+/*
+ * Greedy verification -- Sec. 4.4 at temperature 0, with the K+1 next-token
+ * distributions of one forward pass on the draft (Sec. 3):
+ *   a_i   = argmax_v logits[b, i, v], i = 0..K   (smallest v among equal maxima;
+ *           -0.0 equals +0.0)
+ *   n     = first i < draft_len[b] with draft[b, i] != a_i, else draft_len[b]
+ *   bonus = a_n
+ * accept_len[b] = n and next_token[b] = bonus: the step emits
+ * draft[b, 0..n-1] followed by bonus, exactly what greedy decoding emits.
+ *
+ *  logits     dtype [B, K+1, V], contiguous.  Fast path when logits is 16-byte
+ *             aligned and V * sizeof(dtype) is a multiple of 16.
+ *  draft      int32 [B, K];  draft_len  int32 [B] (outside [0, K]: clamped,
+ *             DRAFT_LEN).  Draft tokens outside [0, V) never match (TOKEN_RANGE).
+ *  argmax     int32 [B, K+1] out or NULL: every a_i.
+ *  accept_len int32 [B] out;  next_token int32 [B] out.
+ *  seq_len    int32 [B] in/out or NULL.  When given (valid range [1, T_cap],
+ *             else SEQ_LEN and no bookkeeping for b), with L the old value:
+ *               kv_keep_len[b] = L + n   (x_t and the n accepted tokens are the
+ *                                         positions whose keys/values survive)
+ *               if L + n + 1 <= T_cap: ids[b, L..L+n-1] = draft[b, 0..n-1],
+ *                 ids[b, L+n] = bonus (ids may be NULL), seq_len[b] = L + n + 1;
+ *               else CAPACITY and neither ids nor seq_len changes.
+ *  ids, ids_stride, T_cap   the context rows to append to (ids may be NULL).
+ *  kv_keep_len int32 [B] out or NULL (needs seq_len).
+ *  status     uint32 [B] or NULL.
+ *  workspace  device scratch of at least pldp_verify_workspace_size(B, K, V)
+ *             bytes, 16-byte aligned, ZEROED by the caller before its first
+ *             use.  Every call returns it to all-zero when it completes, so
+ *             it can be reused by the next call on the same stream (or graph
+ *             replay) without clearing.  Calls that may run concurrently need
+ *             separate workspaces.
+ */
+PLDP_API pldp_status pldp_verify_greedy(const void* logits, pldp_dtype dtype, int B, int K,
+                                        int V, const int32_t* draft, const int32_t* draft_len,
+                                        int32_t* argmax, int32_t* accept_len,
+                                        int32_t* next_token, int32_t* ids, int64_t ids_stride,
+                                        int32_t* seq_len, int64_t T_cap, int32_t* kv_keep_len,
+                                        uint32_t* status, void* workspace,
+                                        size_t workspace_bytes, void* stream);
+
+/* Bytes of workspace pldp_verify_greedy needs for these sizes (0 if invalid). */
+PLDP_API size_t pldp_verify_workspace_size(int B, int K, int V);
+
+/* Message describing the last failed call on this host thread ("" if none). */
+PLDP_API const char* pldp_last_error(void);
+
+/* Library version (major * 10000 + minor * 100 + patch). */
+PLDP_API int pldp_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PLDP_H */

@@ -36,7 +36,7 @@ _LIB_PATH = os.path.join(_HERE, "liboracle.so")
 
 F32, BF16 = 0, 1
 AGG_MAX, AGG_SUM = 0, 1
-ST_CAND_OVERFLOW, ST_TOKEN_RANGE, ST_CAPACITY, ST_SEQ_LEN, ST_DRAFT_LEN = 1, 2, 4, 8, 16
+ST_CAND_OVERFLOW, ST_TOKEN_RANGE, ST_CAPACITY, ST_SEQ_LEN, ST_DRAFT_LEN, ST_ROW_INDEX = 1, 2, 4, 8, 16, 32
 
 _lock = threading.Lock()
 _lib = None
@@ -67,10 +67,10 @@ def _configure(lib):
     P = ctypes.c_void_p
     i32, i64, dbl = ctypes.c_int, ctypes.c_int64, ctypes.c_double
     lib.pldpo_find_candidates.argtypes = [P, i64, P, i32, i64, i32, i32, P, i32, P, P, P]
-    lib.pldpo_rank_hidden.argtypes = [P, i32, i64, i64, P, i32, P, P, i32, dbl, P, P, P]
-    lib.pldpo_rank_attention.argtypes = [P, i32, i32, i64, i64, P, i32, i32, P, i32, P, P, i32,
-                                         P, P, P]
-    lib.pldpo_extract_draft.argtypes = [P, i64, P, P, i32, i32, P, P]
+    lib.pldpo_rank_hidden.argtypes = [P, i32, i64, i64, P, i32, i64, P, P, i32, dbl, P, P, P, P]
+    lib.pldpo_rank_attention.argtypes = [P, i32, i32, i64, i64, P, i32, i32, P, i32, i64, P, P, i32,
+                                         P, P, P, P]
+    lib.pldpo_extract_draft.argtypes = [P, i64, P, i64, P, i32, i32, P, P]
     lib.pldpo_verify_greedy.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64, P, i64, P, P]
     for f in ("pldpo_find_candidates", "pldpo_rank_hidden", "pldpo_rank_attention",
               "pldpo_extract_draft", "pldpo_verify_greedy"):
@@ -139,9 +139,10 @@ def find_candidates(ids, seq_len, ngram_min, ngram_max, C_cap):
     return cand, cnt, ml, st
 
 
-def rank_hidden(H, seq_len, cand_pos, cand_count, threshold=-np.inf):
+def rank_hidden(H, seq_len, cand_pos, cand_count, threshold=-np.inf, status=None):
     """Eq. 3.  H: [B, T_cap, d] float32 or bf16 bits (uint16).  Returns
-    (scores [B, C_cap] f64, best_pos [B] int32, best_score [B] f64)."""
+    (scores [B, C_cap] f64, best_pos [B] int32, best_score [B] f64); ``status``
+    (numpy uint32 [B]) is OR-ed into when given."""
     H, dt = _elem(H)
     B, T_cap, d = H.shape
     cand_pos = _i32(cand_pos)
@@ -150,13 +151,13 @@ def rank_hidden(H, seq_len, cand_pos, cand_count, threshold=-np.inf):
     scores = np.full((B, C_cap), np.nan)
     best = np.zeros(B, np.int32)
     bs = np.zeros(B)
-    _check(_load().pldpo_rank_hidden(_ptr(H), dt, d, T_cap * d, _ptr(seq_len), B, _ptr(cand_pos),
+    _check(_load().pldpo_rank_hidden(_ptr(H), dt, d, T_cap * d, _ptr(seq_len), B, T_cap, _ptr(cand_pos),
                                      _ptr(cand_count), C_cap, float(threshold), _ptr(scores),
-                                     _ptr(best), _ptr(bs)), "rank_hidden")
+                                     _ptr(best), _ptr(bs), _ptr(status)), "rank_hidden")
     return scores, best, bs
 
 
-def rank_attention(A, seq_len, cand_pos, cand_count, row_idx=None, agg=AGG_MAX):
+def rank_attention(A, seq_len, cand_pos, cand_count, row_idx=None, agg=AGG_MAX, status=None):
     """Eq. 2.  A: [B, R, T_cap] float32 or bf16 bits (uint16), row r = attention of
     query t-1 for the r-th (layer, head).  Returns (scores, best_pos, best_score)."""
     A, dt = _elem(A)
@@ -170,8 +171,9 @@ def rank_attention(A, seq_len, cand_pos, cand_count, row_idx=None, agg=AGG_MAX):
     best = np.zeros(B, np.int32)
     bs = np.zeros(B)
     _check(_load().pldpo_rank_attention(_ptr(A), dt, R, T_cap, R * T_cap, _ptr(ri), n_sel, agg,
-                                        _ptr(seq_len), B, _ptr(cand_pos), _ptr(cand_count),
-                                        C_cap, _ptr(scores), _ptr(best), _ptr(bs)), "rank_attention")
+                                        _ptr(seq_len), B, T_cap, _ptr(cand_pos), _ptr(cand_count),
+                                        C_cap, _ptr(scores), _ptr(best), _ptr(bs), _ptr(status)),
+           "rank_attention")
     return scores, best, bs
 
 
@@ -182,7 +184,7 @@ def extract_draft(ids, seq_len, best_pos, K):
     seq_len, best_pos = _i32(seq_len), _i32(best_pos)
     draft = np.zeros((B, K), np.int32)
     dl = np.zeros(B, np.int32)
-    _check(_load().pldpo_extract_draft(_ptr(ids), T_cap, _ptr(seq_len), _ptr(best_pos), B, K,
+    _check(_load().pldpo_extract_draft(_ptr(ids), T_cap, _ptr(seq_len), T_cap, _ptr(best_pos), B, K,
                                        _ptr(draft), _ptr(dl)), "extract_draft")
     return draft, dl
 

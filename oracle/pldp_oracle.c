@@ -38,6 +38,7 @@
 #define ORC_ST_CAPACITY      4u  /* append would exceed T_cap: no append  */
 #define ORC_ST_SEQ_LEN       8u  /* seq_len outside [0, T_cap] (or < 1)   */
 #define ORC_ST_DRAFT_LEN    16u  /* draft_len outside [0, K]: clamped     */
+#define ORC_ST_ROW_INDEX    32u  /* selected row outside [0, R): ignored  */
 
 #define ORC_F32  0
 #define ORC_BF16 1
@@ -122,6 +123,7 @@ int pldpo_find_candidates(const int32_t* ids, int64_t ids_stride,
  * READING: a zero-norm vector gives cos = 0 (no epsilon otherwise).
  * READING: ties go to the smallest position j.
  * scores[b*C_cap + i] is the score of the i-th listed candidate.
+ * A seq_len outside [0, T_cap] skips the sequence (SEQ_LEN, best_pos = -1).
  * ------------------------------------------------------------------------ */
 static double orc_cosine(const void* H, int dtype, int64_t row_a, int64_t row_b, int64_t d) {
     double dot = 0.0, na = 0.0, nb = 0.0;
@@ -137,12 +139,18 @@ static double orc_cosine(const void* H, int dtype, int64_t row_a, int64_t row_b,
 }
 
 int pldpo_rank_hidden(const void* H, int dtype, int64_t d, int64_t seq_stride,
-                      const int32_t* seq_len, int B,
+                      const int32_t* seq_len, int B, int64_t T_cap,
                       const int32_t* cand_pos, const int32_t* cand_count, int C_cap,
                       double threshold, double* scores,
-                      int32_t* best_pos, double* best_score) {
+                      int32_t* best_pos, double* best_score, uint32_t* status) {
     if (B < 0 || d < 1 || C_cap < 0 || (dtype != ORC_F32 && dtype != ORC_BF16)) return 1;
     for (int b = 0; b < B; ++b) {
+        if (seq_len[b] < 0 || seq_len[b] > T_cap) {         /* sequence skipped */
+            if (status) status[b] |= ORC_ST_SEQ_LEN;
+            best_pos[b] = -1;
+            if (best_score) best_score[b] = -INFINITY;
+            continue;
+        }
         int64_t t = (int64_t)seq_len[b] - 1;
         int64_t n = cand_count[b] < 0 ? 0 : cand_count[b];
         if (n > C_cap) n = C_cap;
@@ -179,22 +187,31 @@ int pldpo_rank_hidden(const void* H, int dtype, int64_t d, int64_t seq_stride,
  * earlier occurrence of x_{t-1}, i.e. to the copied token x_j).
  * agg = SUM aggregates by summation instead (the Sec. 7.1 variant).
  * Ties go to the smallest j.  Candidates outside [0, t) score -inf and are
- * not eligible.
+ * not eligible.  Selected rows outside [0, R) are left out (ROW_INDEX).
+ * A seq_len outside [0, T_cap] skips the sequence (SEQ_LEN, best_pos = -1).
  * ------------------------------------------------------------------------ */
 int pldpo_rank_attention(const void* A, int dtype, int R, int64_t row_stride, int64_t seq_stride,
                          const int32_t* row_idx, int n_sel, int agg,
-                         const int32_t* seq_len, int B,
+                         const int32_t* seq_len, int B, int64_t T_cap,
                          const int32_t* cand_pos, const int32_t* cand_count, int C_cap,
-                         double* scores, int32_t* best_pos, double* best_score) {
+                         double* scores, int32_t* best_pos, double* best_score, uint32_t* status) {
     if (B < 0 || R < 1 || C_cap < 0 || (dtype != ORC_F32 && dtype != ORC_BF16)) return 1;
     if (agg != ORC_AGG_MAX && agg != ORC_AGG_SUM) return 1;
     int rows = row_idx ? n_sel : R;
     if (rows < 1) return 1;
+    int bad_rows = 0;
     for (int k = 0; k < rows; ++k) {
         int r = row_idx ? row_idx[k] : k;
-        if (r < 0 || r >= R) return 1;
+        if (r < 0 || r >= R) bad_rows = 1;      /* such rows are left out of the aggregate */
     }
     for (int b = 0; b < B; ++b) {
+        if (seq_len[b] < 0 || seq_len[b] > T_cap) {         /* sequence skipped */
+            if (status) status[b] |= ORC_ST_SEQ_LEN;
+            best_pos[b] = -1;
+            if (best_score) best_score[b] = -INFINITY;
+            continue;
+        }
+        if (bad_rows && status) status[b] |= ORC_ST_ROW_INDEX;
         int64_t t = (int64_t)seq_len[b] - 1;
         int64_t n = cand_count[b] < 0 ? 0 : cand_count[b];
         if (n > C_cap) n = C_cap;
@@ -207,6 +224,7 @@ int pldpo_rank_attention(const void* A, int dtype, int R, int64_t row_stride, in
                 s = (agg == ORC_AGG_MAX) ? -INFINITY : 0.0;
                 for (int k = 0; k < rows; ++k) {
                     int r = row_idx ? row_idx[k] : k;
+                    if (r < 0 || r >= R) continue;
                     double a = orc_load(A, dtype, (int64_t)b * seq_stride + (int64_t)r * row_stride + j);
                     if (agg == ORC_AGG_MAX) { if (a > s) s = a; }
                     else s += a;
@@ -227,17 +245,17 @@ int pldpo_rank_attention(const void* A, int dtype, int R, int64_t row_stride, in
  * Draft prediction (Sec. 4.3):  xhat_i = x_{j*+i}, i = 1..K.
  * READING: the span stops at the last token x_t, so the draft has
  * d = min(K, t - j*) tokens; the rest of draft[b, :] is -1.  No candidate
- * (j* < 0) gives d = 0.
+ * (j* < 0), j* outside [0, t) or a seq_len beyond T_cap gives d = 0.
  * ------------------------------------------------------------------------ */
 int pldpo_extract_draft(const int32_t* ids, int64_t ids_stride, const int32_t* seq_len,
-                        const int32_t* best_pos, int B, int K,
+                        int64_t T_cap, const int32_t* best_pos, int B, int K,
                         int32_t* draft, int32_t* draft_len) {
     if (B < 0 || K < 1) return 1;
     for (int b = 0; b < B; ++b) {
         int64_t t = (int64_t)seq_len[b] - 1;
         int64_t js = best_pos[b];
         int64_t d = 0;
-        if (js >= 0 && js < t) d = (t - js < K) ? (t - js) : K;
+        if (seq_len[b] <= T_cap && js >= 0 && js < t) d = (t - js < K) ? (t - js) : K;
         for (int64_t i = 0; i < K; ++i)
             draft[(int64_t)b * K + i] = (i < d) ? ids[(int64_t)b * ids_stride + js + 1 + i] : -1;
         draft_len[b] = (int32_t)d;

@@ -1,0 +1,251 @@
+"""PLD+ drafting and greedy verification on GB300 (sm_103a).
+
+Python binding of the C ABI in ``include/pldp.h``.  Every function here only
+marshals torch tensors (device pointers, sizes, the current CUDA stream) into
+the library call of the same name; all the work runs in the CUDA kernels of
+``libpldp.so``.  There is no CPU fallback: if the library is missing the calls
+raise.
+
+PLD+ (arXiv 2412.01447), per decode step and per sequence:
+  * ``pldp_find_candidates`` -- Eq. 1 (Sec. 4.2): earlier occurrences of the last
+    token, narrowed to the longest matching suffix n-gram;
+  * ``pldp_rank_hidden``     -- Eq. 3 (Sec. 4.2.2): cosine of hidden states;
+  * ``pldp_rank_attention``  -- Eq. 2 (Sec. 4.2.1): max attention of selected heads;
+  * ``pldp_extract_draft``   -- Sec. 4.3: the K tokens after the best occurrence;
+  * ``pldp_verify_greedy``   -- Sec. 4.4: greedy accept against the target argmax.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+from . import _build
+
+__all__ = [
+    "build", "library_path", "PldpError",
+    "PLDP_F32", "PLDP_BF16", "PLDP_AGG_MAX", "PLDP_AGG_SUM",
+    "PLDP_ST_CAND_OVERFLOW", "PLDP_ST_TOKEN_RANGE", "PLDP_ST_CAPACITY", "PLDP_ST_SEQ_LEN",
+    "PLDP_ST_DRAFT_LEN", "PLDP_ST_ROW_INDEX", "PLDP_ST_TIMEOUT",
+    "pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention", "pldp_extract_draft",
+    "pldp_verify_greedy", "pldp_verify_workspace_size", "pldp_version", "pldp_last_error",
+]
+
+PLDP_F32, PLDP_BF16 = 0, 1
+PLDP_AGG_MAX, PLDP_AGG_SUM = 0, 1
+PLDP_ST_CAND_OVERFLOW = 1
+PLDP_ST_TOKEN_RANGE = 2
+PLDP_ST_CAPACITY = 4
+PLDP_ST_SEQ_LEN = 8
+PLDP_ST_DRAFT_LEN = 16
+PLDP_ST_ROW_INDEX = 32
+PLDP_ST_TIMEOUT = 64
+
+_STATUS_NAMES = {1: "PLDP_ERR_INVALID_ARG", 2: "PLDP_ERR_UNSUPPORTED", 3: "PLDP_ERR_CUDA",
+                 4: "PLDP_ERR_TIMEOUT"}
+
+
+class PldpError(RuntimeError):
+    def __init__(self, fn, code, msg):
+        super().__init__(f"{fn}: {_STATUS_NAMES.get(code, code)}: {msg}")
+        self.code = code
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def build(force: bool = False) -> str:
+    """Compile libpldp.so for sm_103a (in-tree) if it is missing or stale."""
+    return _build.build(force=force)
+
+
+def _load():
+    global _lib
+    if _lib is not None:
+        return _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(_build.LIB):
+                raise RuntimeError("libpldp.so is not built: call paper_2412_01447_gb300.build() "
+                                   "(needs nvcc); there is no CPU fallback")
+            lib = ctypes.CDLL(_build.LIB)
+            P, i32, i64, f32, sz = (ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float,
+                                    ctypes.c_size_t)
+            lib.pldp_find_candidates.argtypes = [P, i64, P, i32, i64, i32, i32, P, i32, P, P, P, P]
+            lib.pldp_rank_hidden.argtypes = [P, i32, i64, i64, P, i32, i64, P, P, i32, f32, P, P, P,
+                                             P, P]
+            lib.pldp_rank_attention.argtypes = [P, i32, i32, i64, i64, P, i32, i32, P, i32, i64, P,
+                                                P, i32, P, P, P, P, P]
+            lib.pldp_extract_draft.argtypes = [P, i64, P, i64, P, i32, i32, P, P, P]
+            lib.pldp_verify_greedy.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64, P, i64,
+                                               P, P, P, sz, P]
+            for f in ("pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention",
+                      "pldp_extract_draft", "pldp_verify_greedy"):
+                getattr(lib, f).restype = ctypes.c_int
+            lib.pldp_verify_workspace_size.argtypes = [i32, i32, i32]
+            lib.pldp_verify_workspace_size.restype = sz
+            lib.pldp_last_error.argtypes = []
+            lib.pldp_last_error.restype = ctypes.c_char_p
+            lib.pldp_version.argtypes = []
+            lib.pldp_version.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+# ----------------------------------------------------------------------------
+# marshalling helpers
+# ----------------------------------------------------------------------------
+def _stream(stream):
+    if stream is None:
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _dev(t, name, dtype=None, allow_none=False):
+    if t is None:
+        if allow_none:
+            return None
+        raise ValueError(f"{name} is required")
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}, got {t.dtype}")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _dense(t, name, dtype=None, allow_none=False):
+    if t is not None and not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return _dev(t, name, dtype, allow_none)
+
+
+def _rows(t, name):
+    """A [B, T] int32 tensor whose rows may be strided (unit inner stride)."""
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError(f"{name} must be 2-D with unit inner stride")
+    return _dev(t, name, torch.int32), t.stride(0), t.shape[1]
+
+
+def _code(x):
+    if x in (torch.float32, "f32", PLDP_F32):
+        return PLDP_F32
+    if x in (torch.bfloat16, "bf16", PLDP_BF16):
+        return PLDP_BF16
+    raise ValueError(f"unsupported dtype {x}")
+
+
+def _check(fn, rc):
+    if rc != 0:
+        raise PldpError(fn, rc, _load().pldp_last_error().decode())
+
+
+# ----------------------------------------------------------------------------
+# the C ABI, one call each
+# ----------------------------------------------------------------------------
+def pldp_find_candidates(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len,
+                         status=None, T_cap=None, stream=None):
+    """Eq. 1 with the longest-suffix n-gram rule.  ids: int32 [B, T] (rows may be
+    strided), seq_len int32 [B]; outputs cand_pos int32 [B, C_cap], cand_count and
+    match_len int32 [B], status uint32-as-int32 [B] (optional)."""
+    p_ids, stride, T = _rows(ids, "ids")
+    B = ids.shape[0]
+    C_cap = cand_pos.shape[1] if cand_pos is not None and cand_pos.dim() == 2 else 0
+    _check("pldp_find_candidates", _load().pldp_find_candidates(
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32), B, T if T_cap is None else T_cap,
+        ngram_min, ngram_max, _dense(cand_pos, "cand_pos", torch.int32, allow_none=True), C_cap,
+        _dense(cand_count, "cand_count", torch.int32), _dense(match_len, "match_len", torch.int32),
+        _dense(status, "status", None, allow_none=True), _stream(stream)))
+
+
+def pldp_rank_hidden(H, seq_len, cand_pos, cand_count, best_pos, scores=None, best_score=None,
+                     threshold=float("-inf"), status=None, stream=None):
+    """Eq. 3.  H: [B, T_cap, d] float32/bfloat16 (the chosen layer), contiguous rows;
+    cand_pos int32 [B, C_cap]; outputs best_pos int32 [B], scores float32 [B, C_cap]
+    and best_score float32 [B] (optional)."""
+    if H.dim() != 3 or H.stride(2) != 1 or H.stride(1) != H.shape[2]:
+        raise ValueError("H must be [B, T_cap, d] with contiguous rows")
+    B, T_cap, d = H.shape
+    C_cap = cand_pos.shape[1]
+    _check("pldp_rank_hidden", _load().pldp_rank_hidden(
+        _dev(H, "H"), _code(H.dtype), d, H.stride(0), _dense(seq_len, "seq_len", torch.int32), B,
+        T_cap, _dense(cand_pos, "cand_pos", torch.int32), _dense(cand_count, "cand_count", torch.int32),
+        C_cap, float(threshold), _dense(scores, "scores", torch.float32, allow_none=True),
+        _dense(best_pos, "best_pos", torch.int32),
+        _dense(best_score, "best_score", torch.float32, allow_none=True),
+        _dense(status, "status", None, allow_none=True), _stream(stream)))
+
+
+def pldp_rank_attention(A, seq_len, cand_pos, cand_count, best_pos, row_idx=None, agg=PLDP_AGG_MAX,
+                        scores=None, best_score=None, status=None, stream=None):
+    """Eq. 2.  A: [B, R, T_cap] float32/bfloat16, attention of query t-1 for each of R
+    (layer, head) rows (unit inner stride); row_idx int32 [n_sel] device or None (all)."""
+    if A.dim() != 3 or A.stride(2) != 1:
+        raise ValueError("A must be [B, R, T_cap] with unit inner stride")
+    B, R, T_cap = A.shape
+    C_cap = cand_pos.shape[1]
+    n_sel = R if row_idx is None else row_idx.numel()
+    _check("pldp_rank_attention", _load().pldp_rank_attention(
+        _dev(A, "A"), _code(A.dtype), R, A.stride(1), A.stride(0),
+        _dense(row_idx, "row_idx", torch.int32, allow_none=True), n_sel, int(agg),
+        _dense(seq_len, "seq_len", torch.int32), B, T_cap, _dense(cand_pos, "cand_pos", torch.int32),
+        _dense(cand_count, "cand_count", torch.int32), C_cap,
+        _dense(scores, "scores", torch.float32, allow_none=True),
+        _dense(best_pos, "best_pos", torch.int32),
+        _dense(best_score, "best_score", torch.float32, allow_none=True),
+        _dense(status, "status", None, allow_none=True), _stream(stream)))
+
+
+def pldp_extract_draft(ids, seq_len, best_pos, draft, draft_len, T_cap=None, stream=None):
+    """Sec. 4.3.  draft int32 [B, K] and draft_len int32 [B] are written."""
+    p_ids, stride, T = _rows(ids, "ids")
+    B, K = draft.shape
+    _check("pldp_extract_draft", _load().pldp_extract_draft(
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32), T if T_cap is None else T_cap,
+        _dense(best_pos, "best_pos", torch.int32), B, K, _dense(draft, "draft", torch.int32),
+        _dense(draft_len, "draft_len", torch.int32), _stream(stream)))
+
+
+def pldp_verify_workspace_size(B, K, V) -> int:
+    return int(_load().pldp_verify_workspace_size(B, K, V))
+
+
+def pldp_verify_greedy(logits, draft, draft_len, accept_len, next_token, workspace, argmax=None,
+                       ids=None, seq_len=None, kv_keep_len=None, status=None, T_cap=None,
+                       stream=None):
+    """Sec. 4.4 (greedy).  logits [B, K+1, V] float32/bfloat16 contiguous; workspace a
+    uint8 CUDA tensor of pldp_verify_workspace_size(B, K, V) bytes, zeroed once before
+    first use (every call leaves it zeroed).  ids/seq_len (optional, modified in place)
+    get the accepted tokens and the bonus token appended."""
+    B, K1, V = logits.shape
+    K = K1 - 1
+    if draft.shape != (B, K):
+        raise ValueError("draft must be [B, K] with K = logits.shape[1] - 1")
+    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids")
+    if T_cap is None:
+        T_cap = T
+    _check("pldp_verify_greedy", _load().pldp_verify_greedy(
+        _dense(logits, "logits"), _code(logits.dtype), B, K, V, _dense(draft, "draft", torch.int32),
+        _dense(draft_len, "draft_len", torch.int32),
+        _dense(argmax, "argmax", torch.int32, allow_none=True),
+        _dense(accept_len, "accept_len", torch.int32), _dense(next_token, "next_token", torch.int32),
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True), T_cap,
+        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True),
+        _dense(status, "status", None, allow_none=True), _dense(workspace, "workspace"),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def pldp_version() -> int:
+    return int(_load().pldp_version())
+
+
+def pldp_last_error() -> str:
+    return _load().pldp_last_error().decode()

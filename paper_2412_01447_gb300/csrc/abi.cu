@@ -1,0 +1,41 @@
+// Error reporting, version and device queries of the C ABI.
+#include <cstdarg>
+#include <cstdio>
+
+#include "pldp_internal.cuh"
+
+namespace pldp {
+
+static thread_local char g_last_error[512] = "";
+
+pldp_status fail(pldp_status code, const char* fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+pldp_status check_launch(const char* what) {
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
+    return PLDP_OK;
+}
+
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
+    return n > 0 ? n : 1;
+}
+
+}  // namespace pldp
+
+extern "C" {
+
+PLDP_API const char* pldp_last_error(void) { return pldp::g_last_error; }
+
+PLDP_API int pldp_version(void) { return 100; }  // 0.1.0
+
+}  // extern "C"

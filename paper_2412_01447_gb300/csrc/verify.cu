@@ -1,0 +1,345 @@
+// Draft prediction (Sec. 4.3) and greedy verification (Sec. 4.4) of PLD+.
+//
+// Verification is one streaming pass over the logits [B, K+1, V].  The
+// flattened logits are cut into equal contiguous ranges, one per warp, sized so
+// that the grid fills every SM once (a persistent split: no tail wave, and
+// each warp's range crosses at most a couple of row boundaries).  A warp keeps
+// a running (max, first index) per lane with 16-byte streaming loads, using a
+// packed max over each vector so that the index search runs only when the
+// running max grows.  Per row, the warps' results meet in a packed 64-bit key
+// (value, inverted index) combined with atomicMax in the workspace, which makes
+// the argmax exact and independent of scheduling: larger value wins, the
+// smaller index wins ties, -0.0 equals +0.0.
+//
+// Every warp that touched sequence b then takes a ticket; the warp holding the
+// last ticket (there is no waiting: the others just leave) reads the K+1 row
+// keys, finds the accepted length and the bonus token, appends them to the
+// context and returns the keys and the ticket to zero for the next call.
+#include <math.h>
+
+#include "pldp_internal.cuh"
+
+namespace pldp {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kUnroll = 8;                  // 16-byte loads in flight per lane
+constexpr int kWarpsPerSm = 32;             // 4 CTAs of 8 warps per SM
+constexpr int64_t kMinChunk = 2048;         // elements per warp, at least
+constexpr int64_t kAlign = 8;               // range boundaries are multiples of 8 elements
+
+__global__ void extract_draft_kernel(const int32_t* __restrict__ ids, int64_t ids_stride,
+                                     const int32_t* __restrict__ seq_len, int64_t T_cap,
+                                     const int32_t* __restrict__ best_pos, int B, int K,
+                                     int32_t* __restrict__ draft, int32_t* __restrict__ draft_len) {
+    const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+    if (idx >= static_cast<int64_t>(B) * K) return;
+    const int b = static_cast<int>(idx / K);
+    const int i = static_cast<int>(idx - static_cast<int64_t>(b) * K);
+    const int64_t L = seq_len[b];
+    const int64_t js = best_pos[b];
+    const int64_t t = L - 1;
+    int64_t d = 0;
+    if (L >= 0 && L <= T_cap && js >= 0 && js < t) d = (t - js < K) ? (t - js) : K;
+    draft[idx] = (i < d) ? ids[static_cast<int64_t>(b) * ids_stride + js + 1 + i] : -1;
+    if (i == 0) draft_len[b] = static_cast<int32_t>(d);
+}
+
+// ---- per-vector max and first index of the max ---------------------------------
+__device__ __forceinline__ float vmax(const uint4& x, __nv_bfloat16) {
+    const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&x.x);
+    const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&x.y);
+    const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&x.z);
+    const __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&x.w);
+    const __nv_bfloat162 m = __hmax2(__hmax2(a, b), __hmax2(c, d));
+    return fmaxf(__low2float(m), __high2float(m));
+}
+__device__ __forceinline__ int vfirst(const uint4& x, float m, __nv_bfloat16) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        if (__uint_as_float(w[k] << 16) == m) return 2 * k;
+        if (__uint_as_float(w[k] & 0xFFFF0000u) == m) return 2 * k + 1;
+    }
+    return 0;
+}
+__device__ __forceinline__ float vmax(const uint4& x, float) {
+    return fmaxf(fmaxf(__uint_as_float(x.x), __uint_as_float(x.y)),
+                 fmaxf(__uint_as_float(x.z), __uint_as_float(x.w)));
+}
+__device__ __forceinline__ int vfirst(const uint4& x, float m, float) {
+    if (__uint_as_float(x.x) == m) return 0;
+    if (__uint_as_float(x.y) == m) return 1;
+    if (__uint_as_float(x.z) == m) return 2;
+    return 3;
+}
+
+// Running (max, first index) of one lane over elements [c0, c1) of a row.
+template <typename T, bool VEC>
+__device__ __forceinline__ void lane_argmax(const T* __restrict__ row, int64_t c0, int64_t c1,
+                                            int lane, float& bv, int64_t& bi) {
+    if constexpr (VEC) {
+        constexpr int VW = 16 / sizeof(T);
+        const uint4* p = reinterpret_cast<const uint4*>(row);
+        const int64_t v0 = c0 / VW, v1 = c1 / VW;
+        for (int64_t vb = v0 + lane; vb < v1; vb += 32 * kUnroll) {
+            uint4 x[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int64_t v = vb + 32 * u;
+                if (v < v1) x[u] = ld_stream16(p + v);
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int64_t v = vb + 32 * u;
+                if (v < v1) {
+                    const float m = vmax(x[u], T());
+                    if (m > bv) {
+                        bv = m;
+                        bi = v * VW + vfirst(x[u], m, T());
+                    }
+                }
+            }
+        }
+    } else {
+        for (int64_t cb = c0 + lane; cb < c1; cb += 32 * kUnroll) {
+            float x[kUnroll];
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                const int64_t c = cb + 32 * u;
+                x[u] = (c < c1) ? to_f32(row[c]) : -INFINITY;
+            }
+#pragma unroll
+            for (int u = 0; u < kUnroll; ++u) {
+                if (x[u] > bv) {
+                    bv = x[u];
+                    bi = cb + 32 * u;
+                }
+            }
+        }
+    }
+}
+
+struct VerifyArgs {
+    const int32_t* draft;
+    const int32_t* draft_len;
+    int32_t* argmax;
+    int32_t* accept_len;
+    int32_t* next_token;
+    int32_t* ids;
+    int64_t ids_stride;
+    int32_t* seq_len;
+    int64_t T_cap;
+    int32_t* kv_keep_len;
+    uint32_t* status;
+    unsigned long long* row_keys;   // [B*(K+1)], zero between calls
+    unsigned int* tickets;          // [B], zero between calls
+    int B, K, V;
+    int64_t chunk;                  // elements per warp
+    int64_t total_warps;
+};
+
+// Accept/bonus/append for sequence b, by the warp that holds its last ticket.
+__device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
+    const int K1 = a.K + 1;
+    unsigned long long* keys = a.row_keys + b * K1;
+    uint32_t st = 0;
+    int d = a.draft_len[b];
+    if (d < 0 || d > a.K) {
+        st |= PLDP_ST_DRAFT_LEN;
+        d = d < 0 ? 0 : a.K;
+    }
+    int n = d;
+    bool range_bad = false;
+    for (int i0 = 0; i0 < K1; i0 += 32) {
+        const int i = i0 + lane;
+        int am = 0;
+        if (i < K1) {
+            am = static_cast<int>(key_index(__ldcg(keys + i)));
+            if (a.argmax) a.argmax[b * K1 + i] = am;
+        }
+        const bool in_draft = i < d;
+        const int tok = in_draft ? a.draft[b * a.K + i] : 0;
+        range_bad |= in_draft && (tok < 0 || tok >= a.V);
+        const unsigned mism = __ballot_sync(0xFFFFFFFFu, in_draft && tok != am);
+        if (n == d && mism) n = i0 + __ffs(mism) - 1;
+    }
+    if (__any_sync(0xFFFFFFFFu, range_bad)) st |= PLDP_ST_TOKEN_RANGE;
+    const int bonus = static_cast<int>(key_index(__ldcg(keys + n)));
+    __syncwarp();
+    for (int i = lane; i < K1; i += 32) keys[i] = 0ull;
+
+    if (lane == 0) {
+        a.accept_len[b] = n;
+        a.next_token[b] = bonus;
+    }
+    if (a.seq_len) {
+        const int64_t L = a.seq_len[b];
+        int64_t kv = -1;
+        if (L < 1 || L > a.T_cap) {
+            st |= PLDP_ST_SEQ_LEN;
+        } else {
+            kv = L + n;
+            if (L + n + 1 > a.T_cap) {
+                st |= PLDP_ST_CAPACITY;
+            } else {
+                if (a.ids) {
+                    int32_t* row = a.ids + b * a.ids_stride + L;
+                    for (int i = lane; i < n; i += 32) row[i] = a.draft[b * a.K + i];
+                    if (lane == 0) row[n] = bonus;
+                }
+                __syncwarp();
+                if (lane == 0) a.seq_len[b] = static_cast<int32_t>(L + n + 1);
+            }
+        }
+        if (a.kv_keep_len && lane == 0) a.kv_keep_len[b] = static_cast<int32_t>(kv);
+    }
+    if (lane == 0) {
+        if (a.status && st) a.status[b] |= st;
+        a.tickets[b] = 0u;
+    }
+}
+
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads)
+verify_greedy_kernel(const T* __restrict__ logits, VerifyArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+    if (w >= a.total_warps) return;
+    const int64_t V = a.V;
+    const int64_t E = static_cast<int64_t>(a.K + 1) * V;        // elements per sequence
+    const int64_t N = E * a.B;
+    const int64_t lo = w * a.chunk;
+    const int64_t hi = lo + a.chunk < N ? lo + a.chunk : N;
+
+    for (int64_t pos = lo; pos < hi;) {
+        const int64_t r = pos / V;
+        const int64_t c0 = pos - r * V;
+        const int64_t c1 = (V < c0 + (hi - pos)) ? V : c0 + (hi - pos);
+        float bv = -INFINITY;
+        int64_t bi = c0;
+        lane_argmax<T, VEC>(logits + r * V, c0, c1, lane, bv, bi);
+        const unsigned long long k = warp_max_u64(pack_key(bv, static_cast<uint32_t>(bi)));
+        if (lane == 0) atomicMax(a.row_keys + r, k);
+        pos += c1 - c0;
+    }
+
+    const int64_t b0 = lo / E, b1 = (hi - 1) / E;
+    for (int64_t b = b0; b <= b1; ++b) {
+        int last = 0;
+        if (lane == 0) {
+            __threadfence();   // this warp's row keys are visible before its ticket
+            const int64_t first_w = (b * E) / a.chunk;
+            const int64_t last_w = ((b + 1) * E - 1) / a.chunk;
+            const unsigned expected = static_cast<unsigned>(last_w - first_w + 1);
+            last = (atomicAdd(a.tickets + b, 1u) == expected - 1u);
+        }
+        last = __shfl_sync(0xFFFFFFFFu, last, 0);
+        if (last) {
+            __threadfence();
+            finish_sequence(a, b, lane);
+        }
+    }
+}
+
+size_t keys_bytes(int B, int K) {
+    return (static_cast<size_t>(B) * (K + 1) * sizeof(unsigned long long) + 255) / 256 * 256;
+}
+
+}  // namespace
+}  // namespace pldp
+
+using namespace pldp;
+
+extern "C" PLDP_API size_t pldp_verify_workspace_size(int B, int K, int V) {
+    if (B < 0 || K < 1 || V < 1) return 0;
+    return keys_bytes(B, K) + (static_cast<size_t>(B) * sizeof(unsigned int) + 255) / 256 * 256;
+}
+
+extern "C" PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
+                                                   const int32_t* seq_len, int64_t T_cap,
+                                                   const int32_t* best_pos, int B, int K,
+                                                   int32_t* draft, int32_t* draft_len,
+                                                   void* stream) {
+    if (B < 0) return fail(PLDP_ERR_INVALID_ARG, "extract_draft: B < 0");
+    if (K < 1) return fail(PLDP_ERR_INVALID_ARG, "extract_draft: K < 1");
+    if (T_cap < 0 || T_cap > INT32_MAX) return fail(PLDP_ERR_INVALID_ARG, "extract_draft: bad T_cap");
+    if (ids_stride < T_cap) return fail(PLDP_ERR_INVALID_ARG, "extract_draft: ids_stride < T_cap");
+    if (B == 0) return PLDP_OK;
+    if (!ids || !seq_len || !best_pos || !draft || !draft_len)
+        return fail(PLDP_ERR_INVALID_ARG, "extract_draft: null pointer");
+    const int64_t n = static_cast<int64_t>(B) * K;
+    const int64_t blocks = (n + 255) / 256;
+    if (blocks > INT32_MAX) return fail(PLDP_ERR_INVALID_ARG, "extract_draft: B*K too large");
+    extract_draft_kernel<<<static_cast<unsigned>(blocks), 256, 0, static_cast<cudaStream_t>(stream)>>>(
+        ids, ids_stride, seq_len, T_cap, best_pos, B, K, draft, draft_len);
+    return check_launch("extract_draft");
+}
+
+extern "C" PLDP_API pldp_status pldp_verify_greedy(
+    const void* logits, pldp_dtype dtype, int B, int K, int V, const int32_t* draft,
+    const int32_t* draft_len, int32_t* argmax, int32_t* accept_len, int32_t* next_token,
+    int32_t* ids, int64_t ids_stride, int32_t* seq_len, int64_t T_cap, int32_t* kv_keep_len,
+    uint32_t* status, void* workspace, size_t workspace_bytes, void* stream) {
+    if (B < 0) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: B < 0");
+    if (K < 1) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: K < 1");
+    if (V < 1) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: V < 1");
+    if (dtype != PLDP_F32 && dtype != PLDP_BF16)
+        return fail(PLDP_ERR_UNSUPPORTED, "verify_greedy: unsupported dtype %d", (int)dtype);
+    if ((ids || kv_keep_len) && !seq_len)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: ids/kv_keep_len need seq_len");
+    if (seq_len && (T_cap < 0 || T_cap > INT32_MAX))
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: bad T_cap");
+    if (ids && ids_stride < T_cap) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: ids_stride < T_cap");
+    if (B == 0) return PLDP_OK;
+    if (!logits || !draft || !draft_len || !accept_len || !next_token)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: null pointer");
+    const size_t need = pldp_verify_workspace_size(B, K, V);
+    if (!workspace || workspace_bytes < need)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: workspace needs %zu bytes", need);
+    if (!aligned16(workspace)) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: workspace not 16-byte aligned");
+
+    const size_t es = dtype == PLDP_F32 ? 4 : 2;
+    const int64_t N = static_cast<int64_t>(B) * (K + 1) * V;
+    const bool vec = aligned16(logits) && (static_cast<size_t>(V) * es) % 16 == 0;
+    const int64_t target = static_cast<int64_t>(sm_count()) * kWarpsPerSm;
+    int64_t chunk = (N + target - 1) / target;
+    if (chunk < kMinChunk) chunk = kMinChunk;
+    chunk = (chunk + kAlign - 1) / kAlign * kAlign;
+    const int64_t warps = (N + chunk - 1) / chunk;
+    const int64_t blocks = (warps + kWarps - 1) / kWarps;
+
+    VerifyArgs a;
+    a.draft = draft;
+    a.draft_len = draft_len;
+    a.argmax = argmax;
+    a.accept_len = accept_len;
+    a.next_token = next_token;
+    a.ids = ids;
+    a.ids_stride = ids_stride;
+    a.seq_len = seq_len;
+    a.T_cap = T_cap;
+    a.kv_keep_len = kv_keep_len;
+    a.status = status;
+    a.row_keys = static_cast<unsigned long long*>(workspace);
+    a.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + keys_bytes(B, K));
+    a.B = B;
+    a.K = K;
+    a.V = V;
+    a.chunk = chunk;
+    a.total_warps = warps;
+
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const unsigned g = static_cast<unsigned>(blocks);
+    if (dtype == PLDP_BF16) {
+        const __nv_bfloat16* l = static_cast<const __nv_bfloat16*>(logits);
+        if (vec) verify_greedy_kernel<__nv_bfloat16, true><<<g, kThreads, 0, s>>>(l, a);
+        else verify_greedy_kernel<__nv_bfloat16, false><<<g, kThreads, 0, s>>>(l, a);
+    } else {
+        const float* l = static_cast<const float*>(logits);
+        if (vec) verify_greedy_kernel<float, true><<<g, kThreads, 0, s>>>(l, a);
+        else verify_greedy_kernel<float, false><<<g, kThreads, 0, s>>>(l, a);
+    }
+    return check_launch("verify_greedy");
+}

@@ -1,0 +1,99 @@
+"""The C ABI library loads without a GPU and exports every call include/pldp.h
+declares; host-side argument checks fail before anything touches CUDA."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2412_01447_gb300 as pk
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "pldp.h")
+
+
+def declared_symbols():
+    src = open(HEADER).read()
+    return sorted(set(re.findall(r"PLDP_API\s+[\w\s\*]+?\b(pldp_\w+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def so():
+    pk.build()
+    return ctypes.CDLL(pk.library_path())
+
+
+def test_header_declares_the_five_steps():
+    names = declared_symbols()
+    for n in ("pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention",
+              "pldp_extract_draft", "pldp_verify_greedy"):
+        assert n in names
+
+
+def test_exports_every_declared_symbol(so):
+    for name in declared_symbols():
+        assert hasattr(so, name), name
+
+
+def test_no_stray_exports(so):
+    out = os.popen(f"nm -D --defined-only {pk.library_path()}").read()
+    exported = sorted(set(re.findall(r"\b(pldp_\w+)\b", out)))
+    assert exported == declared_symbols()
+
+
+def test_version_and_workspace_are_host_only():
+    assert pk.pldp_version() == 100
+    assert pk.pldp_verify_workspace_size(0, 1, 1) == 0 + 0
+    n = pk.pldp_verify_workspace_size(128, 12, 128256)
+    assert n >= 128 * 13 * 8 + 128 * 4 and n % 256 == 0
+    assert pk.pldp_verify_workspace_size(4, 0, 10) == 0
+
+
+def test_host_argument_checks(so):
+    lib = pk._load()
+    null = None
+    # find_candidates: B < 0, bad n-gram range, stride < T_cap
+    assert lib.pldp_find_candidates(null, 8, null, -1, 8, 1, 3, null, 4, null, null, null, null) == 1
+    assert lib.pldp_find_candidates(null, 8, null, 1, 8, 2, 1, null, 4, null, null, null, null) == 1
+    assert lib.pldp_find_candidates(null, 8, null, 1, 8, 1, 9, null, 4, null, null, null, null) == 1
+    assert lib.pldp_find_candidates(null, 4, null, 1, 8, 1, 3, null, 4, null, null, null, null) == 1
+    assert "ids_stride" in pk.pldp_last_error()
+    assert lib.pldp_find_candidates(null, 8, null, 1, 8, 1, 3, null, 4, null, null, null, null) == 1
+    assert "null" in pk.pldp_last_error()
+    assert lib.pldp_find_candidates(null, 8, null, 0, 8, 1, 3, null, 4, null, null, null, null) == 0
+    # rank_hidden: unsupported dtype, d too large, NaN threshold
+    args = [null, 0, 64, 64 * 8, null, 1, 8, null, null, 4, float("-inf"), null, null, null, null, null]
+    bad = list(args); bad[1] = 7
+    assert lib.pldp_rank_hidden(*bad) == 2
+    bad = list(args); bad[2] = 1 << 20; bad[3] = (1 << 20) * 8
+    assert lib.pldp_rank_hidden(*bad) == 2
+    bad = list(args); bad[10] = float("nan")
+    assert lib.pldp_rank_hidden(*bad) == 1
+    # rank_attention: bad aggregation, n_sel out of range
+    a = [null, 1, 4, 8, 32, null, 4, 0, null, 1, 8, null, null, 4, null, null, null, null, null]
+    bad = list(a); bad[7] = 5
+    assert lib.pldp_rank_attention(*bad) == 1
+    bad = list(a); bad[5] = ctypes.c_void_p(16); bad[6] = 0
+    assert lib.pldp_rank_attention(*bad) == 1
+    # extract_draft: K < 1
+    assert lib.pldp_extract_draft(null, 8, null, 8, null, 1, 0, null, null, null) == 1
+    # verify_greedy: K < 1, ids without seq_len, workspace too small
+    v = [null, 1, 2, 4, 100, null, null, null, null, null, null, 0, null, 0, null, null, null, 0, null]
+    bad = list(v); bad[3] = 0
+    assert lib.pldp_verify_greedy(*bad) == 1
+    bad = list(v); bad[10] = ctypes.c_void_p(16)
+    assert lib.pldp_verify_greedy(*bad) == 1
+    bad = list(v)
+    for k in (0, 5, 6, 8, 9):
+        bad[k] = ctypes.c_void_p(256)
+    bad[16] = ctypes.c_void_p(256); bad[17] = 8
+    assert lib.pldp_verify_greedy(*bad) == 1
+    assert "workspace" in pk.pldp_last_error()
+
+
+def test_python_binding_refuses_cpu_tensors():
+    import torch
+    x = torch.zeros((2, 8), dtype=torch.int32)
+    with pytest.raises(ValueError):
+        pk.pldp_find_candidates(x, torch.zeros(2, dtype=torch.int32), 1, 3,
+                                torch.zeros((2, 4), dtype=torch.int32),
+                                torch.zeros(2, dtype=torch.int32), torch.zeros(2, dtype=torch.int32))
