@@ -20,7 +20,8 @@
  * Conventions shared by every call
  *  - Every pointer argument is a DEVICE pointer owned by the caller; the
  *    library allocates nothing and keeps no state between calls, except the
- *    caller-provided verification workspace described at pldp_verify_greedy.
+ *    caller-provided verification workspace described at pldp_verify_greedy
+ *    and the fixed scratch area of pldp_verify_greedy_noalloc.
  *  - All work is enqueued asynchronously on `stream` (a cudaStream_t; NULL is
  *    the legacy default stream).  No call synchronises the device or reads
  *    device memory on the host, so every call may be captured in a CUDA graph.
@@ -221,6 +222,39 @@ PLDP_API pldp_status pldp_verify_greedy(const void* logits, pldp_dtype dtype, in
                                         int32_t* seq_len, int64_t T_cap, int32_t* kv_keep_len,
                                         uint32_t* status, void* workspace,
                                         size_t workspace_bytes, void* stream);
+
+/*
+ * Greedy verification without a caller workspace.  The paper has no counterpart:
+ * this is a deployment convenience.  Same arguments, results and status bits as
+ * pldp_verify_greedy, minus the workspace.
+ *
+ * Who needs it: callers that cannot allocate device memory for a workspace --
+ * code embedded in a host program that owns every GPU allocation, and serving
+ * loops that must not call cudaMalloc/cudaFree after start-up because those
+ * calls can synchronise the whole device.
+ *
+ * The scratch lives in a fixed 1 MiB area compiled into the library; every GPU
+ * that loads the library keeps it until the process exits.  Requests needing
+ * more than that (pldp_verify_workspace_size(B, K, V) > 1048576, i.e. roughly
+ * B*(K+1) > 130000 rows) are rejected with PLDP_ERR_INVALID_ARG.  The call
+ * allocates nothing: it clears the part of the area it uses with
+ * cudaMemsetAsync on `stream`, then launches the kernel.
+ *
+ * The first call on each device looks up the area's device address (once per
+ * device, on the current device); make that first call before any stream
+ * capture.  All calls on a device share the one area, which keeps whatever the
+ * last call left there: calls that can overlap on the GPU (different streams,
+ * or threads without ordering between them) race on it and must be serialised
+ * by the caller.
+ */
+PLDP_API pldp_status pldp_verify_greedy_noalloc(const void* logits, pldp_dtype dtype, int B,
+                                                int K, int V, const int32_t* draft,
+                                                const int32_t* draft_len, int32_t* argmax,
+                                                int32_t* accept_len, int32_t* next_token,
+                                                int32_t* ids, int64_t ids_stride,
+                                                int32_t* seq_len, int64_t T_cap,
+                                                int32_t* kv_keep_len, uint32_t* status,
+                                                void* stream);
 
 /* Bytes of workspace pldp_verify_greedy needs for these sizes (0 if invalid). */
 PLDP_API size_t pldp_verify_workspace_size(int B, int K, int V);

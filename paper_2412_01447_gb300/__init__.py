@@ -30,7 +30,8 @@ __all__ = [
     "PLDP_ST_CAND_OVERFLOW", "PLDP_ST_TOKEN_RANGE", "PLDP_ST_CAPACITY", "PLDP_ST_SEQ_LEN",
     "PLDP_ST_DRAFT_LEN", "PLDP_ST_ROW_INDEX", "PLDP_ST_TIMEOUT",
     "pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention", "pldp_extract_draft",
-    "pldp_verify_greedy", "pldp_verify_workspace_size", "pldp_version", "pldp_last_error",
+    "pldp_verify_greedy", "pldp_verify_greedy_noalloc", "pldp_verify_workspace_size",
+    "pldp_version", "pldp_last_error",
 ]
 
 PLDP_F32, PLDP_BF16 = 0, 1
@@ -89,6 +90,9 @@ def _load():
             for f in ("pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention",
                       "pldp_extract_draft", "pldp_verify_greedy"):
                 getattr(lib, f).restype = ctypes.c_int
+            lib.pldp_verify_greedy_noalloc.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64,
+                                                       P, i64, P, P, P]
+            lib.pldp_verify_greedy_noalloc.restype = ctypes.c_int
             lib.pldp_verify_workspace_size.argtypes = [i32, i32, i32]
             lib.pldp_verify_workspace_size.restype = sz
             lib.pldp_last_error.argtypes = []
@@ -241,6 +245,29 @@ def pldp_verify_greedy(logits, draft, draft_len, accept_len, next_token, workspa
         _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True),
         _dense(status, "status", None, allow_none=True), _dense(workspace, "workspace"),
         workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def pldp_verify_greedy_noalloc(logits, draft, draft_len, accept_len, next_token, argmax=None,
+                               ids=None, seq_len=None, kv_keep_len=None, status=None, T_cap=None,
+                               stream=None):
+    """pldp_verify_greedy for callers that cannot allocate a workspace: the library
+    uses its own fixed scratch area (see include/pldp.h for the size limit and for
+    why overlapping calls on one device must be serialised)."""
+    B, K1, V = logits.shape
+    K = K1 - 1
+    if draft.shape != (B, K):
+        raise ValueError("draft must be [B, K] with K = logits.shape[1] - 1")
+    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids")
+    if T_cap is None:
+        T_cap = T
+    _check("pldp_verify_greedy_noalloc", _load().pldp_verify_greedy_noalloc(
+        _dense(logits, "logits"), _code(logits.dtype), B, K, V, _dense(draft, "draft", torch.int32),
+        _dense(draft_len, "draft_len", torch.int32),
+        _dense(argmax, "argmax", torch.int32, allow_none=True),
+        _dense(accept_len, "accept_len", torch.int32), _dense(next_token, "next_token", torch.int32),
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True), T_cap,
+        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True),
+        _dense(status, "status", None, allow_none=True), _stream(stream)))
 
 
 def pldp_version() -> int:

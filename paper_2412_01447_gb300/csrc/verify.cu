@@ -343,3 +343,133 @@ extern "C" PLDP_API pldp_status pldp_verify_greedy(
     }
     return check_launch("verify_greedy");
 }
+
+// ---------------------------------------------------------------------------
+// Allocation-free greedy verification.
+//
+// Some callers cannot hand the library a workspace: code that owns no device
+// allocator (a plugin living inside a host program that manages all GPU memory
+// itself), and serving loops that forbid cudaMalloc/cudaFree once they are up,
+// because those calls can synchronise the device and stall every stream.  For
+// them this entry point keeps its scratch in a fixed area compiled into the
+// library.  Every GPU that loads the library holds that area until the process
+// exits.
+// ---------------------------------------------------------------------------
+#include <mutex>
+
+namespace pldp {
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = size_t(1) << 20;   // 1 MiB: B*(K+1) up to ~130k rows
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_noalloc_mutex;
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+// Device address of g_noalloc_scratch on the current device, looked up once per
+// device.  In host code the array's name only stands in for the symbol; the
+// kernel must be given this address instead.
+pldp_status noalloc_scratch(void** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return fail(PLDP_ERR_CUDA, "verify_greedy_noalloc: cudaGetDevice: %s", cudaGetErrorString(e));
+    if (dev < 0 || dev >= kMaxDevices)
+        return fail(PLDP_ERR_UNSUPPORTED, "verify_greedy_noalloc: device %d beyond %d", dev, kMaxDevices);
+    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p)
+            return fail(PLDP_ERR_CUDA, "verify_greedy_noalloc: cudaGetSymbolAddress: %s",
+                        cudaGetErrorString(e));
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return PLDP_OK;
+}
+
+}  // namespace
+}  // namespace pldp
+
+extern "C" PLDP_API pldp_status pldp_verify_greedy_noalloc(
+    const void* logits, pldp_dtype dtype, int B, int K, int V, const int32_t* draft,
+    const int32_t* draft_len, int32_t* argmax, int32_t* accept_len, int32_t* next_token,
+    int32_t* ids, int64_t ids_stride, int32_t* seq_len, int64_t T_cap, int32_t* kv_keep_len,
+    uint32_t* status, void* stream) {
+    if (B < 0) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_noalloc: B < 0");
+    if (K < 1) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_noalloc: K < 1");
+    if (V < 1) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_noalloc: V < 1");
+    if (dtype != PLDP_F32 && dtype != PLDP_BF16)
+        return fail(PLDP_ERR_UNSUPPORTED, "verify_greedy_noalloc: unsupported dtype %d", (int)dtype);
+    if ((ids || kv_keep_len) && !seq_len)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_noalloc: ids/kv_keep_len need seq_len");
+    if (seq_len && (T_cap < 0 || T_cap > INT32_MAX))
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_noalloc: bad T_cap");
+    if (ids && ids_stride < T_cap)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_noalloc: ids_stride < T_cap");
+    const size_t need = pldp_verify_workspace_size(B, K, V);
+    if (need > kNoAllocScratchBytes)
+        return fail(PLDP_ERR_INVALID_ARG,
+                    "verify_greedy_noalloc: B=%d, K=%d needs %zu bytes of scratch; the built-in area "
+                    "holds %zu (use pldp_verify_greedy with a caller workspace)",
+                    B, K, need, kNoAllocScratchBytes);
+    if (B == 0) return PLDP_OK;
+    if (!logits || !draft || !draft_len || !accept_len || !next_token)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_noalloc: null pointer");
+
+    void* scratch = nullptr;
+    pldp_status ps = noalloc_scratch(&scratch);
+    if (ps != PLDP_OK) return ps;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // The kernel needs its row keys and tickets at zero.  Each call returns them to
+    // zero when it completes, but the area is shared and outlives every call, so it
+    // is cleared here as well (cudaMemsetAsync allocates nothing).
+    cudaError_t e = cudaMemsetAsync(scratch, 0, need, s);
+    if (e != cudaSuccess)
+        return fail(PLDP_ERR_CUDA, "verify_greedy_noalloc: clearing scratch: %s", cudaGetErrorString(e));
+
+    const size_t es = dtype == PLDP_F32 ? 4 : 2;
+    const int64_t N = static_cast<int64_t>(B) * (K + 1) * V;
+    const bool vec = aligned16(logits) && (static_cast<size_t>(V) * es) % 16 == 0;
+    const int64_t target = static_cast<int64_t>(sm_count()) * kWarpsPerSm;
+    int64_t chunk = (N + target - 1) / target;
+    if (chunk < kMinChunk) chunk = kMinChunk;
+    chunk = (chunk + kAlign - 1) / kAlign * kAlign;
+    const int64_t warps = (N + chunk - 1) / chunk;
+    const int64_t blocks = (warps + kWarps - 1) / kWarps;
+
+    VerifyArgs a;
+    a.draft = draft;
+    a.draft_len = draft_len;
+    a.argmax = argmax;
+    a.accept_len = accept_len;
+    a.next_token = next_token;
+    a.ids = ids;
+    a.ids_stride = ids_stride;
+    a.seq_len = seq_len;
+    a.T_cap = T_cap;
+    a.kv_keep_len = kv_keep_len;
+    a.status = status;
+    a.row_keys = static_cast<unsigned long long*>(scratch);
+    a.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(scratch) + keys_bytes(B, K));
+    a.B = B;
+    a.K = K;
+    a.V = V;
+    a.chunk = chunk;
+    a.total_warps = warps;
+
+    const unsigned g = static_cast<unsigned>(blocks);
+    if (dtype == PLDP_BF16) {
+        const __nv_bfloat16* l = static_cast<const __nv_bfloat16*>(logits);
+        if (vec) verify_greedy_kernel<__nv_bfloat16, true><<<g, kThreads, 0, s>>>(l, a);
+        else verify_greedy_kernel<__nv_bfloat16, false><<<g, kThreads, 0, s>>>(l, a);
+    } else {
+        const float* l = static_cast<const float*>(logits);
+        if (vec) verify_greedy_kernel<float, true><<<g, kThreads, 0, s>>>(l, a);
+        else verify_greedy_kernel<float, false><<<g, kThreads, 0, s>>>(l, a);
+    }
+    return check_launch("verify_greedy_noalloc");
+}
