@@ -1,6 +1,9 @@
 // Error reporting, version and device queries of the C ABI.
 #include <cstdarg>
 #include <cstdio>
+#include <map>
+#include <mutex>
+#include <tuple>
 
 #include "pldp_internal.cuh"
 
@@ -28,6 +31,27 @@ int sm_count() {
     if (cudaGetDevice(&dev) != cudaSuccess) return 1;
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 1;
     return n > 0 ? n : 1;
+}
+
+int resident_blocks(const void* kernel, int threads, size_t smem) {
+    static std::mutex mu;
+    static std::map<std::tuple<int, const void*, int, size_t>, int> cache;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return sm_count();
+    const auto key = std::make_tuple(dev, kernel, threads, smem);
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        auto it = cache.find(key);
+        if (it != cache.end()) return it->second;
+    }
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, smem) != cudaSuccess ||
+        per_sm < 1)
+        per_sm = 1;
+    const int n = per_sm * sm_count();
+    std::lock_guard<std::mutex> lock(mu);
+    cache[key] = n;
+    return n;
 }
 
 }  // namespace pldp

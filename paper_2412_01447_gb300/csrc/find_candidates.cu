@@ -260,7 +260,13 @@ extern "C" PLDP_API pldp_status pldp_find_candidates(const int32_t* ids, int64_t
         return fail(PLDP_ERR_INVALID_ARG, "find_candidates: null pointer");
 
     const bool vec = aligned16(ids) && ids_stride % 4 == 0 && T_cap % 4 == 0;
+    // One CTA per kPositionsPerCta positions, at most a portable cluster, and no
+    // more CTAs in all than fit on the device at once (a single wave).
     int CL = static_cast<int>((T_cap + kPositionsPerCta - 1) / kPositionsPerCta);
+    const void* fn = vec ? reinterpret_cast<const void*>(&find_candidates_kernel<true>)
+                         : reinterpret_cast<const void*>(&find_candidates_kernel<false>);
+    const int per_seq = resident_blocks(fn, kThreads, 0) / B;
+    if (CL > per_seq) CL = per_seq;
     CL = CL < 1 ? 1 : (CL > kMaxCluster ? kMaxCluster : CL);
     int64_t chunk = (T_cap + CL - 1) / CL;
     chunk = (chunk + 3) / 4 * 4;

@@ -18,6 +18,8 @@ namespace cg = cooperative_groups;
 pldp_status fail(pldp_status code, const char* fmt, ...);
 pldp_status check_launch(const char* what);
 int sm_count();  // SMs of the current device
+// CTAs of `kernel` that fit on the whole current device at once (cached).
+int resident_blocks(const void* kernel, int threads, size_t smem);
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 

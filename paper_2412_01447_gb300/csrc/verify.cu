@@ -25,7 +25,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kUnroll = 8;                  // 16-byte loads in flight per lane
-constexpr int kWarpsPerSm = 32;             // 4 CTAs of 8 warps per SM
+constexpr int kMinBlocksPerSm = 4;          // register cap: 4 CTAs of 8 warps per SM
 constexpr int64_t kMinChunk = 2048;         // elements per warp, at least
 constexpr int64_t kAlign = 8;               // range boundaries are multiples of 8 elements
 
@@ -202,7 +202,7 @@ __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
 }
 
 template <typename T, bool VEC>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, kMinBlocksPerSm)
 verify_greedy_kernel(const T* __restrict__ logits, VerifyArgs a) {
     const int lane = threadIdx.x & 31;
     const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
@@ -245,6 +245,60 @@ verify_greedy_kernel(const T* __restrict__ logits, VerifyArgs a) {
 
 size_t keys_bytes(int B, int K) {
     return (static_cast<size_t>(B) * (K + 1) * sizeof(unsigned long long) + 255) / 256 * 256;
+}
+
+// Splits the flattened logits into equal per-warp ranges for a grid that is
+// exactly the number of CTAs resident on the device at once (one wave), and
+// launches.  `a` has everything but the split and the scratch filled in.
+template <typename T, bool VEC>
+pldp_status launch_verify_t(const void* logits, VerifyArgs a, void* scratch, cudaStream_t s,
+                            const char* what) {
+    const void* fn = reinterpret_cast<const void*>(&verify_greedy_kernel<T, VEC>);
+    const int64_t N = static_cast<int64_t>(a.B) * (a.K + 1) * a.V;
+    const int64_t resident_warps = static_cast<int64_t>(resident_blocks(fn, kThreads, 0)) * kWarps;
+    int64_t chunk = (N + resident_warps - 1) / resident_warps;
+    if (chunk < kMinChunk) chunk = kMinChunk;
+    chunk = (chunk + kAlign - 1) / kAlign * kAlign;
+    a.chunk = chunk;
+    a.total_warps = (N + chunk - 1) / chunk;
+    a.row_keys = static_cast<unsigned long long*>(scratch);
+    a.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(scratch) + keys_bytes(a.B, a.K));
+    const unsigned blocks = static_cast<unsigned>((a.total_warps + kWarps - 1) / kWarps);
+    verify_greedy_kernel<T, VEC><<<blocks, kThreads, 0, s>>>(static_cast<const T*>(logits), a);
+    return check_launch(what);
+}
+
+pldp_status launch_verify(const void* logits, pldp_dtype dtype, const VerifyArgs& a, void* scratch,
+                          cudaStream_t s, const char* what) {
+    const size_t es = dtype == PLDP_F32 ? 4 : 2;
+    const bool vec = aligned16(logits) && (static_cast<size_t>(a.V) * es) % 16 == 0;
+    if (dtype == PLDP_BF16)
+        return vec ? launch_verify_t<__nv_bfloat16, true>(logits, a, scratch, s, what)
+                   : launch_verify_t<__nv_bfloat16, false>(logits, a, scratch, s, what);
+    return vec ? launch_verify_t<float, true>(logits, a, scratch, s, what)
+               : launch_verify_t<float, false>(logits, a, scratch, s, what);
+}
+
+VerifyArgs verify_args(int B, int K, int V, const int32_t* draft, const int32_t* draft_len,
+                       int32_t* argmax, int32_t* accept_len, int32_t* next_token, int32_t* ids,
+                       int64_t ids_stride, int32_t* seq_len, int64_t T_cap, int32_t* kv_keep_len,
+                       uint32_t* status) {
+    VerifyArgs a = {};
+    a.draft = draft;
+    a.draft_len = draft_len;
+    a.argmax = argmax;
+    a.accept_len = accept_len;
+    a.next_token = next_token;
+    a.ids = ids;
+    a.ids_stride = ids_stride;
+    a.seq_len = seq_len;
+    a.T_cap = T_cap;
+    a.kv_keep_len = kv_keep_len;
+    a.status = status;
+    a.B = B;
+    a.K = K;
+    a.V = V;
+    return a;
 }
 
 }  // namespace
@@ -300,48 +354,10 @@ extern "C" PLDP_API pldp_status pldp_verify_greedy(
         return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: workspace needs %zu bytes", need);
     if (!aligned16(workspace)) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy: workspace not 16-byte aligned");
 
-    const size_t es = dtype == PLDP_F32 ? 4 : 2;
-    const int64_t N = static_cast<int64_t>(B) * (K + 1) * V;
-    const bool vec = aligned16(logits) && (static_cast<size_t>(V) * es) % 16 == 0;
-    const int64_t target = static_cast<int64_t>(sm_count()) * kWarpsPerSm;
-    int64_t chunk = (N + target - 1) / target;
-    if (chunk < kMinChunk) chunk = kMinChunk;
-    chunk = (chunk + kAlign - 1) / kAlign * kAlign;
-    const int64_t warps = (N + chunk - 1) / chunk;
-    const int64_t blocks = (warps + kWarps - 1) / kWarps;
-
-    VerifyArgs a;
-    a.draft = draft;
-    a.draft_len = draft_len;
-    a.argmax = argmax;
-    a.accept_len = accept_len;
-    a.next_token = next_token;
-    a.ids = ids;
-    a.ids_stride = ids_stride;
-    a.seq_len = seq_len;
-    a.T_cap = T_cap;
-    a.kv_keep_len = kv_keep_len;
-    a.status = status;
-    a.row_keys = static_cast<unsigned long long*>(workspace);
-    a.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(workspace) + keys_bytes(B, K));
-    a.B = B;
-    a.K = K;
-    a.V = V;
-    a.chunk = chunk;
-    a.total_warps = warps;
-
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const unsigned g = static_cast<unsigned>(blocks);
-    if (dtype == PLDP_BF16) {
-        const __nv_bfloat16* l = static_cast<const __nv_bfloat16*>(logits);
-        if (vec) verify_greedy_kernel<__nv_bfloat16, true><<<g, kThreads, 0, s>>>(l, a);
-        else verify_greedy_kernel<__nv_bfloat16, false><<<g, kThreads, 0, s>>>(l, a);
-    } else {
-        const float* l = static_cast<const float*>(logits);
-        if (vec) verify_greedy_kernel<float, true><<<g, kThreads, 0, s>>>(l, a);
-        else verify_greedy_kernel<float, false><<<g, kThreads, 0, s>>>(l, a);
-    }
-    return check_launch("verify_greedy");
+    const VerifyArgs a = verify_args(B, K, V, draft, draft_len, argmax, accept_len, next_token, ids,
+                                     ids_stride, seq_len, T_cap, kv_keep_len, status);
+    return launch_verify(logits, dtype, a, workspace, static_cast<cudaStream_t>(stream),
+                         "verify_greedy");
 }
 
 // ---------------------------------------------------------------------------
@@ -431,45 +447,7 @@ extern "C" PLDP_API pldp_status pldp_verify_greedy_noalloc(
     if (e != cudaSuccess)
         return fail(PLDP_ERR_CUDA, "verify_greedy_noalloc: clearing scratch: %s", cudaGetErrorString(e));
 
-    const size_t es = dtype == PLDP_F32 ? 4 : 2;
-    const int64_t N = static_cast<int64_t>(B) * (K + 1) * V;
-    const bool vec = aligned16(logits) && (static_cast<size_t>(V) * es) % 16 == 0;
-    const int64_t target = static_cast<int64_t>(sm_count()) * kWarpsPerSm;
-    int64_t chunk = (N + target - 1) / target;
-    if (chunk < kMinChunk) chunk = kMinChunk;
-    chunk = (chunk + kAlign - 1) / kAlign * kAlign;
-    const int64_t warps = (N + chunk - 1) / chunk;
-    const int64_t blocks = (warps + kWarps - 1) / kWarps;
-
-    VerifyArgs a;
-    a.draft = draft;
-    a.draft_len = draft_len;
-    a.argmax = argmax;
-    a.accept_len = accept_len;
-    a.next_token = next_token;
-    a.ids = ids;
-    a.ids_stride = ids_stride;
-    a.seq_len = seq_len;
-    a.T_cap = T_cap;
-    a.kv_keep_len = kv_keep_len;
-    a.status = status;
-    a.row_keys = static_cast<unsigned long long*>(scratch);
-    a.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(scratch) + keys_bytes(B, K));
-    a.B = B;
-    a.K = K;
-    a.V = V;
-    a.chunk = chunk;
-    a.total_warps = warps;
-
-    const unsigned g = static_cast<unsigned>(blocks);
-    if (dtype == PLDP_BF16) {
-        const __nv_bfloat16* l = static_cast<const __nv_bfloat16*>(logits);
-        if (vec) verify_greedy_kernel<__nv_bfloat16, true><<<g, kThreads, 0, s>>>(l, a);
-        else verify_greedy_kernel<__nv_bfloat16, false><<<g, kThreads, 0, s>>>(l, a);
-    } else {
-        const float* l = static_cast<const float*>(logits);
-        if (vec) verify_greedy_kernel<float, true><<<g, kThreads, 0, s>>>(l, a);
-        else verify_greedy_kernel<float, false><<<g, kThreads, 0, s>>>(l, a);
-    }
-    return check_launch("verify_greedy_noalloc");
+    const VerifyArgs a = verify_args(B, K, V, draft, draft_len, argmax, accept_len, next_token, ids,
+                                     ids_stride, seq_len, T_cap, kv_keep_len, status);
+    return launch_verify(logits, dtype, a, scratch, s, "verify_greedy_noalloc");
 }
