@@ -53,9 +53,13 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="c5")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--separate", action="store_true",
+                    help="draft with the four separate calls instead of the fused launch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ref-seqs", type=int, default=2, help="sequences per oracle step (reference arm)")
     ap.add_argument("--batch", type=int, default=None, help="override the batch (not the headline)")
+    ap.add_argument("--hidden-width", type=int, default=None,
+                    help="override the hidden width d (not the headline; keeps profiles small)")
     ap.add_argument("--context", type=int, default=None,
                     help="override the initial context, 3/4 prompt + 1/4 output (not the headline)")
     return ap.parse_args()
@@ -184,7 +188,7 @@ def profiled_traffic(kernel_src, profile_name):
 class Path:
     """Device buffers and the five C-ABI calls of one step."""
 
-    def __init__(self, pk, loop: wl.DecodeLoop):
+    def __init__(self, pk, loop: wl.DecodeLoop, fused=True):
         self.pk, self.loop = pk, loop
         w, dev = loop.w, loop.device
         B, K, C = w.B, w.K, w.C_cap
@@ -197,40 +201,57 @@ class Path:
         self.acc, self.nxt, self.kv = torch.zeros(B, **i32), torch.zeros(B, **i32), torch.zeros(B, **i32)
         self.ws = torch.zeros(pk.pldp_verify_workspace_size(B, K, w.V), dtype=torch.uint8, device=dev)
         self.row_idx = None   # all R rows of the chosen layers
+        self.fused = fused
+        self.kernels = (["draft_step"] if fused else
+                        ["find_candidates", "rank_hidden", "rank_attention", "extract_draft"]) + ["verify_greedy"]
 
     def run(self, ev=None, stream=None):
+        """One step: the drafting half (one fused launch, or the four separate calls)
+        then verification.  ev: events recorded before the first and after every kernel."""
         pk, lp, w = self.pk, self.loop, self.loop.w
         s = torch.cuda.current_stream() if stream is None else stream
-        rec = (lambda i: ev[i].record(s)) if ev is not None else (lambda i: None)
-        rec(0)
-        pk.pldp_find_candidates(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt,
-                                self.ml, self.status, stream=s)
-        rec(1)
-        pk.pldp_rank_hidden(lp.H, lp.seq_len, self.cand, self.cnt, self.best_h, status=self.status,
-                            stream=s)
-        rec(2)
-        pk.pldp_rank_attention(lp.A, lp.seq_len, self.cand, self.cnt, self.best_a, row_idx=self.row_idx,
+        k = [0]
+
+        def rec():
+            if ev is not None:
+                ev[k[0]].record(s)
+                k[0] += 1
+
+        rec()
+        if self.fused:
+            pk.pldp_draft_step(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt, self.ml,
+                               w.K, self.draft, self.dlen, H=lp.H, best_h=self.best_h, A=lp.A,
+                               best_a=self.best_a, row_idx=self.row_idx, draft_from="hidden",
                                status=self.status, stream=s)
-        rec(3)
-        pk.pldp_extract_draft(lp.ids, lp.seq_len, self.best_h, self.draft, self.dlen, stream=s)
-        rec(4)
+            rec()
+        else:
+            pk.pldp_find_candidates(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt,
+                                    self.ml, self.status, stream=s)
+            rec()
+            pk.pldp_rank_hidden(lp.H, lp.seq_len, self.cand, self.cnt, self.best_h, status=self.status,
+                                stream=s)
+            rec()
+            pk.pldp_rank_attention(lp.A, lp.seq_len, self.cand, self.cnt, self.best_a,
+                                   row_idx=self.row_idx, status=self.status, stream=s)
+            rec()
+            pk.pldp_extract_draft(lp.ids, lp.seq_len, self.best_h, self.draft, self.dlen, stream=s)
+            rec()
         pk.pldp_verify_greedy(lp.logits, self.draft, self.dlen, self.acc, self.nxt, self.ws, ids=lp.ids,
                               seq_len=lp.seq_len, kv_keep_len=self.kv, status=self.status, stream=s)
-        rec(5)
-
-
-KERNELS = ["find_candidates", "rank_hidden", "rank_attention", "extract_draft", "verify_greedy"]
+        rec()
 
 
 def step_bytes(w, seq_len_mean, cand_mean):
     """Algorithmic bytes per step: ids scanned, hidden rows (query + candidates),
     attention values gathered, draft tokens read, logits read."""
     B = w.B
-    return dict(find_candidates=4.0 * B * seq_len_mean,
-                rank_hidden=2.0 * B * (cand_mean + 1) * w.d,
-                rank_attention=2.0 * B * cand_mean * w.R,
-                extract_draft=4.0 * B * w.K,
-                verify_greedy=2.0 * B * (w.K + 1) * w.V)
+    by = dict(find_candidates=4.0 * B * seq_len_mean,
+              rank_hidden=2.0 * B * (cand_mean + 1) * w.d,
+              rank_attention=2.0 * B * cand_mean * w.R,
+              extract_draft=4.0 * B * w.K,
+              verify_greedy=2.0 * B * (w.K + 1) * w.V)
+    by["draft_step"] = by["find_candidates"] + by["rank_hidden"] + by["rank_attention"] + by["extract_draft"]
+    return by
 
 
 def workload(args):
@@ -239,6 +260,8 @@ def workload(args):
         w = w.replace(B=args.batch)
     if args.context:
         w = w.replace(prompt_len=args.context * 3 // 4, out_len=args.context - args.context * 3 // 4)
+    if args.hidden_width:
+        w = w.replace(d=args.hidden_width)
     return w
 
 
@@ -253,7 +276,8 @@ def run_ours(args, ws_, rank, local):
     K_steps, W_steps = args.steps, args.warmup
     t0 = time.perf_counter()
     loop = wl.DecodeLoop(w, steps=W_steps + K_steps, device=dev)
-    path = Path(pk, loop)
+    path = Path(pk, loop, fused=not args.separate)
+    nk = len(path.kernels)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)     # 2x the 129 MB L2
     torch.cuda.synchronize()
     setup_s = time.perf_counter() - t0
@@ -264,7 +288,7 @@ def run_ours(args, ws_, rank, local):
         path.run()
     torch.cuda.synchronize()
 
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(K_steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(K_steps)]
     cand_sum = torch.zeros((), dtype=torch.int64, device=dev)
     len_sum = torch.zeros((), dtype=torch.int64, device=dev)
     acc_sum = torch.zeros((), dtype=torch.int64, device=dev)
@@ -285,9 +309,9 @@ def run_ours(args, ws_, rank, local):
     barrier(ws_)
     clk = clocks.stop()
 
-    per_k = np.zeros(5)
+    per_k = np.zeros(nk)
     for e in evs:
-        for k in range(5):
+        for k in range(nk):
             per_k[k] += e[k].elapsed_time(e[k + 1])
     step_ms_total = float(per_k.sum())                        # device ms over K steps
     step_ms_total = max_over_ranks(step_ms_total, ws_)
@@ -299,12 +323,13 @@ def run_ours(args, ws_, rank, local):
     L_mean = float(len_sum) / (K_steps * w.B)
     by = step_bytes(w, L_mean, cand_mean)
     peak, peak_kind = measured_peak()
-    ver_s = per_k[4] / K_steps / 1e3
+    ver_s = per_k[nk - 1] / K_steps / 1e3
     ver_bytes = by["verify_greedy"]
     achieved = ver_bytes / ver_s / 1e9
     traffic = profiled_traffic(os.path.join(ROOT, "paper_2412_01447_gb300", "csrc", "verify.cu"),
                                "verify_greedy_c5.md")
-    step_bytes_total = sum(by.values())
+    step_bytes_total = sum(by[k] for k in ("find_candidates", "rank_hidden", "rank_attention",
+                                            "extract_draft", "verify_greedy"))
     lossless = bool(torch.equal(loop.ids[:, :w.T], loop.gt[:, :w.T]))
     L_now = loop.seq_len.long()
     pos = torch.arange(loop.T_cap, device=dev)[None]
@@ -333,18 +358,21 @@ def run_ours(args, ws_, rank, local):
                    "attention_rows": w.R, "C_cap": w.C_cap,
                    "l2": "flushed before every step (256 MB write); per-step logits 427 MB and "
                          "attention rows 1.18 GB regenerated between steps",
-                   "timing": "CUDA events around the five kernels of each step on the launch stream; "
+                   "path": ("pldp_draft_step (fused scan + both rankings + draft) + pldp_verify_greedy"
+                            if path.fused else "five separate C-ABI calls"),
+                   "timing": "CUDA events around every kernel of each step on the launch stream; "
                              "artifact generation between steps is not timed",
                    "parallelism": f"{ws_} independent replicas (batch shards)"},
         "achieved_step_gbs": round(step_bytes_total / (ms_per_step / 1e3) / 1e9, 1),
         "frac_step_of_nominal_8tbs": round(step_bytes_total / (ms_per_step / 1e3) / 1e9 / NOMINAL_HBM_GBS, 4),
-        "kernel_us": {k: round(per_k[i] / K_steps * 1e3, 2) for i, k in enumerate(KERNELS)},
-        "kernel_gbs": {k: round(by[k] / (per_k[i] / K_steps / 1e3) / 1e9, 1) for i, k in enumerate(KERNELS)},
+        "kernel_us": {k: round(per_k[i] / K_steps * 1e3, 2) for i, k in enumerate(path.kernels)},
+        "kernel_gbs": {k: round(by[k] / (per_k[i] / K_steps / 1e3) / 1e9, 1)
+                       for i, k in enumerate(path.kernels)},
         "roofline": {"kernel": "verify_greedy", "bound": "hbm", "achieved": round(achieved, 1),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
                      "traffic": traffic, "algorithmic_bytes": ver_bytes},
-        "gpu_launches": 5 * K_steps,
+        "gpu_launches": nk * K_steps,
         "clocks": clk,
         "stats": {"mean_candidates": round(cand_mean, 3), "mean_accept": round(acc_mean, 3),
                   "mean_context": round(L_mean, 1), "status_nonzero": int((st != 0).sum()),

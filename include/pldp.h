@@ -183,6 +183,74 @@ PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
                                         int32_t* draft, int32_t* draft_len, void* stream);
 
 /*
+ * The drafting half of a step in one launch: candidate search, ranking by
+ * hidden states and/or attentions, and draft extraction, with the results of
+ * pldp_find_candidates, pldp_rank_hidden, pldp_rank_attention and
+ * pldp_extract_draft called in turn (same conventions, same status bits; the
+ * fp32 score sums may be split differently, so scores can differ in the last
+ * bits and a tie within rounding may be broken differently).
+ * One thread-block cluster per sequence scans the context, ranks the matches
+ * (the two rankings on different CTAs of the cluster, in parallel) and writes
+ * the draft; the query row H_{t-1} is fetched at kernel entry, overlapping the
+ * scan.  Eq. 1-3 (Sec. 4.2) and Sec. 4.3.
+ *
+ * Fields of the argument block (device pointers unless stated):
+ *  ids .. match_len      as pldp_find_candidates; ids must be 16-byte aligned
+ *                        with ids_stride and T_cap multiples of 4.
+ *  H .. best_h_score     as pldp_rank_hidden (H = NULL skips hidden ranking;
+ *                        H rows must be 16-byte aligned).  h_scores and
+ *                        best_h_score may be NULL.
+ *  A .. best_a_score     as pldp_rank_attention (A = NULL skips it); a_scores
+ *                        and best_a_score may be NULL.
+ *  draft_from            0: draft after best_h, 1: after best_a (that ranking
+ *                        must be given).
+ *  K, draft, draft_len   as pldp_extract_draft.
+ *  status                uint32 [B] or NULL.
+ * Layouts the fused kernel does not take return PLDP_ERR_UNSUPPORTED; the
+ * separate calls accept them.
+ */
+typedef struct pldp_draft_step_args {
+    const int32_t* ids;
+    int64_t ids_stride;
+    const int32_t* seq_len;
+    int B;
+    int64_t T_cap;
+    int ngram_min;
+    int ngram_max;
+    int32_t* cand_pos;
+    int C_cap;
+    int32_t* cand_count;
+    int32_t* match_len;
+    const void* H;
+    pldp_dtype h_dtype;
+    int64_t d;
+    int64_t h_seq_stride;
+    float threshold;
+    float* h_scores;
+    int32_t* best_h;
+    float* best_h_score;
+    const void* A;
+    pldp_dtype a_dtype;
+    int R;
+    int64_t a_row_stride;
+    int64_t a_seq_stride;
+    const int32_t* row_idx;
+    int n_sel;
+    pldp_agg agg;
+    float* a_scores;
+    int32_t* best_a;
+    float* best_a_score;
+    int draft_from;
+    int K;
+    int32_t* draft;
+    int32_t* draft_len;
+    uint32_t* status;
+} pldp_draft_step_args;
+
+/* `args` is a HOST pointer to the argument block, read before the call returns. */
+PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* args, void* stream);
+
+/*
  * Greedy verification -- Sec. 4.4 at temperature 0, with the K+1 next-token
  * distributions of one forward pass on the draft (Sec. 3):
  *   a_i   = argmax_v logits[b, i, v], i = 0..K   (smallest v among equal maxima;

@@ -30,7 +30,7 @@ __all__ = [
     "PLDP_ST_CAND_OVERFLOW", "PLDP_ST_TOKEN_RANGE", "PLDP_ST_CAPACITY", "PLDP_ST_SEQ_LEN",
     "PLDP_ST_DRAFT_LEN", "PLDP_ST_ROW_INDEX", "PLDP_ST_TIMEOUT",
     "pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention", "pldp_extract_draft",
-    "pldp_verify_greedy", "pldp_verify_greedy_noalloc", "pldp_verify_workspace_size",
+    "pldp_draft_step", "pldp_draft_step_args", "pldp_verify_greedy", "pldp_verify_greedy_noalloc", "pldp_verify_workspace_size",
     "pldp_version", "pldp_last_error",
 ]
 
@@ -56,6 +56,25 @@ class PldpError(RuntimeError):
 
 _lock = threading.Lock()
 _lib = None
+
+
+class pldp_draft_step_args(ctypes.Structure):
+    """Mirror of the C argument block of pldp_draft_step (include/pldp.h)."""
+    _fields_ = [
+        ("ids", ctypes.c_void_p), ("ids_stride", ctypes.c_int64), ("seq_len", ctypes.c_void_p),
+        ("B", ctypes.c_int), ("T_cap", ctypes.c_int64), ("ngram_min", ctypes.c_int),
+        ("ngram_max", ctypes.c_int), ("cand_pos", ctypes.c_void_p), ("C_cap", ctypes.c_int),
+        ("cand_count", ctypes.c_void_p), ("match_len", ctypes.c_void_p),
+        ("H", ctypes.c_void_p), ("h_dtype", ctypes.c_int), ("d", ctypes.c_int64),
+        ("h_seq_stride", ctypes.c_int64), ("threshold", ctypes.c_float), ("h_scores", ctypes.c_void_p),
+        ("best_h", ctypes.c_void_p), ("best_h_score", ctypes.c_void_p),
+        ("A", ctypes.c_void_p), ("a_dtype", ctypes.c_int), ("R", ctypes.c_int),
+        ("a_row_stride", ctypes.c_int64), ("a_seq_stride", ctypes.c_int64), ("row_idx", ctypes.c_void_p),
+        ("n_sel", ctypes.c_int), ("agg", ctypes.c_int), ("a_scores", ctypes.c_void_p),
+        ("best_a", ctypes.c_void_p), ("best_a_score", ctypes.c_void_p),
+        ("draft_from", ctypes.c_int), ("K", ctypes.c_int), ("draft", ctypes.c_void_p),
+        ("draft_len", ctypes.c_void_p), ("status", ctypes.c_void_p),
+    ]
 
 
 def library_path() -> str:
@@ -90,6 +109,8 @@ def _load():
             for f in ("pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention",
                       "pldp_extract_draft", "pldp_verify_greedy"):
                 getattr(lib, f).restype = ctypes.c_int
+            lib.pldp_draft_step.argtypes = [ctypes.POINTER(pldp_draft_step_args), P]
+            lib.pldp_draft_step.restype = ctypes.c_int
             lib.pldp_verify_greedy_noalloc.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64,
                                                        P, i64, P, P, P]
             lib.pldp_verify_greedy_noalloc.restype = ctypes.c_int
@@ -216,6 +237,50 @@ def pldp_extract_draft(ids, seq_len, best_pos, draft, draft_len, T_cap=None, str
         p_ids, stride, _dense(seq_len, "seq_len", torch.int32), T if T_cap is None else T_cap,
         _dense(best_pos, "best_pos", torch.int32), B, K, _dense(draft, "draft", torch.int32),
         _dense(draft_len, "draft_len", torch.int32), _stream(stream)))
+
+
+def pldp_draft_step(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, draft,
+                    draft_len, H=None, best_h=None, h_scores=None, best_h_score=None,
+                    threshold=float("-inf"), A=None, best_a=None, row_idx=None, agg=PLDP_AGG_MAX,
+                    a_scores=None, best_a_score=None, draft_from="hidden", status=None, T_cap=None,
+                    stream=None):
+    """Candidate search, ranking (hidden and/or attention) and draft in one launch;
+    the arguments mean what they mean in the separate calls."""
+    p_ids, stride, T = _rows(ids, "ids")
+    B = ids.shape[0]
+    a = pldp_draft_step_args()
+    a.ids, a.ids_stride, a.seq_len, a.B = p_ids, stride, _dense(seq_len, "seq_len", torch.int32), B
+    a.T_cap = T if T_cap is None else T_cap
+    a.ngram_min, a.ngram_max = ngram_min, ngram_max
+    a.cand_pos = _dense(cand_pos, "cand_pos", torch.int32, allow_none=True)
+    a.C_cap = cand_pos.shape[1] if cand_pos is not None and cand_pos.dim() == 2 else 0
+    a.cand_count = _dense(cand_count, "cand_count", torch.int32)
+    a.match_len = _dense(match_len, "match_len", torch.int32)
+    if H is not None:
+        if H.dim() != 3 or H.stride(2) != 1 or H.stride(1) != H.shape[2]:
+            raise ValueError("H must be [B, T_cap, d] with contiguous rows")
+        a.H, a.h_dtype, a.d, a.h_seq_stride = _dev(H, "H"), _code(H.dtype), H.shape[2], H.stride(0)
+        a.threshold = float(threshold)
+        a.h_scores = _dense(h_scores, "h_scores", torch.float32, allow_none=True)
+        a.best_h = _dense(best_h, "best_h", torch.int32)
+        a.best_h_score = _dense(best_h_score, "best_h_score", torch.float32, allow_none=True)
+    if A is not None:
+        if A.dim() != 3 or A.stride(2) != 1:
+            raise ValueError("A must be [B, R, T_cap] with unit inner stride")
+        a.A, a.a_dtype, a.R = _dev(A, "A"), _code(A.dtype), A.shape[1]
+        a.a_row_stride, a.a_seq_stride = A.stride(1), A.stride(0)
+        a.row_idx = _dense(row_idx, "row_idx", torch.int32, allow_none=True)
+        a.n_sel = A.shape[1] if row_idx is None else row_idx.numel()
+        a.agg = int(agg)
+        a.a_scores = _dense(a_scores, "a_scores", torch.float32, allow_none=True)
+        a.best_a = _dense(best_a, "best_a", torch.int32)
+        a.best_a_score = _dense(best_a_score, "best_a_score", torch.float32, allow_none=True)
+    a.draft_from = {"hidden": 0, "attention": 1, 0: 0, 1: 1}[draft_from]
+    a.K = K
+    a.draft = _dense(draft, "draft", torch.int32)
+    a.draft_len = _dense(draft_len, "draft_len", torch.int32)
+    a.status = _dense(status, "status", None, allow_none=True)
+    _check("pldp_draft_step", _load().pldp_draft_step(ctypes.byref(a), _stream(stream)))
 
 
 def pldp_verify_workspace_size(B, K, V) -> int:

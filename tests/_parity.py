@@ -51,8 +51,25 @@ class Buffers:
 
 def gpu_step(buf, ids, seq_len, logits, ngram=(1, 3), H=None, A=None, row_idx=None,
              agg=pk.PLDP_AGG_MAX, draft_from="hidden", threshold=float("-inf"), append=True,
-             stream=None):
-    """One step through the C ABI; ids/seq_len are updated in place when append."""
+             stream=None, fused=False):
+    """One step through the C ABI; ids/seq_len are updated in place when append.
+    fused: the drafting half runs as the single pldp_draft_step launch."""
+    if fused:
+        ri = None if row_idx is None or A is None else torch.as_tensor(row_idx, dtype=torch.int32,
+                                                                        device=A.device)
+        pk.pldp_draft_step(ids, seq_len, ngram[0], ngram[1], buf.cand, buf.cnt, buf.ml, buf.draft.shape[1],
+                           buf.draft, buf.dlen, H=H, best_h=buf.best_h if H is not None else None,
+                           h_scores=buf.scores_h, best_h_score=buf.bscore_h, threshold=threshold, A=A,
+                           best_a=buf.best_a if A is not None else None, row_idx=ri, agg=agg,
+                           a_scores=buf.scores_a, best_a_score=buf.bscore_a, draft_from=draft_from,
+                           status=buf.status, stream=stream)
+        if logits is not None:
+            pk.pldp_verify_greedy(logits, buf.draft, buf.dlen, buf.acc, buf.nxt, buf.ws,
+                                  argmax=buf.argmax, ids=ids if append else None,
+                                  seq_len=seq_len if append else None,
+                                  kv_keep_len=buf.kv if append else None, status=buf.status,
+                                  stream=stream)
+        return
     pk.pldp_find_candidates(ids, seq_len, ngram[0], ngram[1], buf.cand, buf.cnt, buf.ml,
                             buf.status, stream=stream)
     if H is not None:

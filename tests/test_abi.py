@@ -97,3 +97,21 @@ def test_python_binding_refuses_cpu_tensors():
         pk.pldp_find_candidates(x, torch.zeros(2, dtype=torch.int32), 1, 3,
                                 torch.zeros((2, 4), dtype=torch.int32),
                                 torch.zeros(2, dtype=torch.int32), torch.zeros(2, dtype=torch.int32))
+
+
+def test_draft_step_args_layout_matches_header(tmp_path):
+    """The Python mirror of pldp_draft_step_args has the C layout (gcc offsetof)."""
+    names = [f for f, _ in pk.pldp_draft_step_args._fields_]
+    src = ['#include <stdio.h>', '#include <stddef.h>', f'#include "{HEADER}"', "int main(void) {",
+           'printf("%zu\\n", sizeof(pldp_draft_step_args));']
+    src += [f'printf("%zu\\n", offsetof(pldp_draft_step_args, {n}));' for n in names]
+    src += ["return 0; }"]
+    c = tmp_path / "layout.c"
+    c.write_text("\n".join(src))
+    exe = tmp_path / "layout"
+    import subprocess
+    subprocess.check_call(["gcc", str(c), "-o", str(exe)])
+    out = [int(x) for x in subprocess.check_output([str(exe)]).split()]
+    assert out[0] == ctypes.sizeof(pk.pldp_draft_step_args)
+    for n, off in zip(names, out[1:]):
+        assert getattr(pk.pldp_draft_step_args, n).offset == off, n

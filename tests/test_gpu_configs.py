@@ -20,8 +20,9 @@ def _sample(B, k, seed):
     return sorted(np.random.default_rng(seed).choice(B, k, replace=False).tolist())
 
 
+@pytest.mark.parametrize("fused", [False, True], ids=["calls", "fused"])
 @pytest.mark.parametrize("name", ["c1", "c2", "c3", "c4"])
-def test_single_step_config(lib, name):
+def test_single_step_config(lib, name, fused):
     w = wl.CONFIGS[name]
     inp = wl.single_step(w, device=DEV)
     B, K, C = w.B, w.K, w.C_cap
@@ -29,7 +30,7 @@ def test_single_step_config(lib, name):
     buf = Buffers(B, K, w.V, C, DEV)
     draft_from = "hidden" if inp["H"] is not None else "attention"
     gpu_step(buf, inp["ids"], inp["seq_len"], inp["logits"], ngram=(w.ngram_min, w.ngram_max),
-             H=inp["H"], A=inp["A"], row_idx=None, draft_from=draft_from)
+             H=inp["H"], A=inp["A"], row_idx=None, draft_from=draft_from, fused=fused)
     g = snapshot(buf)
 
     o_cand, o_cnt, o_ml, o_st = oracle.find_candidates(ids0, L0, w.ngram_min, w.ngram_max, C)
@@ -65,7 +66,8 @@ def test_single_step_config(lib, name):
         assert g["acc"].tolist() == [6]
 
 
-def test_decode_loop_c5(lib):
+@pytest.mark.parametrize("fused", [False, True], ids=["calls", "fused"])
+def test_decode_loop_c5(lib, fused):
     """The sustained loop: every step compared with the oracle run on the same
     pre-step state; the emitted streams equal the ground truth (losslessness)."""
     w = wl.CONFIGS["c5"]
@@ -81,7 +83,7 @@ def test_decode_loop_c5(lib):
         ids0, L0 = host(loop.ids), host(loop.seq_len)
         As, lg = host(loop.A[sel]), host(loop.logits)
         gpu_step(buf, loop.ids, loop.seq_len, loop.logits, ngram=(w.ngram_min, w.ngram_max), H=loop.H,
-                 A=loop.A, draft_from="hidden")
+                 A=loop.A, draft_from="hidden", fused=fused)
         g = snapshot(buf)
         o_cand, o_cnt, o_ml, _ = oracle.find_candidates(ids0, L0, w.ngram_min, w.ngram_max, C)
         assert np.array_equal(g["cnt"], o_cnt) and np.array_equal(g["ml"], o_ml)
@@ -109,7 +111,8 @@ def test_decode_loop_c5(lib):
     assert (L - w.T).mean() > steps * 1.5      # drafts are accepted: more than one token per step
 
 
-def test_graph_capture_replays_the_step(lib):
+@pytest.mark.parametrize("fused", [False, True], ids=["calls", "fused"])
+def test_graph_capture_replays_the_step(lib, fused):
     """The five calls captured in one CUDA graph give the eager results, and the
     verify workspace returns to zero between replays."""
     w = wl.CONFIGS["c5"].replace(B=16, prompt_len=3000, out_len=1000, V=32000, d=1024)
@@ -123,12 +126,13 @@ def test_graph_capture_replays_the_step(lib):
     b.step_inputs(0)
     torch.cuda.synchronize()
     with torch.cuda.graph(graph, stream=stream):
-        gpu_step(buf_b, b.ids, b.seq_len, b.logits, H=b.H, A=b.A, stream=torch.cuda.current_stream())
+        gpu_step(buf_b, b.ids, b.seq_len, b.logits, H=b.H, A=b.A, stream=torch.cuda.current_stream(),
+                 fused=fused)
     b.reset()
     for s in range(6):
         a.step_inputs(s)
         b.step_inputs(s)
-        gpu_step(buf_a, a.ids, a.seq_len, a.logits, H=a.H, A=a.A)
+        gpu_step(buf_a, a.ids, a.seq_len, a.logits, H=a.H, A=a.A, fused=fused)
         graph.replay()
         torch.cuda.synchronize()
         ga, gb = snapshot(buf_a), snapshot(buf_b)
