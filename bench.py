@@ -53,6 +53,9 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="c5")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--flush", choices=["write-read", "write"], default="write-read",
+                    help="L2 flush before each step: write 256 MB then read 256 MB (cold, clean L2), "
+                         "or the write alone (cold L2 full of dirty lines)")
     ap.add_argument("--separate", action="store_true",
                     help="draft with the four separate calls instead of the fused launch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -200,8 +203,10 @@ class Path:
         self.draft, self.dlen = torch.zeros((B, K), **i32), torch.zeros(B, **i32)
         self.acc, self.nxt, self.kv = torch.zeros(B, **i32), torch.zeros(B, **i32), torch.zeros(B, **i32)
         self.ws = torch.zeros(pk.pldp_verify_workspace_size(B, K, w.V), dtype=torch.uint8, device=dev)
+        self.dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=dev)
         self.row_idx = None   # all R rows of the chosen layers
         self.fused = fused
+        self.launches_per_step = 3 if fused else 5     # pldp_draft_step launches two kernels
         self.kernels = (["draft_step"] if fused else
                         ["find_candidates", "rank_hidden", "rank_attention", "extract_draft"]) + ["verify_greedy"]
 
@@ -220,7 +225,7 @@ class Path:
         rec()
         if self.fused:
             pk.pldp_draft_step(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt, self.ml,
-                               w.K, self.draft, self.dlen, H=lp.H, best_h=self.best_h, A=lp.A,
+                               w.K, self.draft, self.dlen, self.dws, H=lp.H, best_h=self.best_h, A=lp.A,
                                best_a=self.best_a, row_idx=self.row_idx, draft_from="hidden",
                                status=self.status, stream=s)
             rec()
@@ -279,12 +284,18 @@ def run_ours(args, ws_, rank, local):
     path = Path(pk, loop, fused=not args.separate)
     nk = len(path.kernels)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)     # 2x the 129 MB L2
+    flush_sink = torch.empty((), dtype=torch.int64, device=dev)
+
+    def flush_l2(s):
+        flush.fill_(s & 0xFF)
+        if args.flush == "write-read":
+            torch.sum(flush.view(torch.int64), dim=0, out=flush_sink)   # evicts the dirty lines
     torch.cuda.synchronize()
     setup_s = time.perf_counter() - t0
 
     for s in range(W_steps):
         loop.step_inputs(s)
-        flush.zero_()
+        flush_l2(s)
         path.run()
     torch.cuda.synchronize()
 
@@ -299,8 +310,8 @@ def run_ours(args, ws_, rank, local):
     wall0 = time.perf_counter()
     for s in range(K_steps):
         loop.step_inputs(W_steps + s)
-        flush.zero_()
         len_sum += loop.seq_len.sum()
+        flush_l2(s)
         path.run(evs[s])
         cand_sum += path.cnt.clamp(max=w.C_cap).sum()
         acc_sum += path.acc.sum()
@@ -356,8 +367,10 @@ def run_ours(args, ws_, rank, local):
                                "heads, both rankings every step",
                    "batch_per_gpu": w.B, "context": w.T, "vocab": w.V, "K": w.K, "d": w.d,
                    "attention_rows": w.R, "C_cap": w.C_cap,
-                   "l2": "flushed before every step (256 MB write); per-step logits 427 MB and "
-                         "attention rows 1.18 GB regenerated between steps",
+                   "l2": ("flushed before every step: 256 MB write then 256 MB read (cold, clean L2)"
+                          if args.flush == "write-read" else
+                          "flushed before every step: 256 MB write (cold L2 holding dirty lines)")
+                         + "; per-step logits 427 MB and attention rows 1.18 GB regenerated between steps",
                    "path": ("pldp_draft_step (fused scan + both rankings + draft) + pldp_verify_greedy"
                             if path.fused else "five separate C-ABI calls"),
                    "timing": "CUDA events around every kernel of each step on the launch stream; "
@@ -372,7 +385,7 @@ def run_ours(args, ws_, rank, local):
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
                      "traffic": traffic, "algorithmic_bytes": ver_bytes},
-        "gpu_launches": nk * K_steps,
+        "gpu_launches": path.launches_per_step * K_steps,
         "clocks": clk,
         "stats": {"mean_candidates": round(cand_mean, 3), "mean_accept": round(acc_mean, 3),
                   "mean_context": round(L_mean, 1), "status_nonzero": int((st != 0).sum()),

@@ -183,20 +183,23 @@ PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
                                         int32_t* draft, int32_t* draft_len, void* stream);
 
 /*
- * The drafting half of a step in one launch: candidate search, ranking by
- * hidden states and/or attentions, and draft extraction, with the results of
+ * The drafting half of a step in one call: candidate search, ranking by hidden
+ * states and/or attentions, and draft extraction, with the results of
  * pldp_find_candidates, pldp_rank_hidden, pldp_rank_attention and
  * pldp_extract_draft called in turn (same conventions, same status bits; the
  * fp32 score sums may be split differently, so scores can differ in the last
- * bits and a tie within rounding may be broken differently).
- * One thread-block cluster per sequence scans the context, ranks the matches
- * (the two rankings on different CTAs of the cluster, in parallel) and writes
- * the draft; the query row H_{t-1} is fetched at kernel entry, overlapping the
- * scan.  Eq. 1-3 (Sec. 4.2) and Sec. 4.3.
+ * bits and a tie within rounding may be broken differently).  Eq. 1-3
+ * (Sec. 4.2) and Sec. 4.3.
+ *
+ * Two short kernels: a flat (chunk, sequence) grid streams the contexts and
+ * records every occurrence of x_t with its suffix-match length in a small
+ * per-sequence list held in the workspace; then one CTA per sequence orders the
+ * list into the candidate list, ranks it and writes the draft (the query row
+ * H_{t-1} is fetched by a bulk copy at that kernel's entry).  More than 256
+ * occurrences in a sequence fall back to an ordered rescan of its context.
  *
  * Fields of the argument block (device pointers unless stated):
- *  ids .. match_len      as pldp_find_candidates; ids must be 16-byte aligned
- *                        with ids_stride and T_cap multiples of 4.
+ *  ids .. match_len      as pldp_find_candidates (T_cap <= 2^27).
  *  H .. best_h_score     as pldp_rank_hidden (H = NULL skips hidden ranking;
  *                        H rows must be 16-byte aligned).  h_scores and
  *                        best_h_score may be NULL.
@@ -206,7 +209,11 @@ PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
  *                        must be given).
  *  K, draft, draft_len   as pldp_extract_draft.
  *  status                uint32 [B] or NULL.
- * Layouts the fused kernel does not take return PLDP_ERR_UNSUPPORTED; the
+ *  workspace             device scratch of pldp_draft_workspace_size(B) bytes,
+ *                        16-byte aligned, ZEROED by the caller before its first
+ *                        use; every call leaves it zeroed again.  Calls that may
+ *                        run concurrently need separate workspaces.
+ * Layouts the fused path does not take return PLDP_ERR_UNSUPPORTED; the
  * separate calls accept them.
  */
 typedef struct pldp_draft_step_args {
@@ -245,10 +252,15 @@ typedef struct pldp_draft_step_args {
     int32_t* draft;
     int32_t* draft_len;
     uint32_t* status;
+    void* workspace;
+    size_t workspace_bytes;
 } pldp_draft_step_args;
 
 /* `args` is a HOST pointer to the argument block, read before the call returns. */
 PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* args, void* stream);
+
+/* Bytes of workspace pldp_draft_step needs for B sequences (0 if B < 0). */
+PLDP_API size_t pldp_draft_workspace_size(int B);
 
 /*
  * Greedy verification -- Sec. 4.4 at temperature 0, with the K+1 next-token

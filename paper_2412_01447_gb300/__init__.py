@@ -30,7 +30,7 @@ __all__ = [
     "PLDP_ST_CAND_OVERFLOW", "PLDP_ST_TOKEN_RANGE", "PLDP_ST_CAPACITY", "PLDP_ST_SEQ_LEN",
     "PLDP_ST_DRAFT_LEN", "PLDP_ST_ROW_INDEX", "PLDP_ST_TIMEOUT",
     "pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention", "pldp_extract_draft",
-    "pldp_draft_step", "pldp_draft_step_args", "pldp_verify_greedy", "pldp_verify_greedy_noalloc", "pldp_verify_workspace_size",
+    "pldp_draft_step", "pldp_draft_step_args", "pldp_draft_workspace_size", "pldp_verify_greedy", "pldp_verify_greedy_noalloc", "pldp_verify_workspace_size",
     "pldp_version", "pldp_last_error",
 ]
 
@@ -74,6 +74,7 @@ class pldp_draft_step_args(ctypes.Structure):
         ("best_a", ctypes.c_void_p), ("best_a_score", ctypes.c_void_p),
         ("draft_from", ctypes.c_int), ("K", ctypes.c_int), ("draft", ctypes.c_void_p),
         ("draft_len", ctypes.c_void_p), ("status", ctypes.c_void_p),
+        ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
     ]
 
 
@@ -111,6 +112,8 @@ def _load():
                 getattr(lib, f).restype = ctypes.c_int
             lib.pldp_draft_step.argtypes = [ctypes.POINTER(pldp_draft_step_args), P]
             lib.pldp_draft_step.restype = ctypes.c_int
+            lib.pldp_draft_workspace_size.argtypes = [i32]
+            lib.pldp_draft_workspace_size.restype = sz
             lib.pldp_verify_greedy_noalloc.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64,
                                                        P, i64, P, P, P]
             lib.pldp_verify_greedy_noalloc.restype = ctypes.c_int
@@ -239,13 +242,18 @@ def pldp_extract_draft(ids, seq_len, best_pos, draft, draft_len, T_cap=None, str
         _dense(draft_len, "draft_len", torch.int32), _stream(stream)))
 
 
+def pldp_draft_workspace_size(B) -> int:
+    return int(_load().pldp_draft_workspace_size(B))
+
+
 def pldp_draft_step(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, draft,
-                    draft_len, H=None, best_h=None, h_scores=None, best_h_score=None,
+                    draft_len, workspace, H=None, best_h=None, h_scores=None, best_h_score=None,
                     threshold=float("-inf"), A=None, best_a=None, row_idx=None, agg=PLDP_AGG_MAX,
                     a_scores=None, best_a_score=None, draft_from="hidden", status=None, T_cap=None,
                     stream=None):
-    """Candidate search, ranking (hidden and/or attention) and draft in one launch;
-    the arguments mean what they mean in the separate calls."""
+    """Candidate search, ranking (hidden and/or attention) and draft in one call; the
+    arguments mean what they mean in the separate calls.  workspace: a uint8 CUDA
+    tensor of pldp_draft_workspace_size(B) bytes, zeroed once before first use."""
     p_ids, stride, T = _rows(ids, "ids")
     B = ids.shape[0]
     a = pldp_draft_step_args()
@@ -280,6 +288,8 @@ def pldp_draft_step(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, ma
     a.draft = _dense(draft, "draft", torch.int32)
     a.draft_len = _dense(draft_len, "draft_len", torch.int32)
     a.status = _dense(status, "status", None, allow_none=True)
+    a.workspace = _dense(workspace, "workspace")
+    a.workspace_bytes = workspace.numel() * workspace.element_size()
     _check("pldp_draft_step", _load().pldp_draft_step(ctypes.byref(a), _stream(stream)))
 
 

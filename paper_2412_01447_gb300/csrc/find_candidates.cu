@@ -16,6 +16,7 @@ find_candidates_kernel(const int32_t* __restrict__ ids, int64_t ids_stride,
                        int32_t* __restrict__ cand_count, int32_t* __restrict__ match_len,
                        uint32_t* __restrict__ status, int64_t chunk) {
     __shared__ ScanShared sh;
+    pdl_enter();
     cg::cluster_group cluster = cg::this_cluster();
     const int CL = static_cast<int>(cluster.num_blocks());
     const int rank = static_cast<int>(cluster.block_rank());
@@ -48,7 +49,8 @@ find_candidates_kernel(const int32_t* __restrict__ ids, int64_t ids_stride,
     int c[PLDP_MAX_NGRAM];
 #pragma unroll
     for (int k = 0; k < PLDP_MAX_NGRAM; ++k) c[k] = 0;
-    scan_count<VEC>(row, c0, c1, t, ngram_max, c);
+    const GlobalIds src{row};
+    scan_count<VEC>(src, row, c0, c1, t, ngram_max, c);
     __syncthreads();                       // sh.cnt zeroed before the adds
     scan_reduce_counts(c, ngram_max, sh);
 
@@ -60,7 +62,7 @@ find_candidates_kernel(const int32_t* __restrict__ ids, int64_t ids_stride,
         match_len[b] = sh.nstar;
         if (status && sh.total > C_cap) status[b] |= PLDP_ST_CAND_OVERFLOW;
     }
-    scan_write<VEC>(row, c0, c1, t, ngram_max, sh, cand_pos + static_cast<int64_t>(b) * C_cap, C_cap);
+    scan_write<VEC>(src, row, c0, c1, t, ngram_max, sh, cand_pos + static_cast<int64_t>(b) * C_cap, C_cap);
     cluster_wait();
 }
 
@@ -101,13 +103,15 @@ extern "C" PLDP_API pldp_status pldp_find_candidates(const int32_t* ids, int64_t
     cfg.blockDim = dim3(kScanThreads);
     cfg.dynamicSmemBytes = 0;
     cfg.stream = static_cast<cudaStream_t>(stream);
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = CL;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     cudaError_t e;
     if (vec)
         e = cudaLaunchKernelEx(&cfg, find_candidates_kernel<true>, ids, ids_stride, seq_len, T_cap,

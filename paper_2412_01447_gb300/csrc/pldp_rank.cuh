@@ -36,12 +36,26 @@ struct Batch {
     int n_local, P, G, slot, sub;
 };
 
-__device__ __forceinline__ Batch batch_shape(int n, int S, int rank) {
-    const int warp = threadIdx.x >> 5;
+// A group of NW warps (first warp w0) that ranks on its own, synchronising on
+// named barrier `bar` (0 = the whole CTA, i.e. __syncthreads when NW = 8).
+struct WarpGroup {
+    int w0, nw, bar;
+    __device__ __forceinline__ int warp() const { return (static_cast<int>(threadIdx.x) >> 5) - w0; }
+    __device__ __forceinline__ void sync() const {
+        asm volatile("bar.sync %0, %1;" ::"r"(bar), "r"(nw * 32) : "memory");
+    }
+};
+
+__device__ __forceinline__ WarpGroup whole_cta() { return WarpGroup{0, kRankWarps, 0}; }
+
+__device__ __forceinline__ Batch batch_shape(int n, int S, int rank, const WarpGroup& wg) {
+    const int warp = wg.warp();
+    const int pmax = wg.nw;   // 8 or 4
     Batch bt;
     bt.n_local = (n > rank) ? (n - rank + S - 1) / S : 0;
-    bt.P = bt.n_local >= 8 ? 8 : (bt.n_local >= 4 ? 4 : (bt.n_local >= 2 ? 2 : 1));
-    bt.G = kRankWarps / bt.P;
+    bt.P = (bt.n_local >= 8 && pmax >= 8) ? 8 : (bt.n_local >= 4 ? 4 : (bt.n_local >= 2 ? 2 : 1));
+    if (bt.P > pmax) bt.P = pmax;
+    bt.G = wg.nw / bt.P;
     bt.slot = warp / bt.G;
     bt.sub = warp - bt.slot * bt.G;
     return bt;
@@ -96,10 +110,11 @@ __device__ __forceinline__ void accum16<float>(const uint4& a, const uint4& q, f
 }
 
 // cos = dot / sqrt(|a|^2 |q|^2); a zero norm gives 0 (the library's stated reading).
+// fp32 throughout (the double-precision units of this GPU are few); the two
+// reciprocal square roots keep the product of the norms from overflowing.
 __device__ __forceinline__ float finish_cosine(float dot, float na, float nq) {
     if (na == 0.0f || nq == 0.0f) return 0.0f;
-    return static_cast<float>(static_cast<double>(dot) /
-                              sqrt(static_cast<double>(na) * static_cast<double>(nq)));
+    return dot * rsqrtf(na) * rsqrtf(nq);
 }
 
 // Eq. 3 for this CTA's candidates.  `hb` is the sequence's hidden slice, `cands`
@@ -108,21 +123,24 @@ __device__ __forceinline__ float finish_cosine(float dot, float na, float nq) {
 // Scores go to scores_row[i] (if given); keys of eligible candidates to
 // sh.slot_key.  CTA-uniform call; `jpre` (optional, shared) holds the first
 // batch's positions.  Returns with sh.err set if the query never arrived.
-template <typename T, bool VEC>
+// With CANDS_SHARED the candidate list is in shared memory (else global, read
+// through L2 since other CTAs of the cluster may have just written it).
+template <typename T, bool VEC, bool CANDS_SHARED = false>
 __device__ __forceinline__ void hidden_rank_cta(const T* __restrict__ hb, int64_t d, int64_t t,
                                                 const int32_t* __restrict__ cands, int n, int S,
                                                 int rank, const int32_t* jpre, const T* q_sh,
                                                 uint64_t* bar, bool q_pending, float threshold,
-                                                float* __restrict__ scores_row, RankShared& sh) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const Batch bt = batch_shape(n, S, rank);
+                                                float* __restrict__ scores_row, RankShared& sh,
+                                                const WarpGroup& wg = whole_cta()) {
+    const int lane = threadIdx.x & 31, warp = wg.warp();
+    const Batch bt = batch_shape(n, S, rank, wg);
     bool q_ready = !q_pending, timed_out = false;
     for (int k0 = 0; k0 < bt.n_local; k0 += bt.P) {
         const int k = k0 + bt.slot;
         const bool active = k < bt.n_local;
         const int i = rank + S * k;
         int64_t j = -1;
-        if (active) j = (k0 == 0 && jpre) ? jpre[k] : __ldcg(cands + i);
+        if (active) j = (k0 == 0 && jpre) ? jpre[k] : (CANDS_SHARED ? cands[i] : __ldcg(cands + i));
         const bool ok = active && j >= 1 && j < t;
         float dot = 0.f, na = 0.f, nq = 0.f;
         if (ok) {
@@ -170,7 +188,7 @@ __device__ __forceinline__ void hidden_rank_cta(const T* __restrict__ hb, int64_
             sh.part[warp][2] = nq;
         }
         if (__any_sync(0xFFFFFFFFu, timed_out) && lane == 0) sh.err = 1;
-        __syncthreads();
+        wg.sync();
         if (bt.sub == 0 && lane == 0 && active) {
             float s = -INFINITY;
             if (ok) {
@@ -188,8 +206,8 @@ __device__ __forceinline__ void hidden_rank_cta(const T* __restrict__ hb, int64_
                 if (key > sh.slot_key[bt.slot]) sh.slot_key[bt.slot] = key;
             }
         }
-        __syncthreads();
-        if (sh.err) break;                                // CTA-uniform after the barrier
+        wg.sync();
+        if (sh.err) break;                                // group-uniform after the barrier
     }
 }
 
@@ -201,21 +219,24 @@ __device__ __forceinline__ float load_attn(const void* base, int64_t idx, bool a
 
 // Eq. 2 for this CTA's candidates.  `rows_sh` (shared) holds the element offset
 // of each selected row, or -1 for an invalid one.  Same conventions as
-// hidden_rank_cta; every candidate in [0, t) is eligible.
+// hidden_rank_cta; every candidate in [0, t) is eligible.  With CANDS_SHARED
+// the candidate list is in shared memory (else global, read through L2).
+template <bool CANDS_SHARED = false>
 __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
                                                    const int64_t* rows_sh, int n_sel, int64_t t,
                                                    const int32_t* __restrict__ cands, int n, int S,
                                                    int rank, const int32_t* jpre, bool is_max,
-                                                   float* __restrict__ scores_row, RankShared& sh) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const Batch bt = batch_shape(n, S, rank);
+                                                   float* __restrict__ scores_row, RankShared& sh,
+                                                   const WarpGroup& wg = whole_cta()) {
+    const int lane = threadIdx.x & 31, warp = wg.warp();
+    const Batch bt = batch_shape(n, S, rank, wg);
     constexpr int U = 4;
     for (int k0 = 0; k0 < bt.n_local; k0 += bt.P) {
         const int k = k0 + bt.slot;
         const bool active = k < bt.n_local;
         const int i = rank + S * k;
         int64_t j = -1;
-        if (active) j = (k0 == 0 && jpre) ? jpre[k] : __ldcg(cands + i);
+        if (active) j = (k0 == 0 && jpre) ? jpre[k] : (CANDS_SHARED ? cands[i] : __ldcg(cands + i));
         const bool ok = active && j >= 0 && j < t;
         float acc = is_max ? -INFINITY : 0.0f;
         if (ok) {
@@ -240,7 +261,7 @@ __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
             acc = warp_sum(acc);
         }
         if (lane == 0) sh.part[warp][0] = acc;
-        __syncthreads();
+        wg.sync();
         if (bt.sub == 0 && lane == 0 && active) {
             float s = -INFINITY;
             if (ok) {
@@ -254,7 +275,7 @@ __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
                 if (key > sh.slot_key[bt.slot]) sh.slot_key[bt.slot] = key;
             }
         }
-        __syncthreads();
+        wg.sync();
     }
 }
 

@@ -42,23 +42,40 @@ __device__ __forceinline__ void count_hit(int (&c)[PLDP_MAX_NGRAM], int m) {
     for (int k = 0; k < PLDP_MAX_NGRAM; ++k) c[k] += (k < m) ? 1 : 0;
 }
 
+// Where pass 1 and pass 2 read the ids from: global memory (16-byte or 4-byte
+// loads) or a copy of the CTA's chunk staged in shared memory (`base` = ids of
+// positions c0, c0 + 1, ...).  `load4(q)` returns positions 4q .. 4q + 3.
+struct GlobalIds {
+    const int32_t* row;
+    __device__ __forceinline__ int4 load4(int64_t q) const {
+        return __ldg(reinterpret_cast<const int4*>(row) + q);
+    }
+};
+struct SharedIds {
+    const int32_t* base;   // shared memory, 16-byte aligned
+    int64_t q0;            // first int4 index of the staged chunk (c0 / 4)
+    __device__ __forceinline__ int4 load4(int64_t q) const {
+        return reinterpret_cast<const int4*>(base)[q - q0];
+    }
+};
+
 // Pass 1 over positions [c0, c1) (c0 a multiple of 4 when VEC; all < t):
-// c[k] += number of positions whose match length exceeds k.
-template <bool VEC>
-__device__ __forceinline__ void scan_count(const int32_t* __restrict__ row, int64_t c0, int64_t c1,
-                                           int64_t t, int n_max, int (&c)[PLDP_MAX_NGRAM]) {
+// c[k] += number of positions whose match length exceeds k.  With VEC the ids
+// come through `src` (16-byte units); otherwise 4-byte global loads from `row`.
+template <bool VEC, typename Src>
+__device__ __forceinline__ void scan_count(const Src& src, const int32_t* __restrict__ row, int64_t c0,
+                                           int64_t c1, int64_t t, int n_max, int (&c)[PLDP_MAX_NGRAM]) {
     if (c0 >= c1) return;
     const int tid = threadIdx.x;
     const int32_t xt = __ldg(row + t);
     if constexpr (VEC) {
-        const int4* row4 = reinterpret_cast<const int4*>(row);
         const int64_t q0 = c0 >> 2, q1 = (c1 + 3) >> 2;
         for (int64_t qb = q0 + tid; qb < q1; qb += static_cast<int64_t>(kScanThreads) * kScanUnroll) {
             int4 v[kScanUnroll];
 #pragma unroll
             for (int u = 0; u < kScanUnroll; ++u) {
                 const int64_t q = qb + static_cast<int64_t>(u) * kScanThreads;
-                if (q < q1) v[u] = __ldg(row4 + q);
+                if (q < q1) v[u] = src.load4(q);
             }
 #pragma unroll
             for (int u = 0; u < kScanUnroll; ++u) {
@@ -138,10 +155,16 @@ __device__ __forceinline__ void scan_decide(cg::cluster_group& cluster, ScanShar
 
 // Pass 2: writes this CTA's matches of length >= nstar, in ascending order, to
 // dst[sh.offset ...] (entries at or past C_cap are dropped).  CTA-uniform call.
-template <bool VEC>
-__device__ __forceinline__ void scan_write(const int32_t* __restrict__ row, int64_t c0, int64_t c1,
-                                           int64_t t, int n_max, ScanShared& sh,
-                                           int32_t* __restrict__ dst, int C_cap) {
+// `on_write(j)` is called by the thread that writes position j.
+struct NoHook {
+    __device__ __forceinline__ void operator()(int64_t) const {}
+};
+
+template <bool VEC, typename Src, typename Hook = NoHook>
+__device__ __forceinline__ void scan_write(const Src& src, const int32_t* __restrict__ row, int64_t c0,
+                                           int64_t c1, int64_t t, int n_max, ScanShared& sh,
+                                           int32_t* __restrict__ dst, int C_cap,
+                                           const Hook& on_write = Hook()) {
     const int nstar = sh.nstar, mine = sh.mine;
     int64_t out = sh.offset;
     if (!(nstar > 0 && mine > 0 && out < C_cap)) return;
@@ -156,7 +179,7 @@ __device__ __forceinline__ void scan_write(const int32_t* __restrict__ row, int6
         if (g < g1) {
             int32_t e[G];
             if constexpr (VEC) {
-                const int4 v = __ldg(reinterpret_cast<const int4*>(row) + g);
+                const int4 v = src.load4(g);
                 e[0] = v.x;
                 e[1] = v.y;
                 e[2] = v.z;
@@ -190,7 +213,10 @@ __device__ __forceinline__ void scan_write(const int32_t* __restrict__ row, int6
         while (mask) {
             const int k = __ffs(mask) - 1;
             mask &= mask - 1;
-            if (pos < C_cap) dst[pos] = static_cast<int32_t>(g * G + k);
+            if (pos < C_cap) {
+                dst[pos] = static_cast<int32_t>(g * G + k);
+                on_write(g * G + k);
+            }
             ++pos;
         }
         out += tile;

@@ -97,6 +97,7 @@ rank_hidden_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride,
     __shared__ CtaBest mine;
     __shared__ __align__(8) uint64_t bar;
 
+    pdl_enter();
     const int b = blockIdx.x / S;
     const int rank = blockIdx.x - b * S;
     const int tid = threadIdx.x;
@@ -156,6 +157,7 @@ rank_attention_kernel(const void* __restrict__ A, bool a_bf16, int R, int64_t ro
     __shared__ CtaBest mine;
     __shared__ int bad_rows;
 
+    pdl_enter();
     const int b = blockIdx.x / S;
     const int rank = blockIdx.x - b * S;
     const int tid = threadIdx.x;
@@ -198,13 +200,15 @@ cudaError_t launch_rank(K kernel, int B, int S, size_t smem, void* stream, Args.
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = static_cast<cudaStream_t>(stream);
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = S;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = S;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = S > 1 ? 1 : 0;
+    cfg.numAttrs = S > 1 ? 2 : 1;
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              static_cast<int>(smem));

@@ -33,6 +33,7 @@ __global__ void extract_draft_kernel(const int32_t* __restrict__ ids, int64_t id
                                      const int32_t* __restrict__ seq_len, int64_t T_cap,
                                      const int32_t* __restrict__ best_pos, int B, int K,
                                      int32_t* __restrict__ draft, int32_t* __restrict__ draft_len) {
+    pdl_enter();
     const int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
     if (idx >= static_cast<int64_t>(B) * K) return;
     const int b = static_cast<int>(idx / K);
@@ -204,6 +205,7 @@ __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads, kMinBlocksPerSm)
 verify_greedy_kernel(const T* __restrict__ logits, VerifyArgs a) {
+    pdl_enter();
     const int lane = threadIdx.x & 31;
     const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
     if (w >= a.total_warps) return;
@@ -264,8 +266,10 @@ pldp_status launch_verify_t(const void* logits, VerifyArgs a, void* scratch, cud
     a.row_keys = static_cast<unsigned long long*>(scratch);
     a.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(scratch) + keys_bytes(a.B, a.K));
     const unsigned blocks = static_cast<unsigned>((a.total_warps + kWarps - 1) / kWarps);
-    verify_greedy_kernel<T, VEC><<<blocks, kThreads, 0, s>>>(static_cast<const T*>(logits), a);
-    return check_launch(what);
+    const cudaError_t e = launch_pdl(verify_greedy_kernel<T, VEC>, dim3(blocks), dim3(kThreads), 0, s, 0,
+                                     static_cast<const T*>(logits), a);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
+    return PLDP_OK;
 }
 
 pldp_status launch_verify(const void* logits, pldp_dtype dtype, const VerifyArgs& a, void* scratch,
@@ -326,9 +330,12 @@ extern "C" PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t i
     const int64_t n = static_cast<int64_t>(B) * K;
     const int64_t blocks = (n + 255) / 256;
     if (blocks > INT32_MAX) return fail(PLDP_ERR_INVALID_ARG, "extract_draft: B*K too large");
-    extract_draft_kernel<<<static_cast<unsigned>(blocks), 256, 0, static_cast<cudaStream_t>(stream)>>>(
-        ids, ids_stride, seq_len, T_cap, best_pos, B, K, draft, draft_len);
-    return check_launch("extract_draft");
+    const cudaError_t e = launch_pdl(extract_draft_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0,
+                                     static_cast<cudaStream_t>(stream), 0, ids, ids_stride, seq_len, T_cap,
+                                     best_pos, B, K, draft, draft_len);
+    if (e != cudaSuccess)
+        return fail(PLDP_ERR_CUDA, "extract_draft: launch failed: %s", cudaGetErrorString(e));
+    return PLDP_OK;
 }
 
 extern "C" PLDP_API pldp_status pldp_verify_greedy(

@@ -47,6 +47,7 @@ class Buffers:
         self.nxt = torch.zeros(B, **i32)
         self.kv = torch.zeros(B, **i32)
         self.ws = torch.zeros(pk.pldp_verify_workspace_size(B, K, V), dtype=torch.uint8, device=device)
+        self.dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=device)
 
 
 def gpu_step(buf, ids, seq_len, logits, ngram=(1, 3), H=None, A=None, row_idx=None,
@@ -58,7 +59,7 @@ def gpu_step(buf, ids, seq_len, logits, ngram=(1, 3), H=None, A=None, row_idx=No
         ri = None if row_idx is None or A is None else torch.as_tensor(row_idx, dtype=torch.int32,
                                                                         device=A.device)
         pk.pldp_draft_step(ids, seq_len, ngram[0], ngram[1], buf.cand, buf.cnt, buf.ml, buf.draft.shape[1],
-                           buf.draft, buf.dlen, H=H, best_h=buf.best_h if H is not None else None,
+                           buf.draft, buf.dlen, buf.dws, H=H, best_h=buf.best_h if H is not None else None,
                            h_scores=buf.scores_h, best_h_score=buf.bscore_h, threshold=threshold, A=A,
                            best_a=buf.best_a if A is not None else None, row_idx=ri, agg=agg,
                            a_scores=buf.scores_a, best_a_score=buf.bscore_a, draft_from=draft_from,
@@ -93,7 +94,7 @@ def gpu_step(buf, ids, seq_len, logits, ngram=(1, 3), H=None, A=None, row_idx=No
 
 def snapshot(buf):
     torch.cuda.synchronize()
-    return {k: host(v) for k, v in vars(buf).items() if k != "ws"}
+    return {k: host(v) for k, v in vars(buf).items() if k not in ("ws", "dws")}
 
 
 def check_scores(g_scores, o_scores, cnt, C_cap, rows=None):

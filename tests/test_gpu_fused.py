@@ -42,7 +42,10 @@ def _compare(g, ids0, L0, H, A, row_idx, agg, ngram, C, K, draft_from, thr=float
     assert np.array_equal(g["status"].view(np.uint32), st)
 
 
-@pytest.mark.parametrize("T,V,B", [(300, 5, 12), (4096, 50, 8), (20000, 7, 3), (36096, 3000, 16)])
+# B >= half the SMs with contexts up to 40k tokens take the one-CTA-per-sequence kernel
+# (whole context in shared memory); smaller batches take the cluster kernel.
+@pytest.mark.parametrize("T,V,B", [(300, 5, 12), (4096, 50, 8), (20000, 7, 3), (36096, 3000, 16),
+                                   (3000, 5, 96), (5000, 40, 96), (36096, 3000, 96), (2048, 2, 80)])
 @pytest.mark.parametrize("mode", ["both", "hidden", "attention"])
 def test_draft_step_random(lib, T, V, B, mode):
     rng = np.random.default_rng(T + V)
