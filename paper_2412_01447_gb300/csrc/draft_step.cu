@@ -11,6 +11,8 @@
 //  1. scan: a flat grid of (chunk, sequence) CTAs streams the contexts with
 //     16-byte loads and appends every occurrence j of x_t, with its suffix-match
 //     length m, to a short per-sequence list in the workspace ((j << 4) | m).
+//     It also starts pulling into L2 what the rank kernel will read for each
+//     occurrence (its hidden row, its attention values) and the query row.
 //  2. rank: one CTA per sequence reads its list, takes n* = the largest m, orders
 //     the occurrences with m >= n* by position (the candidate list), scores them
 //     by hidden states on half its warps while the other half scores attentions,
@@ -54,6 +56,7 @@ struct DraftParams {
     int32_t* cand_count;
     int32_t* match_len;
     const void* H;
+    bool h_bf16;
     int64_t d;
     int64_t h_seq_stride;
     float threshold;
@@ -88,6 +91,33 @@ __device__ __forceinline__ int32_t* hit_list(unsigned char* ws, int b) {
 }
 
 // ---- 1. scan -----------------------------------------------------------------------
+__device__ __forceinline__ void prefetch_l2_bulk(const void* ptr, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void prefetch_l2(const void* ptr) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(ptr));
+}
+
+// The rank kernel reads, per occurrence j, the hidden row H_{j-1} and the
+// attention values A[r, j]; the scan finds j several microseconds earlier, so the
+// warp that found it starts pulling those lines into L2 (and their address
+// translations into the TLBs) right away.  Warp-uniform call.
+__device__ __forceinline__ void prefetch_candidate(const DraftParams& p, int b, int64_t j, int lane) {
+    if (p.H && j >= 1 && lane == 0) {
+        const size_t es = p.h_bf16 ? 2 : 4;
+        const char* hrow = static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (j - 1) * p.d) * es;
+        prefetch_l2_bulk(hrow, static_cast<uint32_t>(p.d * es));
+    }
+    if (p.A) {
+        const size_t es = p.a_bf16 ? 2 : 4;
+        const char* ab = static_cast<const char*>(p.A) + static_cast<int64_t>(b) * p.a_seq_stride * es;
+        for (int k = lane; k < p.n_sel; k += 32) {
+            const int r = p.row_idx ? __ldg(p.row_idx + k) : k;
+            if (r >= 0 && r < p.R) prefetch_l2(ab + (static_cast<int64_t>(r) * p.a_row_stride + j) * es);
+        }
+    }
+}
+
 template <bool VEC>
 __global__ void __launch_bounds__(kThreads) draft_scan_kernel(const DraftParams p) {
     pdl_enter();
@@ -95,17 +125,20 @@ __global__ void __launch_bounds__(kThreads) draft_scan_kernel(const DraftParams 
     const int64_t L = p.seq_len[b];
     if (L < 2 || L > p.T_cap) return;                 // nothing to find; the rank kernel reports
     const int64_t t = L - 1;
+    const int tid = threadIdx.x, lane = tid & 31;
+    if (blockIdx.x == 0 && tid == 0 && p.H && t >= 2) {   // the query row H_{t-1}, for the rank kernel
+        const size_t es = p.h_bf16 ? 2 : 4;
+        prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (t - 1) * p.d) * es,
+                         static_cast<uint32_t>(p.d * es));
+    }
     const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kChunk;
     const int64_t c1 = c0 + kChunk < t ? c0 + kChunk : t;
     if (c0 >= c1) return;
     const int32_t* row = p.ids + static_cast<int64_t>(b) * p.ids_stride;
     const int32_t xt = __ldg(row + t);
-    const int tid = threadIdx.x;
-    auto hit = [&](int64_t j) {
-        const int m = suffix_match(row, j, t, p.ngram_max);
-        const unsigned slot = atomicAdd(hit_count(p.ws, b), 1u);
-        if (slot < kHitCap) hit_list(p.ws, b)[slot] = static_cast<int32_t>((j << 4) | m);
-    };
+
+    // Each thread covers 4 * kScanVec positions; bit i of `mask` marks its i-th.
+    uint32_t mask = 0;
     if constexpr (VEC) {
         const int4* row4 = reinterpret_cast<const int4*>(row);
         const int64_t q0 = c0 >> 2, q1 = (c1 + 3) >> 2;
@@ -122,7 +155,7 @@ __global__ void __launch_bounds__(kThreads) draft_scan_kernel(const DraftParams 
             const int32_t e[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
             for (int k = 0; k < 4; ++k)
-                if (e[k] == xt && 4 * q + k < c1) hit(4 * q + k);
+                if (e[k] == xt && 4 * q + k < c1) mask |= 1u << (4 * u + k);
         }
     } else {
         int32_t v[kScanVec * 4];
@@ -134,8 +167,32 @@ __global__ void __launch_bounds__(kThreads) draft_scan_kernel(const DraftParams 
 #pragma unroll
         for (int u = 0; u < kScanVec * 4; ++u) {
             const int64_t j = c0 + tid + u * kThreads;
-            if (j < c1 && v[u] == xt) hit(j);
+            if (j < c1 && v[u] == xt) mask |= 1u << u;
         }
+    }
+    // Occurrences, one at a time per warp: prefetch for the rank kernel, then record.
+    unsigned pending = __ballot_sync(0xFFFFFFFFu, mask != 0);
+    while (pending) {
+        const int src = __ffs(pending) - 1;
+        const uint32_t m_src = __shfl_sync(0xFFFFFFFFu, mask, src);
+        const int bit = __ffs(m_src) - 1;
+        int64_t j;
+        if constexpr (VEC) {
+            const int64_t q = (c0 >> 2) + (tid - lane + src) + (bit >> 2) * kThreads;
+            j = 4 * q + (bit & 3);
+        } else {
+            j = c0 + (tid - lane + src) + static_cast<int64_t>(bit) * kThreads;
+        }
+        unsigned slot = 0;
+        if (lane == src) {
+            const int m = suffix_match(row, j, t, p.ngram_max);
+            slot = atomicAdd(hit_count(p.ws, b), 1u);
+            if (slot < kHitCap) hit_list(p.ws, b)[slot] = static_cast<int32_t>((j << 4) | m);
+            mask &= mask - 1;
+        }
+        // Past kHitCap the rank kernel rescans; prefetching stops there too.
+        if (__shfl_sync(0xFFFFFFFFu, slot, src) < kHitCap) prefetch_candidate(p, b, j, lane);
+        pending = __ballot_sync(0xFFFFFFFFu, mask != 0);
     }
 }
 
@@ -437,6 +494,7 @@ extern "C" PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* a, v
     p.cand_count = a->cand_count;
     p.match_len = a->match_len;
     p.H = a->H;
+    p.h_bf16 = a->h_dtype == PLDP_BF16;
     p.d = a->d;
     p.h_seq_stride = a->h_seq_stride;
     p.threshold = a->threshold;
