@@ -56,6 +56,9 @@ def parse():
     ap.add_argument("--flush", choices=["write-read", "write"], default="write-read",
                     help="L2 flush before each step: write 256 MB then read 256 MB (cold, clean L2), "
                          "or the write alone (cold L2 full of dirty lines)")
+    ap.add_argument("--events", choices=["kernel", "step"], default="kernel",
+                    help="CUDA events around every kernel (per-kernel times, the roofline) or only "
+                         "around each step (kernels chained by programmatic dependent launch)")
     ap.add_argument("--separate", action="store_true",
                     help="draft with the four separate calls instead of the fused launch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -210,15 +213,19 @@ class Path:
         self.kernels = (["draft_step"] if fused else
                         ["find_candidates", "rank_hidden", "rank_attention", "extract_draft"]) + ["verify_greedy"]
 
-    def run(self, ev=None, stream=None):
+    def run(self, ev=None, stream=None, step_only=False):
         """One step: the drafting half (one fused launch, or the four separate calls)
-        then verification.  ev: events recorded before the first and after every kernel."""
+        then verification.  ev: events recorded before the first and after every kernel
+        (step_only: before the first and after the last only)."""
         pk, lp, w = self.pk, self.loop, self.loop.w
         s = torch.cuda.current_stream() if stream is None else stream
         k = [0]
+        n_rec = [0]
+        n_total = len(self.kernels) + 1
 
         def rec():
-            if ev is not None:
+            n_rec[0] += 1
+            if ev is not None and (not step_only or n_rec[0] in (1, n_total)):
                 ev[k[0]].record(s)
                 k[0] += 1
 
@@ -312,7 +319,7 @@ def run_ours(args, ws_, rank, local):
         loop.step_inputs(W_steps + s)
         len_sum += loop.seq_len.sum()
         flush_l2(s)
-        path.run(evs[s])
+        path.run(evs[s], step_only=args.events == "step")
         cand_sum += path.cnt.clamp(max=w.C_cap).sum()
         acc_sum += path.acc.sum()
     torch.cuda.synchronize()
@@ -321,10 +328,14 @@ def run_ours(args, ws_, rank, local):
     clk = clocks.stop()
 
     per_k = np.zeros(nk)
-    for e in evs:
-        for k in range(nk):
-            per_k[k] += e[k].elapsed_time(e[k + 1])
-    step_ms_total = float(per_k.sum())                        # device ms over K steps
+    if args.events == "step":                                 # no per-kernel split in this mode
+        step_ms_total = float(sum(e[0].elapsed_time(e[1]) for e in evs))
+        per_k[:] = np.nan
+    else:
+        for e in evs:
+            for k in range(nk):
+                per_k[k] += e[k].elapsed_time(e[k + 1])
+        step_ms_total = float(per_k.sum())                    # device ms over K steps
     step_ms_total = max_over_ranks(step_ms_total, ws_)
     ms_per_step = step_ms_total / K_steps
     value = ws_ * K_steps / (step_ms_total / 1e3)
@@ -445,6 +456,17 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
                       "calls, D2H of accept/next/seq_len/draft, synchronize"}
 
 
+def _finite(x):
+    """NaN / inf (a figure the chosen timing mode does not give) -> null."""
+    if isinstance(x, dict):
+        return {k: _finite(v) for k, v in x.items()}
+    if isinstance(x, (list, tuple)):
+        return [_finite(v) for v in x]
+    if isinstance(x, float) and not np.isfinite(x):
+        return None
+    return x
+
+
 def _host(t):
     if t.dtype == torch.bfloat16:
         return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
@@ -538,7 +560,7 @@ def main():
         return
     out = run_ours(args, ws_, rank, local)
     if rank == 0:
-        print(json.dumps(out))
+        print(json.dumps(_finite(out)))
 
 
 if __name__ == "__main__":

@@ -191,12 +191,14 @@ PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
  * bits and a tie within rounding may be broken differently).  Eq. 1-3
  * (Sec. 4.2) and Sec. 4.3.
  *
- * Two short kernels: a flat (chunk, sequence) grid streams the contexts and
- * records every occurrence of x_t with its suffix-match length in a small
- * per-sequence list held in the workspace; then one CTA per sequence orders the
- * list into the candidate list, ranks it and writes the draft (the query row
- * H_{t-1} is fetched by a bulk copy at that kernel's entry).  More than 256
- * occurrences in a sequence fall back to an ordered rescan of its context.
+ * One launch over a flat (chunk, sequence) grid.  Each CTA streams its chunk of
+ * the context, scores every occurrence of x_t it finds (cosine and attention
+ * score, with all its threads) and records it with its suffix-match length in a
+ * small per-sequence list held in the workspace; the CTA that finishes a
+ * sequence last (an atomic ticket, no waiting) orders the list into the
+ * candidate list, picks the best of each ranking and writes the draft.  More
+ * than 256 occurrences in a sequence fall back to an ordered rescan of its
+ * context by that CTA.
  *
  * Fields of the argument block (device pointers unless stated):
  *  ids .. match_len      as pldp_find_candidates (T_cap <= 2^27).

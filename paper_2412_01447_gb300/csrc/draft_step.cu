@@ -1,31 +1,31 @@
 // pldp_draft_step: the drafting half of a PLD+ step -- candidate search (Eq. 1
 // with the longest-suffix n-gram rule), ranking by hidden states (Eq. 3) and/or
-// by attentions (Eq. 2), and draft extraction (Sec. 4.3) -- in two short kernels.
+// by attentions (Eq. 2), and draft extraction (Sec. 4.3) -- in one launch.
 //
-// Both kernels are kept small on purpose.  Between decode steps the model's own
-// traffic evicts this library's code from L2, so every distinct stretch of code a
-// CTA reaches costs an instruction fetch from DRAM; a long multi-phase kernel with
-// one CTA per SM pays that many times in series.  Short straight-line kernels
-// with many CTAs pay it once, in parallel.
+// A flat grid of (chunk, sequence) CTAs.  Each CTA
+//  1. streams its chunk of the context with 16-byte loads and, for every
+//     occurrence j of x_t, takes the suffix-match length m and a slot in a short
+//     per-sequence list held in the workspace;
+//  2. scores each occurrence it found with all its threads -- cos(H_{j-1},
+//     H_{t-1}) and the max (or sum) of the selected attention rows at key j, both
+//     in one round trip to memory -- and stores (j, m, scores) in the slot;
+//  3. takes a ticket.  The CTA that takes a sequence's last ticket finishes it:
+//     it reads the list, takes n* = the largest m, orders the occurrences with
+//     m >= n* by position (the candidate list), picks the best of each ranking
+//     from the stored scores, writes the draft, and returns the list's header to
+//     zero for the next call.
+// No CTA waits for another.  Occurrences are scored before n* is known, so
+// those with m < n* are scored for nothing; they are few.  A list that
+// overflowed (more than kHitCap occurrences) is redone by the finishing CTA: an
+// ordered rescan of the context, then the same scorer per candidate.
 //
-//  1. scan: a flat grid of (chunk, sequence) CTAs streams the contexts with
-//     16-byte loads and appends every occurrence j of x_t, with its suffix-match
-//     length m, to a short per-sequence list in the workspace ((j << 4) | m).
-//     It also starts pulling into L2 what the rank kernel will read for each
-//     occurrence (its hidden row, its attention values) and the query row.
-//  2. rank: one CTA per sequence reads its list, takes n* = the largest m, orders
-//     the occurrences with m >= n* by position (the candidate list), scores them
-//     by hidden states on half its warps while the other half scores attentions,
-//     and writes the draft.  It returns
-//     the list's count to zero for the next call.  A list that overflowed (more
-//     than kHitCap occurrences) is redone by an ordered rescan of the context
-//     inside the CTA.
-//
-// The query row H_{t-1} depends only on seq_len: the rank kernel's bulk copy of
-// it into shared memory is issued at entry and lands while the list is read.
-// Results are those of pldp_find_candidates, pldp_rank_hidden,
-// pldp_rank_attention and pldp_extract_draft called in turn (fp32 score sums may
-// be split differently, so scores can differ in their last bits).
+// Every score comes from the same CTA-wide reduction (a fixed share per thread,
+// partial sums combined in warp order), whichever CTA computes it, so results
+// are deterministic.  Results are those of pldp_find_candidates,
+// pldp_rank_hidden, pldp_rank_attention and pldp_extract_draft called in turn
+// (fp32 score sums are split differently, so scores can differ in their last
+// bits).
+#include <climits>
 #include <type_traits>
 
 #include "pldp_rank.cuh"
@@ -35,13 +35,18 @@ namespace pldp {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kScanVec = 8;                                    // int4 loads per scan thread
-constexpr int64_t kChunk = int64_t(kThreads) * kScanVec * 4;   // positions per scan CTA
+constexpr int kWarps = kThreads / 32;
+constexpr int kScanVec = 9;                                    // int4 loads per scan thread
+constexpr int64_t kChunk = int64_t(kThreads) * kScanVec * 4;   // positions per CTA
 constexpr int kHitCap = 256;                                   // occurrences kept per sequence
-constexpr size_t kSeqWs = 16 + kHitCap * 4;                    // workspace bytes per sequence
+constexpr size_t kSeqWs = 16 + kHitCap * 16;                   // header + 16-byte entries
+constexpr int kScoreUnroll = 2;                                // 16-byte row loads in flight
+constexpr int kScoreBatch = 2;                                 // occurrences scored per pass
 constexpr size_t kMaxQueryBytes = 196608;
 constexpr int kMaxSelRows = 8192;
 constexpr int64_t kMaxPositions = int64_t(1) << 27;            // (j << 4) | m fits 31 bits
+
+static_assert(kHitCap <= kThreads, "the finish gives each list entry its own thread");
 
 struct NoHidden {};
 
@@ -79,175 +84,349 @@ struct DraftParams {
     int32_t* draft;
     int32_t* draft_len;
     uint32_t* status;
-    unsigned char* ws;    // kSeqWs per sequence: the count (u32), then kHitCap entries
-    size_t rows_offset;   // byte offset of the attention row table in dynamic shared memory
+    unsigned char* ws;    // kSeqWs per sequence: count, ticket (u32 each), pad; entries
 };
 
-__device__ __forceinline__ unsigned* hit_count(unsigned char* ws, int b) {
+// Workspace of sequence b: header[0] = occurrences recorded, header[1] = tickets
+// taken; entry i = ((j << 4) | m, hidden score bits, attention score bits, 0).
+__device__ __forceinline__ unsigned* seq_header(unsigned char* ws, int b) {
     return reinterpret_cast<unsigned*>(ws + static_cast<size_t>(b) * kSeqWs);
 }
-__device__ __forceinline__ int32_t* hit_list(unsigned char* ws, int b) {
-    return reinterpret_cast<int32_t*>(ws + static_cast<size_t>(b) * kSeqWs + 16);
+__device__ __forceinline__ uint4* seq_entries(unsigned char* ws, int b) {
+    return reinterpret_cast<uint4*>(ws + static_cast<size_t>(b) * kSeqWs + 16);
 }
 
-// ---- 1. scan -----------------------------------------------------------------------
 __device__ __forceinline__ void prefetch_l2_bulk(const void* ptr, uint32_t bytes) {
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ void prefetch_l2(const void* ptr) {
-    asm volatile("prefetch.global.L2 [%0];" ::"l"(ptr));
+
+__device__ __forceinline__ float warp_max_f(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+    return v;
 }
 
-// The rank kernel reads, per occurrence j, the hidden row H_{j-1} and the
-// attention values A[r, j]; the scan finds j several microseconds earlier, so the
-// warp that found it starts pulling those lines into L2 (and their address
-// translations into the TLBs) right away.  Warp-uniform call.
-__device__ __forceinline__ void prefetch_candidate(const DraftParams& p, int b, int64_t j, int lane) {
-    if (p.H && j >= 1 && lane == 0) {
-        const size_t es = p.h_bf16 ? 2 : 4;
-        const char* hrow = static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (j - 1) * p.d) * es;
-        prefetch_l2_bulk(hrow, static_cast<uint32_t>(p.d * es));
-    }
-    if (p.A) {
-        const size_t es = p.a_bf16 ? 2 : 4;
-        const char* ab = static_cast<const char*>(p.A) + static_cast<int64_t>(b) * p.a_seq_stride * es;
-        for (int k = lane; k < p.n_sel; k += 32) {
-            const int r = p.row_idx ? __ldg(p.row_idx + k) : k;
-            if (r >= 0 && r < p.R) prefetch_l2(ab + (static_cast<int64_t>(r) * p.a_row_stride + j) * es);
-        }
-    }
-}
-
-template <bool VEC>
-__global__ void __launch_bounds__(kThreads) draft_scan_kernel(const DraftParams p) {
-    pdl_enter();
-    const int b = blockIdx.y;
-    const int64_t L = p.seq_len[b];
-    if (L < 2 || L > p.T_cap) return;                 // nothing to find; the rank kernel reports
-    const int64_t t = L - 1;
-    const int tid = threadIdx.x, lane = tid & 31;
-    if (blockIdx.x == 0 && tid == 0 && p.H && t >= 2) {   // the query row H_{t-1}, for the rank kernel
-        const size_t es = p.h_bf16 ? 2 : 4;
-        prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (t - 1) * p.d) * es,
-                         static_cast<uint32_t>(p.d * es));
-    }
-    const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kChunk;
-    const int64_t c1 = c0 + kChunk < t ? c0 + kChunk : t;
-    if (c0 >= c1) return;
-    const int32_t* row = p.ids + static_cast<int64_t>(b) * p.ids_stride;
-    const int32_t xt = __ldg(row + t);
-
-    // Each thread covers 4 * kScanVec positions; bit i of `mask` marks its i-th.
-    uint32_t mask = 0;
-    if constexpr (VEC) {
-        const int4* row4 = reinterpret_cast<const int4*>(row);
-        const int64_t q0 = c0 >> 2, q1 = (c1 + 3) >> 2;
-        int4 v[kScanVec];
-#pragma unroll
-        for (int u = 0; u < kScanVec; ++u) {
-            const int64_t q = q0 + tid + u * kThreads;
-            if (q < q1) v[u] = __ldg(row4 + q);
-        }
-#pragma unroll
-        for (int u = 0; u < kScanVec; ++u) {
-            const int64_t q = q0 + tid + u * kThreads;
-            if (q >= q1) continue;
-            const int32_t e[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-                if (e[k] == xt && 4 * q + k < c1) mask |= 1u << (4 * u + k);
-        }
-    } else {
-        int32_t v[kScanVec * 4];
-#pragma unroll
-        for (int u = 0; u < kScanVec * 4; ++u) {
-            const int64_t j = c0 + tid + u * kThreads;
-            if (j < c1) v[u] = __ldg(row + j);
-        }
-#pragma unroll
-        for (int u = 0; u < kScanVec * 4; ++u) {
-            const int64_t j = c0 + tid + u * kThreads;
-            if (j < c1 && v[u] == xt) mask |= 1u << u;
-        }
-    }
-    // Occurrences, one at a time per warp: prefetch for the rank kernel, then record.
-    unsigned pending = __ballot_sync(0xFFFFFFFFu, mask != 0);
-    while (pending) {
-        const int src = __ffs(pending) - 1;
-        const uint32_t m_src = __shfl_sync(0xFFFFFFFFu, mask, src);
-        const int bit = __ffs(m_src) - 1;
-        int64_t j;
-        if constexpr (VEC) {
-            const int64_t q = (c0 >> 2) + (tid - lane + src) + (bit >> 2) * kThreads;
-            j = 4 * q + (bit & 3);
-        } else {
-            j = c0 + (tid - lane + src) + static_cast<int64_t>(bit) * kThreads;
-        }
-        unsigned slot = 0;
-        if (lane == src) {
-            const int m = suffix_match(row, j, t, p.ngram_max);
-            slot = atomicAdd(hit_count(p.ws, b), 1u);
-            if (slot < kHitCap) hit_list(p.ws, b)[slot] = static_cast<int32_t>((j << 4) | m);
-            mask &= mask - 1;
-        }
-        // Past kHitCap the rank kernel rescans; prefetching stops there too.
-        if (__shfl_sync(0xFFFFFFFFu, slot, src) < kHitCap) prefetch_candidate(p, b, j, lane);
-        pending = __ballot_sync(0xFFFFFFFFu, mask != 0);
-    }
-}
-
-// ---- 2. rank -----------------------------------------------------------------------
-struct ListState {
-    int32_t sorted[kHitCap];   // the candidate list, in order
-    int32_t raw[kHitCap];      // the recorded occurrences, (j << 4) | m
-    int nstar, total;
+struct Hit {
+    int32_t j, m;
 };
 
-template <typename TH, bool IVEC>
-__global__ void __launch_bounds__(kThreads) draft_rank_kernel(const DraftParams p) {
-    constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
-    using TQ = typename std::conditional<HAS_H, TH, float>::type;
-    extern __shared__ __align__(128) unsigned char dyn_smem[];
-    TQ* q_sh = reinterpret_cast<TQ*>(dyn_smem);                                   // H_{t-1}
-    int64_t* rows_sh = reinterpret_cast<int64_t*>(dyn_smem + p.rows_offset);     // attention rows
-    __shared__ ListState ls;
-    __shared__ ScanShared ss;
-    __shared__ RankShared hs, as;
-    __shared__ __align__(8) uint64_t q_bar;
-    __shared__ int bad_rows;
+struct StepShared {
+    Hit hit[kHitCap];                        // occurrences this CTA found (the first kHitCap)
+    float part[2][kScoreBatch][kWarps][4];   // per-warp partial sums: dot, |a|^2, |q|^2, attention
+    int32_t jl[kHitCap];                     // finish: positions of the candidates (else INT_MAX)
+    unsigned long long wkey[2][kWarps];      // finish: per-warp best keys (hidden, attention)
+    int wmax[kWarps];
+    int32_t suf[PLDP_MAX_NGRAM];             // x_t, x_{t-1}, ... (n_max of them)
+    int nhit, skip, last;
+    ScanShared ss;                           // finish: the ordered rescan of an overflowed list
+};
 
-    pdl_enter();
-    const int b = blockIdx.x;
+// Eq. 3 and Eq. 2 for candidates j[0 .. nb) of sequence b (nb <= kScoreBatch),
+// by all threads of the CTA: thread i takes 16-byte chunks i, i + 256, ... of
+// H_{j-1} and H_{t-1} and selected rows i, i + 256, ...; partial sums meet in
+// `part` and thread 0 combines them in warp order.  The candidates of one pass
+// share the loads of H_{t-1} and are otherwise independent: a score does not
+// depend on which pass or slot computes it.  Scores are returned in thread 0:
+// the cosine (-inf when j = 0 has no H_{j-1}) and the attention max / sum.
+// CTA-uniform call with one barrier; callers alternate `part` buffers.
+template <typename TH>
+__device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int64_t (&j)[kScoreBatch], int nb,
+                                          int64_t t, float (&part)[kScoreBatch][kWarps][4],
+                                          float (&s_h)[kScoreBatch], float (&s_a)[kScoreBatch]) {
+    constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
+    constexpr int NB = kScoreBatch;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const bool is_max = p.agg == PLDP_AGG_MAX;
+    bool h_ok[NB], a_ok[NB];
+    bool any_h = false;
+#pragma unroll
+    for (int h = 0; h < NB; ++h) {
+        h_ok[h] = HAS_H && h < nb && j[h] >= 1 && j[h] < t;
+        a_ok[h] = p.A != nullptr && h < nb && j[h] >= 0 && j[h] < t;
+        any_h |= h_ok[h];
+    }
+    float dot[NB], na[NB], nq = 0.f, acc[NB];
+#pragma unroll
+    for (int h = 0; h < NB; ++h) {
+        dot[h] = 0.f;
+        na[h] = 0.f;
+        acc[h] = is_max ? -INFINITY : 0.0f;
+    }
+    if constexpr (HAS_H) {
+        if (any_h) {
+            constexpr int E = 16 / sizeof(TH);
+            const TH* hb = static_cast<const TH*>(p.H) + static_cast<int64_t>(b) * p.h_seq_stride;
+            const TH* qrow = hb + (t - 1) * p.d;                  // H_{t-1}
+            const TH* arow[NB];
+#pragma unroll
+            for (int h = 0; h < NB; ++h) arow[h] = h_ok[h] ? hb + (j[h] - 1) * p.d : qrow;   // H_{j-1}
+            const int64_t nch = p.d / E;
+            for (int64_t c0 = tid; c0 < nch; c0 += static_cast<int64_t>(kThreads) * kScoreUnroll) {
+                uint4 q[kScoreUnroll], a[NB][kScoreUnroll];
+#pragma unroll
+                for (int u = 0; u < kScoreUnroll; ++u) {
+                    const int64_t c = c0 + static_cast<int64_t>(kThreads) * u;
+                    if (c < nch) {
+                        q[u] = ld_stream16(qrow + c * E);
+#pragma unroll
+                        for (int h = 0; h < NB; ++h)
+                            if (h_ok[h]) a[h][u] = ld_stream16(arow[h] + c * E);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < kScoreUnroll; ++u) {
+                    if (c0 + static_cast<int64_t>(kThreads) * u >= nch) continue;
+                    float dead0 = 0.f, dead1 = 0.f;                 // |H_{t-1}|^2 once for the pass
+                    accum16<TH>(q[u], q[u], dead0, dead1, nq);
+#pragma unroll
+                    for (int h = 0; h < NB; ++h) {
+                        float dead2 = 0.f;
+                        if (h_ok[h]) accum16<TH>(a[h][u], q[u], dot[h], na[h], dead2);
+                    }
+                }
+            }
+        }
+    }
+    if (p.A != nullptr) {
+        const size_t es = p.a_bf16 ? 2 : 4;
+        const void* ab = static_cast<const char*>(p.A) + static_cast<int64_t>(b) * p.a_seq_stride * es;
+        for (int k = tid; k < p.n_sel; k += kThreads) {
+            const int r = p.row_idx ? __ldg(p.row_idx + k) : k;
+            const bool rv = r >= 0 && r < p.R;
+            float v[NB];
+#pragma unroll
+            for (int h = 0; h < NB; ++h)
+                v[h] = (rv && a_ok[h]) ? load_attn(ab, static_cast<int64_t>(r) * p.a_row_stride + j[h], p.a_bf16) : NAN;
+#pragma unroll
+            for (int h = 0; h < NB; ++h)
+                if (v[h] == v[h]) acc[h] = is_max ? fmaxf(acc[h], v[h]) : acc[h] + v[h];
+        }
+    }
+    if constexpr (HAS_H) nq = warp_sum(nq);
+#pragma unroll
+    for (int h = 0; h < NB; ++h) {
+        if constexpr (HAS_H) {
+            dot[h] = warp_sum(dot[h]);
+            na[h] = warp_sum(na[h]);
+        }
+        acc[h] = is_max ? warp_max_f(acc[h]) : warp_sum(acc[h]);
+        if (lane == 0) {
+            part[h][warp][0] = dot[h];
+            part[h][warp][1] = na[h];
+            part[h][warp][2] = nq;
+            part[h][warp][3] = acc[h];
+        }
+    }
+    __syncthreads();
+    if (tid == 0) {
+#pragma unroll
+        for (int h = 0; h < NB; ++h) {
+            float D = 0.f, N = 0.f, Q = 0.f, S = part[h][0][3];
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) {
+                D += part[h][w][0];
+                N += part[h][w][1];
+                Q += part[h][w][2];
+                if (w > 0) S = is_max ? fmaxf(S, part[h][w][3]) : S + part[h][w][3];
+            }
+            s_h[h] = h_ok[h] ? finish_cosine(D, N, Q) : -INFINITY;
+            s_a[h] = a_ok[h] ? S : -INFINITY;
+        }
+    }
+}
+
+// The finish of a sequence whose list overflowed (more than kHitCap occurrences):
+// an ordered rescan of the context writes the candidate list, then each
+// candidate is scored by cta_score.  Kept out of line: its registers do not
+// weigh on the common path.  CTA-uniform call; keys are left in thread 0.
+template <typename TH, bool IVEC>
+__device__ __noinline__ void finish_overflow(const DraftParams& p, int b, int64_t t, const int32_t* row,
+                                             int32_t* cand_row, float* hsc, float* asc, StepShared& sh,
+                                             unsigned long long& hk, unsigned long long& ak, int& nstar,
+                                             int& total) {
+    constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
     const bool has_a = p.A != nullptr;
+    const int tid = threadIdx.x;
+    int c[PLDP_MAX_NGRAM];
+#pragma unroll
+    for (int k = 0; k < PLDP_MAX_NGRAM; ++k) c[k] = 0;
+    scan_count<IVEC>(GlobalIds{row}, row, 0, t, t, p.ngram_max, c);
+    scan_reduce_counts(c, p.ngram_max, sh.ss);
+    __syncthreads();
+    if (tid == 0) {
+        int ns = 0, tot = 0;
+        for (int n = p.ngram_max; n >= p.ngram_min; --n)
+            if (sh.ss.cnt[n] > 0) {
+                ns = n;
+                tot = sh.ss.cnt[n];
+                break;
+            }
+        sh.ss.nstar = ns;
+        sh.ss.total = tot;
+        sh.ss.offset = 0;
+        sh.ss.mine = tot;
+    }
+    __syncthreads();
+    nstar = sh.ss.nstar;
+    total = sh.ss.total;
+    scan_write<IVEC>(GlobalIds{row}, row, 0, t, t, p.ngram_max, sh.ss, cand_row, p.C_cap);
+    __syncthreads();
+    const int n = total < p.C_cap ? total : p.C_cap;
+    for (int i0 = 0; i0 < n; i0 += kScoreBatch) {
+        const int nb = n - i0 < kScoreBatch ? n - i0 : kScoreBatch;
+        int64_t j[kScoreBatch];
+#pragma unroll
+        for (int h = 0; h < kScoreBatch; ++h) j[h] = h < nb ? __ldcg(cand_row + i0 + h) : -1;
+        float s_h[kScoreBatch], s_a[kScoreBatch];
+        cta_score<TH>(p, b, j, nb, t, sh.part[(i0 / kScoreBatch) & 1], s_h, s_a);
+        if (tid == 0)
+            for (int h = 0; h < nb; ++h) {
+                const int i = i0 + h;
+                if (HAS_H) {
+                    if (hsc) hsc[i] = s_h[h];
+                    if (j[h] >= 1 && s_h[h] > p.threshold) {
+                        const unsigned long long key = pack_key(s_h[h], static_cast<uint32_t>(j[h]));
+                        hk = key > hk ? key : hk;
+                    }
+                }
+                if (has_a) {
+                    if (asc) asc[i] = s_a[h];
+                    const unsigned long long key = pack_key(s_a[h], static_cast<uint32_t>(j[h]));
+                    ak = key > ak ? key : ak;
+                }
+            }
+    }
+}
+
+template <typename TH, bool IVEC>
+__global__ void __launch_bounds__(kThreads, 4) draft_step_kernel(const DraftParams p) {
+    constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
+    __shared__ StepShared sh;
+    pdl_enter();
+    const int b = blockIdx.y;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int64_t L = p.seq_len[b];
     const bool valid = L >= 0 && L <= p.T_cap;
     const int64_t t = L - 1;
     const int32_t* row = p.ids + static_cast<int64_t>(b) * p.ids_stride;
-    const bool q_fetch = HAS_H && valid && t >= 2;
-    const TQ* hb = nullptr;
-    if constexpr (HAS_H) {
-        hb = static_cast<const TQ*>(p.H) + static_cast<int64_t>(b) * p.h_seq_stride;
-        if (q_fetch && tid == 0) {
-            const uint32_t qbytes = static_cast<uint32_t>(p.d * sizeof(TQ));
-            mbar_init(&q_bar, 1);
-            fence_mbar_init();
-            mbar_arrive_expect_tx(&q_bar, qbytes);
-            bulk_g2s(q_sh, hb + (t - 1) * p.d, qbytes, &q_bar);
+    unsigned* hdr = seq_header(p.ws, b);
+    const size_t h_es = p.h_bf16 ? 2 : 4;
+    // The chunk's ids do not depend on seq_len: their loads go out first, bounded
+    // by the row's capacity, and land while seq_len and the suffix arrive.
+    const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kChunk;
+    const int64_t ce = c0 + kChunk < p.T_cap ? c0 + kChunk : p.T_cap;
+    constexpr int NV = IVEC ? kScanVec : kScanVec * 4;
+    using VT = typename std::conditional<IVEC, int4, int32_t>::type;
+    VT v[NV];
+#pragma unroll
+    for (int u = 0; u < NV; ++u) {
+        if constexpr (IVEC) {
+            const int64_t q = (c0 >> 2) + tid + u * kThreads;
+            if (q < (ce >> 2)) v[u] = __ldg(reinterpret_cast<const int4*>(row) + q);
+        } else {
+            const int64_t j = c0 + tid + u * kThreads;
+            if (j < ce) v[u] = __ldg(row + j);
         }
     }
-    unsigned* cnt_g = hit_count(p.ws, b);
-    const unsigned nh = __ldcg(cnt_g);
-    rank_shared_init(hs);
-    rank_shared_init(as);
-    if (tid <= PLDP_MAX_NGRAM) ss.cnt[tid] = 0;
-    const bool listed = nh <= static_cast<unsigned>(kHitCap);
-    if (valid && listed)
-        for (int i = tid; i < static_cast<int>(nh); i += kThreads) ls.raw[i] = __ldcg(hit_list(p.ws, b) + i);
-    bool bad = false;
-    if (has_a && valid) bad = stage_rows(rows_sh, p.row_idx, p.n_sel, p.R, p.a_row_stride, &bad_rows);
+    if (tid < PLDP_MAX_NGRAM)                                     // x_t and the n_max - 1 tokens before it
+        sh.suf[tid] = (valid && tid < p.ngram_max && t - tid >= 0) ? __ldg(row + t - tid) : 0;
+    if (tid == 0) {
+        sh.nhit = 0;
+        if (HAS_H && valid && t >= 2 && blockIdx.x == 0)        // H_{t-1}: every scored candidate reads it
+            prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (t - 1) * p.d) * h_es,
+                             static_cast<uint32_t>(p.d * h_es));
+    }
     __syncthreads();
-    if (tid == 0) *cnt_g = 0u;                        // ready for the next call
+
+    // ---- 1. scan this chunk for x_t ------------------------------------------------------
+    const int64_t c1 = c0 + kChunk < t ? c0 + kChunk : t;
+    if (valid && t >= 1 && c0 < c1) {
+        const int32_t xt = sh.suf[0];
+        uint64_t mask = 0;                                        // bit i: this thread's i-th position
+#pragma unroll
+        for (int u = 0; u < NV; ++u) {
+            if constexpr (IVEC) {
+                const int64_t q = (c0 >> 2) + tid + u * kThreads;
+                const int32_t e[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    if (e[k] == xt && 4 * q + k < c1) mask |= 1ull << (4 * u + k);
+            } else {
+                const int64_t j = c0 + tid + u * kThreads;
+                if (j < c1 && v[u] == xt) mask |= 1ull << u;
+            }
+        }
+        while (mask) {                                            // rarely more than one
+            const int bit = __ffsll(static_cast<long long>(mask)) - 1;
+            mask &= mask - 1;
+            int64_t j;
+            if constexpr (IVEC)
+                j = 4 * ((c0 >> 2) + tid + (bit >> 2) * kThreads) + (bit & 3);
+            else
+                j = c0 + tid + static_cast<int64_t>(bit) * kThreads;
+            int m = 1;                                            // common suffix of x[..j] and x[..t]
+            while (m < p.ngram_max && j - m >= 0 && __ldg(row + j - m) == sh.suf[m]) ++m;
+            const int k = atomicAdd(&sh.nhit, 1);
+            if (k < kHitCap) {                                    // more: the list overflows anyway
+                sh.hit[k] = Hit{static_cast<int32_t>(j), m};
+                if (HAS_H && j >= 1)
+                    prefetch_l2_bulk(static_cast<const char*>(p.H) +
+                                         (static_cast<int64_t>(b) * p.h_seq_stride + (j - 1) * p.d) * h_es,
+                                     static_cast<uint32_t>(p.d * h_es));
+            }
+        }
+    }
+    __syncthreads();
+
+    // ---- 2. score what this CTA found ----------------------------------------------------
+    // One atomic reserves the CTA's slots in the sequence's list; its answer is
+    // needed only when the entries are written, so it runs under the scoring.
+    const int nhit = sh.nhit;
+    if (nhit > 0) {
+        unsigned base = 0;
+        if (tid == 0) base = atomicAdd(hdr, static_cast<unsigned>(nhit));
+        if (nhit > 8) {                                           // skip the scores of a list that overflowed
+            if (tid == 0) sh.skip = base + static_cast<unsigned>(nhit) > static_cast<unsigned>(kHitCap);
+            __syncthreads();
+        }
+        if (nhit <= 8 || !sh.skip)                                // (nhit > kHitCap always skips)
+            for (int k = 0; k < nhit; k += kScoreBatch) {
+                const int nb = nhit - k < kScoreBatch ? nhit - k : kScoreBatch;
+                int64_t j[kScoreBatch];
+#pragma unroll
+                for (int h = 0; h < kScoreBatch; ++h) j[h] = h < nb ? sh.hit[k + h].j : -1;
+                float s_h[kScoreBatch], s_a[kScoreBatch];
+                cta_score<TH>(p, b, j, nb, t, sh.part[(k / kScoreBatch) & 1], s_h, s_a);
+                if (tid == 0)
+                    for (int h = 0; h < nb; ++h) {
+                        const Hit e = sh.hit[k + h];
+                        const unsigned slot = base + static_cast<unsigned>(k + h);
+                        if (slot < static_cast<unsigned>(kHitCap))
+                            seq_entries(p.ws, b)[slot] = make_uint4(static_cast<unsigned>((e.j << 4) | e.m),
+                                                                    __float_as_uint(s_h[h]), __float_as_uint(s_a[h]), 0u);
+                    }
+            }
+    }
+
+    // ---- 3. ticket: the last CTA of the sequence finishes it -----------------------------
+    if (tid == 0) {
+        __threadfence();                                          // entries before the ticket
+        sh.last = atomicAdd(hdr + 1, 1u) == gridDim.x - 1;
+        __threadfence();
+    }
+    if (tid <= PLDP_MAX_NGRAM) sh.ss.cnt[tid] = 0;
+    __syncthreads();
+    if (!sh.last) return;
+
+    const bool has_a = p.A != nullptr;
+    bool bad = false;                                             // a selected row outside [0, R)
+    if (has_a && valid && p.row_idx)
+        for (int k = tid; k < p.n_sel; k += kThreads) {
+            const int r = __ldg(p.row_idx + k);
+            bad |= r < 0 || r >= p.R;
+        }
+    const unsigned nh = __ldcg(hdr);
+    bad = __syncthreads_or(bad) != 0;
 
     if (!valid) {
         for (int i = tid; i < p.K; i += kThreads) p.draft[static_cast<int64_t>(b) * p.K + i] = -1;
@@ -264,157 +443,111 @@ __global__ void __launch_bounds__(kThreads) draft_rank_kernel(const DraftParams 
             }
             p.draft_len[b] = 0;
             if (p.status) atomicOr(p.status + b, PLDP_ST_SEQ_LEN);
+            hdr[0] = 0u;
+            hdr[1] = 0u;
         }
         return;
     }
 
-    // ---- the candidate list ------------------------------------------------------------
     int32_t* cand_row = p.cand_pos + static_cast<int64_t>(b) * p.C_cap;
-    if (listed) {
-        if (tid == 0) {
-            int mx = 0;
-            for (int i = 0; i < static_cast<int>(nh); ++i) mx = max(mx, ls.raw[i] & 15);
-            const int nstar = mx >= p.ngram_min ? mx : 0;
-            int total = 0;
-            if (nstar)
-                for (int i = 0; i < static_cast<int>(nh); ++i) total += ((ls.raw[i] & 15) >= nstar) ? 1 : 0;
-            ls.nstar = nstar;
-            ls.total = total;
-        }
+    float* hsc = (HAS_H && p.h_scores) ? p.h_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
+    float* asc = (has_a && p.a_scores) ? p.a_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
+    unsigned long long hk = 0, ak = 0;                            // this thread's best keys
+    int nstar, total;
+    if (nh <= static_cast<unsigned>(kHitCap)) {
+        // ---- the list: one entry per thread ----
+        const bool have = tid < static_cast<int>(nh);
+        uint4 e = make_uint4(0u, 0u, 0u, 0u);
+        if (have) e = __ldcg(seq_entries(p.ws, b) + tid);
+        const int m = have ? static_cast<int>(e.x & 15u) : 0;
+        const int32_t j = static_cast<int32_t>(e.x >> 4);
+        const int wm = __reduce_max_sync(0xFFFFFFFFu, m);
+        if (lane == 0) sh.wmax[warp] = wm;
         __syncthreads();
-        const int nstar = ls.nstar;
-        if (nstar > 0)
-            for (int i = tid; i < static_cast<int>(nh); i += kThreads) {
-                const int32_t e = ls.raw[i];
-                if ((e & 15) < nstar) continue;
-                int r = 0;                              // positions are distinct: so are ranks
-                for (int k = 0; k < static_cast<int>(nh); ++k) {
-                    const int32_t f = ls.raw[k];
-                    r += ((f & 15) >= nstar && f < e) ? 1 : 0;
-                }
-                ls.sorted[r] = e >> 4;
-            }
-        __syncthreads();
-    } else {
-        // more occurrences than the list holds: an ordered rescan of the whole context
-        int c[PLDP_MAX_NGRAM];
+        int mx = 0;
 #pragma unroll
-        for (int k = 0; k < PLDP_MAX_NGRAM; ++k) c[k] = 0;
-        scan_count<IVEC>(GlobalIds{row}, row, 0, t, t, p.ngram_max, c);
-        scan_reduce_counts(c, p.ngram_max, ss);
-        __syncthreads();
-        if (tid == 0) {
-            int nstar = 0, total = 0;
-            for (int n = p.ngram_max; n >= p.ngram_min; --n)
-                if (ss.cnt[n] > 0) {
-                    nstar = n;
-                    total = ss.cnt[n];
-                    break;
+        for (int w = 0; w < kWarps; ++w) mx = max(mx, sh.wmax[w]);
+        nstar = mx >= p.ngram_min ? mx : 0;                       // m <= ngram_max already
+        const bool cand = have && nstar > 0 && m >= nstar;
+        sh.jl[tid] = cand ? j : INT_MAX;
+        total = __syncthreads_count(cand);
+        if (cand) {
+            int r = 0;                                            // positions are distinct: so are ranks
+            for (int k = 0; k < static_cast<int>(nh); ++k) r += sh.jl[k] < j ? 1 : 0;
+            if (r < p.C_cap) {
+                cand_row[r] = j;
+                const float s_h = __uint_as_float(e.y), s_a = __uint_as_float(e.z);
+                if (HAS_H) {
+                    if (hsc) hsc[r] = s_h;
+                    if (j >= 1 && s_h > p.threshold) hk = pack_key(s_h, static_cast<uint32_t>(j));
                 }
-            ss.nstar = nstar;
-            ss.total = total;
-            ss.offset = 0;
-            ss.mine = total;
-            ls.nstar = nstar;
-            ls.total = total;
+                if (has_a) {
+                    if (asc) asc[r] = s_a;
+                    ak = pack_key(s_a, static_cast<uint32_t>(j));
+                }
+            }
         }
-        __syncthreads();
-        scan_write<IVEC>(GlobalIds{row}, row, 0, t, t, p.ngram_max, ss, cand_row, p.C_cap);
+    } else {
+        finish_overflow<TH, IVEC>(p, b, t, row, cand_row, hsc, asc, sh, hk, ak, nstar, total);
     }
-    const int total = ls.total;
-    const int n = total < p.C_cap ? total : p.C_cap;
-    if (listed)
-        for (int i = tid; i < n; i += kThreads) cand_row[i] = ls.sorted[i];
-    if (tid == 0) {
-        p.cand_count[b] = total;
-        p.match_len[b] = ls.nstar;
-        if (p.status && total > p.C_cap) atomicOr(p.status + b, PLDP_ST_CAND_OVERFLOW);
-        if (bad && p.status) atomicOr(p.status + b, PLDP_ST_ROW_INDEX);
-    }
-    __syncthreads();                                   // cand_row is complete for the rescan path
 
-    // ---- ranking: hidden states on warps 0-3 while attentions run on warps 4-7 ----------
-    const bool split = HAS_H && has_a;
-    const WarpGroup hg = split ? WarpGroup{0, 4, 1} : whole_cta();
-    const WarpGroup ag = split ? WarpGroup{4, 4, 2} : whole_cta();
-    if constexpr (HAS_H) {
-        if (!split || warp < 4) {
-            float* hsc = p.h_scores ? p.h_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
-            if (listed)
-                hidden_rank_cta<TQ, true, true>(hb, p.d, t, ls.sorted, n, 1, 0, nullptr, q_sh, &q_bar, q_fetch,
-                                                p.threshold, hsc, hs, hg);
-            else
-                hidden_rank_cta<TQ, true, false>(hb, p.d, t, cand_row, n, 1, 0, nullptr, q_sh, &q_bar,
-                                                 q_fetch, p.threshold, hsc, hs, hg);
-            if (q_fetch && tid == 0 && !mbar_wait(&q_bar, 0, kMbarPolls)) hs.err = 1;   // landed before exit
-        }
-    }
-    if (has_a && (!split || warp >= 4)) {
-        const size_t es = p.a_bf16 ? 2 : 4;
-        const void* ab = static_cast<const char*>(p.A) + static_cast<int64_t>(b) * p.a_seq_stride * es;
-        float* asc = p.a_scores ? p.a_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
-        if (listed)
-            attention_rank_cta<true>(ab, p.a_bf16, rows_sh, p.n_sel, t, ls.sorted, n, 1, 0, nullptr,
-                                     p.agg == PLDP_AGG_MAX, asc, as, ag);
-        else
-            attention_rank_cta<false>(ab, p.a_bf16, rows_sh, p.n_sel, t, cand_row, n, 1, 0, nullptr,
-                                      p.agg == PLDP_AGG_MAX, asc, as, ag);
+    // ---- best of each ranking, then the draft (Sec. 4.3) ----------------------------------
+    hk = warp_max_u64(hk);
+    ak = warp_max_u64(ak);
+    if (lane == 0) {
+        sh.wkey[0][warp] = hk;
+        sh.wkey[1][warp] = ak;
     }
     __syncthreads();
-
-    // ---- best and draft (warp 0) -----------------------------------------------------------
-    if (warp == 0) {
-        const unsigned long long hk = rank_best_key(hs), ak = rank_best_key(as);
-        const int err = hs.err;
-        const int32_t bh = (err || hk == 0) ? -1 : static_cast<int32_t>(key_index(hk));
-        const int32_t ba = ak == 0 ? -1 : static_cast<int32_t>(key_index(ak));
-        if (tid == 0) {
-            if (HAS_H) {
-                p.best_h[b] = bh;
-                if (p.best_h_score) p.best_h_score[b] = bh >= 0 ? key_value(hk) : -INFINITY;
-                if (err && p.status) atomicOr(p.status + b, PLDP_ST_TIMEOUT);
-            }
-            if (has_a) {
-                p.best_a[b] = ba;
-                if (p.best_a_score) p.best_a_score[b] = ba >= 0 ? key_value(ak) : -INFINITY;
-            }
+    if (warp != 0) return;
+    hk = 0;
+    ak = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+        hk = sh.wkey[0][w] > hk ? sh.wkey[0][w] : hk;
+        ak = sh.wkey[1][w] > ak ? sh.wkey[1][w] : ak;
+    }
+    const int32_t bh = hk == 0 ? -1 : static_cast<int32_t>(key_index(hk));
+    const int32_t ba = ak == 0 ? -1 : static_cast<int32_t>(key_index(ak));
+    const int64_t js = p.draft_from == 0 ? bh : ba;
+    int64_t dl = 0;
+    if (js >= 0 && js < t) dl = (t - js < p.K) ? (t - js) : p.K;
+    for (int i = lane; i < p.K; i += 32)
+        p.draft[static_cast<int64_t>(b) * p.K + i] = (i < dl) ? __ldg(row + js + 1 + i) : -1;
+    if (lane == 0) {
+        p.cand_count[b] = total;
+        p.match_len[b] = nstar;
+        if (HAS_H) {
+            p.best_h[b] = bh;
+            if (p.best_h_score) p.best_h_score[b] = bh >= 0 ? key_value(hk) : -INFINITY;
         }
-        const int64_t js = p.draft_from == 0 ? bh : ba;
-        int64_t dl = 0;
-        if (js >= 0 && js < t) dl = (t - js < p.K) ? (t - js) : p.K;
-        for (int i = lane; i < p.K; i += 32)
-            p.draft[static_cast<int64_t>(b) * p.K + i] = (i < dl) ? __ldg(row + js + 1 + i) : -1;
-        if (tid == 0) p.draft_len[b] = static_cast<int32_t>(dl);
+        if (has_a) {
+            p.best_a[b] = ba;
+            if (p.best_a_score) p.best_a_score[b] = ba >= 0 ? key_value(ak) : -INFINITY;
+        }
+        p.draft_len[b] = static_cast<int32_t>(dl);
+        if (p.status && total > p.C_cap) atomicOr(p.status + b, PLDP_ST_CAND_OVERFLOW);
+        if (p.status && bad) atomicOr(p.status + b, PLDP_ST_ROW_INDEX);
+        hdr[0] = 0u;                                              // ready for the next call
+        hdr[1] = 0u;
     }
 }
 
 template <typename TH, bool IVEC>
-pldp_status launch_t(const DraftParams& p, int B, size_t smem, cudaStream_t s) {
-    const int64_t chunks = (p.T_cap + kChunk - 1) / kChunk;
-    if (chunks > 65535) return fail(PLDP_ERR_UNSUPPORTED, "draft_step: T_cap too large for the scan grid");
-    if (chunks > 0) {
-        cudaError_t e = launch_pdl(draft_scan_kernel<IVEC>, dim3(static_cast<unsigned>(chunks), static_cast<unsigned>(B)),
-                                   dim3(kThreads), 0, s, 0, p);
-        if (e != cudaSuccess)
-            return fail(PLDP_ERR_CUDA, "draft_step (scan): launch failed: %s", cudaGetErrorString(e));
-    }
-    if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(draft_rank_kernel<TH, IVEC>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             static_cast<int>(smem));
-        if (e != cudaSuccess)
-            return fail(PLDP_ERR_CUDA, "draft_step: shared memory attribute: %s", cudaGetErrorString(e));
-    }
-    cudaError_t e = launch_pdl(draft_rank_kernel<TH, IVEC>, dim3(static_cast<unsigned>(B)), dim3(kThreads), smem, s,
+pldp_status launch_t(const DraftParams& p, int B, cudaStream_t s) {
+    int64_t chunks = (p.T_cap + kChunk - 1) / kChunk;
+    if (chunks < 1) chunks = 1;                                   // every sequence needs its finish
+    if (chunks > 65535) return fail(PLDP_ERR_UNSUPPORTED, "draft_step: T_cap too large for the grid");
+    cudaError_t e = launch_pdl(draft_step_kernel<TH, IVEC>,
+                               dim3(static_cast<unsigned>(chunks), static_cast<unsigned>(B)), dim3(kThreads), 0, s,
                                0, p);
-    if (e != cudaSuccess)
-        return fail(PLDP_ERR_CUDA, "draft_step (rank): launch failed: %s", cudaGetErrorString(e));
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "draft_step: launch failed: %s", cudaGetErrorString(e));
     return PLDP_OK;
 }
 
 template <typename TH>
-pldp_status launch_draft_step(const DraftParams& p, int B, size_t smem, cudaStream_t s, bool ivec) {
-    return ivec ? launch_t<TH, true>(p, B, smem, s) : launch_t<TH, false>(p, B, smem, s);
+pldp_status launch_draft_step(const DraftParams& p, int B, cudaStream_t s, bool ivec) {
+    return ivec ? launch_t<TH, true>(p, B, s) : launch_t<TH, false>(p, B, s);
 }
 
 }  // namespace
@@ -518,11 +651,9 @@ extern "C" PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* a, v
     p.draft_len = a->draft_len;
     p.status = a->status;
     p.ws = static_cast<unsigned char*>(a->workspace);
-    p.rows_offset = (qbytes + 127) / 128 * 128;
-    const size_t smem = p.rows_offset + static_cast<size_t>(sel) * sizeof(int64_t);
     const bool ivec = aligned16(a->ids) && a->ids_stride % 4 == 0 && a->T_cap % 4 == 0;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (!a->H) return launch_draft_step<NoHidden>(p, B, smem, s, ivec);
-    if (a->h_dtype == PLDP_BF16) return launch_draft_step<__nv_bfloat16>(p, B, smem, s, ivec);
-    return launch_draft_step<float>(p, B, smem, s, ivec);
+    if (!a->H) return launch_draft_step<NoHidden>(p, B, s, ivec);
+    if (a->h_dtype == PLDP_BF16) return launch_draft_step<__nv_bfloat16>(p, B, s, ivec);
+    return launch_draft_step<float>(p, B, s, ivec);
 }
