@@ -209,7 +209,7 @@ class Path:
         self.dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=dev)
         self.row_idx = None   # all R rows of the chosen layers
         self.fused = fused
-        self.launches_per_step = 3 if fused else 5     # pldp_draft_step launches two kernels
+        self.launches_per_step = 3 if fused else 6     # pldp_verify_greedy launches two kernels
         self.kernels = (["draft_step"] if fused else
                         ["find_candidates", "rank_hidden", "rank_attention", "extract_draft"]) + ["verify_greedy"]
 

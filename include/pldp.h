@@ -320,7 +320,7 @@ PLDP_API pldp_status pldp_verify_greedy(const void* logits, pldp_dtype dtype, in
  * more than that (pldp_verify_workspace_size(B, K, V) > 1048576, i.e. roughly
  * B*(K+1) > 130000 rows) are rejected with PLDP_ERR_INVALID_ARG.  The call
  * allocates nothing: it clears the part of the area it uses with
- * cudaMemsetAsync on `stream`, then launches the kernel.
+ * cudaMemsetAsync on `stream`, then launches the verification kernels.
  *
  * The first call on each device looks up the area's device address (once per
  * device, on the current device); make that first call before any stream

@@ -1,20 +1,23 @@
 // Draft prediction (Sec. 4.3) and greedy verification (Sec. 4.4) of PLD+.
 //
-// Verification is one streaming pass over the logits [B, K+1, V].  The
-// flattened logits are cut into equal contiguous ranges, one per warp, sized so
-// that the grid fills every SM once (a persistent split: no tail wave, and
-// each warp's range crosses at most a couple of row boundaries).  A warp keeps
-// a running (max, first index) per lane with 16-byte streaming loads, using a
-// packed max over each vector so that the index search runs only when the
-// running max grows.  Per row, the warps' results meet in a packed 64-bit key
-// (value, inverted index) combined with atomicMax in the workspace, which makes
-// the argmax exact and independent of scheduling: larger value wins, the
-// smaller index wins ties, -0.0 equals +0.0.
+// Verification is two kernels chained by programmatic dependent launch.
 //
-// Every warp that touched sequence b then takes a ticket; the warp holding the
-// last ticket (there is no waiting: the others just leave) reads the K+1 row
-// keys, finds the accepted length and the bonus token, appends them to the
-// context and returns the keys and the ticket to zero for the next call.
+// 1. One streaming pass over the flattened logits [B, K+1, V], cut into 2 KB
+//    segments.  Warp w of the W in the grid takes segments w, w + W, w + 2W, ...
+//    so the segments in flight form a moving window over memory, and the grid
+//    is several waves of small CTAs, so the block scheduler keeps every SM busy
+//    to the end (faster SMs take more CTAs).  Each lane issues its four 16-byte
+//    loads of a segment at once and keeps a running (max, first index) with a
+//    packed max over each vector, so the index search runs only when the max
+//    grows.  A segment crosses at most one row boundary (rows are longer than a
+//    segment on this path); per row, the warps' results meet in a packed 64-bit
+//    key (value, inverted index) combined with atomicMax in the workspace, which
+//    makes the argmax exact and independent of scheduling: larger value wins,
+//    the smaller index wins ties, -0.0 equals +0.0.  The pass never waits on
+//    another warp and never fences.
+// 2. One warp per sequence reads its K+1 row keys, finds the accepted length and
+//    the bonus token, appends them to the context and returns the keys to zero
+//    for the next call.  Its launch is hidden behind the pass's last wave.
 #include <math.h>
 
 #include "pldp_internal.cuh"
@@ -24,10 +27,11 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
-constexpr int kUnroll = 8;                  // 16-byte loads in flight per lane
-constexpr int kMinBlocksPerSm = 4;          // register cap: 4 CTAs of 8 warps per SM
-constexpr int64_t kMinChunk = 2048;         // elements per warp, at least
-constexpr int64_t kAlign = 8;               // range boundaries are multiples of 8 elements
+constexpr int kUnroll = 8;                  // loads in flight per lane on the row-loop path
+constexpr int kSegLoads = 4;                // 16-byte loads per lane per segment
+constexpr int64_t kSegBytes = 32 * kSegLoads * 16;   // 2 KB
+constexpr int kPassBlocksPerSm = 8;         // register cap: 8 CTAs of 8 warps per SM
+constexpr int kPassWaves = 6;               // grid = up to 6 waves of resident CTAs
 
 __global__ void extract_draft_kernel(const int32_t* __restrict__ ids, int64_t ids_stride,
                                      const int32_t* __restrict__ seq_len, int64_t T_cap,
@@ -135,13 +139,10 @@ struct VerifyArgs {
     int32_t* kv_keep_len;
     uint32_t* status;
     unsigned long long* row_keys;   // [B*(K+1)], zero between calls
-    unsigned int* tickets;          // [B], zero between calls
     int B, K, V;
-    int64_t chunk;                  // elements per warp
-    int64_t total_warps;
 };
 
-// Accept/bonus/append for sequence b, by the warp that holds its last ticket.
+// Accept/bonus/append for sequence b, by one warp, once the row keys are final.
 __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
     const int K1 = a.K + 1;
     unsigned long long* keys = a.row_keys + b * K1;
@@ -198,76 +199,127 @@ __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
     }
     if (lane == 0) {
         if (a.status && st) a.status[b] |= st;
-        a.tickets[b] = 0u;
     }
 }
 
-template <typename T, bool VEC>
-__global__ void __launch_bounds__(kThreads, kMinBlocksPerSm)
-verify_greedy_kernel(const T* __restrict__ logits, VerifyArgs a) {
-    pdl_enter();
-    const int lane = threadIdx.x & 31;
-    const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
-    if (w >= a.total_warps) return;
-    const int64_t V = a.V;
-    const int64_t E = static_cast<int64_t>(a.K + 1) * V;        // elements per sequence
-    const int64_t N = E * a.B;
-    const int64_t lo = w * a.chunk;
-    const int64_t hi = lo + a.chunk < N ? lo + a.chunk : N;
+// Segment [s0, s0 + 32 * kSegLoads) of the flattened logits, in 16-byte vectors
+// (nvec of them in all, vrow per row; rows are at least a segment long, and
+// nvec < 2^31 so that 32-bit indices hold): the segment holds the end of row r0
+// and possibly the start of row r0 + 1.
+template <typename T>
+__device__ __forceinline__ void segment_two_rows(const uint4* __restrict__ p, uint32_t s0, uint32_t nvec,
+                                                 uint32_t vrow, int lane, unsigned long long* __restrict__ keys) {
+    constexpr uint32_t VW = 16 / sizeof(T);
+    constexpr uint32_t seg = 32 * kSegLoads;
+    const uint32_t r0 = s0 / vrow;
+    const uint32_t bnd = (r0 + 1) * vrow;                   // first vector of row r0 + 1
+    uint4 x[kSegLoads];
+#pragma unroll
+    for (int u = 0; u < kSegLoads; ++u) {
+        const uint32_t v = s0 + lane + 32 * u;
+        if (v < nvec) x[u] = ld_stream16(p + v);
+    }
+    float b0 = -INFINITY, b1 = -INFINITY;
+    uint32_t i0 = (s0 - r0 * vrow) * VW, i1 = 0;
+#pragma unroll
+    for (int u = 0; u < kSegLoads; ++u) {
+        const uint32_t v = s0 + lane + 32 * u;
+        if (v < nvec) {
+            const float m = vmax(x[u], T());
+            if (v < bnd) {
+                if (m > b0) {
+                    b0 = m;
+                    i0 = (v - r0 * vrow) * VW + vfirst(x[u], m, T());
+                }
+            } else if (m > b1) {
+                b1 = m;
+                i1 = (v - bnd) * VW + vfirst(x[u], m, T());
+            }
+        }
+    }
+    const unsigned long long k0 = warp_max_u64(pack_key(b0, i0));
+    if (lane == 0) atomicMax(keys + r0, k0);
+    if (s0 + seg > bnd && bnd < nvec) {
+        const unsigned long long k1 = warp_max_u64(pack_key(b1, i1));
+        if (lane == 0) atomicMax(keys + r0 + 1, k1);
+    }
+}
 
-    for (int64_t pos = lo; pos < hi;) {
+// Any segment: row by row, each row piece with the lane loop above.
+template <typename T, bool VEC>
+__device__ __forceinline__ void segment_rows(const T* __restrict__ logits, int64_t e0, int64_t e1, int64_t V,
+                                             int lane, unsigned long long* __restrict__ keys) {
+    for (int64_t pos = e0; pos < e1;) {
         const int64_t r = pos / V;
         const int64_t c0 = pos - r * V;
-        const int64_t c1 = (V < c0 + (hi - pos)) ? V : c0 + (hi - pos);
+        const int64_t c1 = (V < c0 + (e1 - pos)) ? V : c0 + (e1 - pos);
         float bv = -INFINITY;
         int64_t bi = c0;
         lane_argmax<T, VEC>(logits + r * V, c0, c1, lane, bv, bi);
         const unsigned long long k = warp_max_u64(pack_key(bv, static_cast<uint32_t>(bi)));
-        if (lane == 0) atomicMax(a.row_keys + r, k);
+        if (lane == 0) atomicMax(keys + r, k);
         pos += c1 - c0;
     }
+}
 
-    const int64_t b0 = lo / E, b1 = (hi - 1) / E;
-    for (int64_t b = b0; b <= b1; ++b) {
-        int last = 0;
-        if (lane == 0) {
-            __threadfence();   // this warp's row keys are visible before its ticket
-            const int64_t first_w = (b * E) / a.chunk;
-            const int64_t last_w = ((b + 1) * E - 1) / a.chunk;
-            const unsigned expected = static_cast<unsigned>(last_w - first_w + 1);
-            last = (atomicAdd(a.tickets + b, 1u) == expected - 1u);
-        }
-        last = __shfl_sync(0xFFFFFFFFu, last, 0);
-        if (last) {
-            __threadfence();
-            finish_sequence(a, b, lane);
+// 1. the row argmax pass.  W = warps in the grid.  PATH 0: 16-byte loads, rows of
+// at least a segment (the streaming path); 1: 16-byte loads, short rows; 2: element
+// loads (unaligned logits or rows that are not a whole number of 16 bytes).
+template <typename T, int PATH>
+__global__ void __launch_bounds__(kThreads, PATH == 0 ? kPassBlocksPerSm : 4)
+verify_argmax_kernel(const T* __restrict__ logits, int64_t N, int64_t V, int64_t W,
+                     unsigned long long* __restrict__ keys) {
+    pdl_enter();
+    const int lane = threadIdx.x & 31;
+    const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+    if constexpr (PATH == 0) {
+        constexpr uint32_t VW = 16 / sizeof(T);
+        constexpr uint32_t seg = 32 * kSegLoads;
+        const uint32_t nvec = static_cast<uint32_t>(N / VW), vrow = static_cast<uint32_t>(V / VW);
+        const uint32_t stride = static_cast<uint32_t>(W) * seg;
+        const uint4* p = reinterpret_cast<const uint4*>(logits);
+        for (uint32_t s0 = static_cast<uint32_t>(w) * seg; s0 < nvec; s0 += stride)
+            segment_two_rows<T>(p, s0, nvec, vrow, lane, keys);
+    } else {
+        constexpr int64_t SEG = kSegBytes / static_cast<int64_t>(sizeof(T));   // elements per segment
+        for (int64_t e0 = w * SEG; e0 < N; e0 += W * SEG) {
+            const int64_t e1 = e0 + SEG < N ? e0 + SEG : N;
+            segment_rows<T, PATH == 1>(logits, e0, e1, V, lane, keys);
         }
     }
+}
+
+// 2. accept, bonus and append: one warp per sequence.
+__global__ void __launch_bounds__(kThreads) verify_finish_kernel(VerifyArgs a) {
+    pdl_enter();                                           // the pass's keys are final
+    const int64_t b = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+    if (b < a.B) finish_sequence(a, b, threadIdx.x & 31);
 }
 
 size_t keys_bytes(int B, int K) {
     return (static_cast<size_t>(B) * (K + 1) * sizeof(unsigned long long) + 255) / 256 * 256;
 }
 
-// Splits the flattened logits into equal per-warp ranges for a grid that is
-// exactly the number of CTAs resident on the device at once (one wave), and
-// launches.  `a` has everything but the split and the scratch filled in.
-template <typename T, bool VEC>
+// Sizes the pass's grid (up to kPassWaves waves of resident CTAs, no more warps
+// than segments) and launches both kernels.  `a` has everything but the keys.
+template <typename T, int PATH>
 pldp_status launch_verify_t(const void* logits, VerifyArgs a, void* scratch, cudaStream_t s,
                             const char* what) {
-    const void* fn = reinterpret_cast<const void*>(&verify_greedy_kernel<T, VEC>);
+    const void* fn = reinterpret_cast<const void*>(&verify_argmax_kernel<T, PATH>);
     const int64_t N = static_cast<int64_t>(a.B) * (a.K + 1) * a.V;
-    const int64_t resident_warps = static_cast<int64_t>(resident_blocks(fn, kThreads, 0)) * kWarps;
-    int64_t chunk = (N + resident_warps - 1) / resident_warps;
-    if (chunk < kMinChunk) chunk = kMinChunk;
-    chunk = (chunk + kAlign - 1) / kAlign * kAlign;
-    a.chunk = chunk;
-    a.total_warps = (N + chunk - 1) / chunk;
+    constexpr int64_t SEG = kSegBytes / static_cast<int64_t>(sizeof(T));
+    const int64_t segs = (N + SEG - 1) / SEG;
+    int64_t blocks = static_cast<int64_t>(resident_blocks(fn, kThreads, 0)) * kPassWaves;
+    const int64_t need = (segs + kWarps - 1) / kWarps;
+    if (blocks > need) blocks = need;
+    if (blocks < 1) blocks = 1;
     a.row_keys = static_cast<unsigned long long*>(scratch);
-    a.tickets = reinterpret_cast<unsigned int*>(static_cast<char*>(scratch) + keys_bytes(a.B, a.K));
-    const unsigned blocks = static_cast<unsigned>((a.total_warps + kWarps - 1) / kWarps);
-    const cudaError_t e = launch_pdl(verify_greedy_kernel<T, VEC>, dim3(blocks), dim3(kThreads), 0, s, 0,
-                                     static_cast<const T*>(logits), a);
+    cudaError_t e = launch_pdl(verify_argmax_kernel<T, PATH>, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0,
+                               s, 0, static_cast<const T*>(logits), N, static_cast<int64_t>(a.V),
+                               blocks * kWarps, a.row_keys);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
+    const unsigned fblocks = static_cast<unsigned>((a.B + kWarps - 1) / kWarps);
+    e = launch_pdl(verify_finish_kernel, dim3(fblocks), dim3(kThreads), 0, s, 0, a);
     if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
     return PLDP_OK;
 }
@@ -276,11 +328,18 @@ pldp_status launch_verify(const void* logits, pldp_dtype dtype, const VerifyArgs
                           cudaStream_t s, const char* what) {
     const size_t es = dtype == PLDP_F32 ? 4 : 2;
     const bool vec = aligned16(logits) && (static_cast<size_t>(a.V) * es) % 16 == 0;
-    if (dtype == PLDP_BF16)
-        return vec ? launch_verify_t<__nv_bfloat16, true>(logits, a, scratch, s, what)
-                   : launch_verify_t<__nv_bfloat16, false>(logits, a, scratch, s, what);
-    return vec ? launch_verify_t<float, true>(logits, a, scratch, s, what)
-               : launch_verify_t<float, false>(logits, a, scratch, s, what);
+    const int64_t bytes = static_cast<int64_t>(a.B) * (a.K + 1) * a.V * static_cast<int64_t>(es);
+    const bool long_rows = static_cast<int64_t>(a.V) * static_cast<int64_t>(es) >= kSegBytes;
+    const bool small = bytes / 16 < (int64_t(1) << 31);     // 32-bit vector indices
+    const int path = vec ? (long_rows && small ? 0 : 1) : 2;
+    if (dtype == PLDP_BF16) {
+        if (path == 0) return launch_verify_t<__nv_bfloat16, 0>(logits, a, scratch, s, what);
+        if (path == 1) return launch_verify_t<__nv_bfloat16, 1>(logits, a, scratch, s, what);
+        return launch_verify_t<__nv_bfloat16, 2>(logits, a, scratch, s, what);
+    }
+    if (path == 0) return launch_verify_t<float, 0>(logits, a, scratch, s, what);
+    if (path == 1) return launch_verify_t<float, 1>(logits, a, scratch, s, what);
+    return launch_verify_t<float, 2>(logits, a, scratch, s, what);
 }
 
 VerifyArgs verify_args(int B, int K, int V, const int32_t* draft, const int32_t* draft_len,
@@ -312,7 +371,7 @@ using namespace pldp;
 
 extern "C" PLDP_API size_t pldp_verify_workspace_size(int B, int K, int V) {
     if (B < 0 || K < 1 || V < 1) return 0;
-    return keys_bytes(B, K) + (static_cast<size_t>(B) * sizeof(unsigned int) + 255) / 256 * 256;
+    return keys_bytes(B, K);
 }
 
 extern "C" PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
@@ -447,9 +506,9 @@ extern "C" PLDP_API pldp_status pldp_verify_greedy_noalloc(
     pldp_status ps = noalloc_scratch(&scratch);
     if (ps != PLDP_OK) return ps;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    // The kernel needs its row keys and tickets at zero.  Each call returns them to
-    // zero when it completes, but the area is shared and outlives every call, so it
-    // is cleared here as well (cudaMemsetAsync allocates nothing).
+    // The kernels need the row keys at zero.  Each call returns them to zero when
+    // it completes, but the area is shared and outlives every call, so it is
+    // cleared here as well (cudaMemsetAsync allocates nothing).
     cudaError_t e = cudaMemsetAsync(scratch, 0, need, s);
     if (e != cudaSuccess)
         return fail(PLDP_ERR_CUDA, "verify_greedy_noalloc: clearing scratch: %s", cudaGetErrorString(e));
