@@ -143,32 +143,38 @@ struct VerifyArgs {
 };
 
 // Accept/bonus/append for sequence b, by one warp, once the row keys are final.
+// Everything it reads is requested up front (one round trip when K < 32).
 __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
     const int K1 = a.K + 1;
     unsigned long long* keys = a.row_keys + b * K1;
+    const int d_in = a.draft_len[b];
+    const int64_t L = a.seq_len ? a.seq_len[b] : 0;
+    const unsigned long long k_first = lane < K1 ? __ldcg(keys + lane) : 0ull;
+    const int tok_first = lane < a.K ? a.draft[b * a.K + lane] : 0;
     uint32_t st = 0;
-    int d = a.draft_len[b];
+    int d = d_in;
     if (d < 0 || d > a.K) {
         st |= PLDP_ST_DRAFT_LEN;
         d = d < 0 ? 0 : a.K;
     }
     int n = d;
     bool range_bad = false;
+    int am_first = 0;
     for (int i0 = 0; i0 < K1; i0 += 32) {
         const int i = i0 + lane;
-        int am = 0;
-        if (i < K1) {
-            am = static_cast<int>(key_index(__ldcg(keys + i)));
-            if (a.argmax) a.argmax[b * K1 + i] = am;
-        }
+        const unsigned long long kk = i0 == 0 ? k_first : (i < K1 ? __ldcg(keys + i) : 0ull);
+        const int tok = i0 == 0 ? tok_first : (i < a.K ? a.draft[b * a.K + i] : 0);
+        const int am = static_cast<int>(key_index(kk));
+        if (i0 == 0) am_first = am;
+        if (i < K1 && a.argmax) a.argmax[b * K1 + i] = am;
         const bool in_draft = i < d;
-        const int tok = in_draft ? a.draft[b * a.K + i] : 0;
         range_bad |= in_draft && (tok < 0 || tok >= a.V);
         const unsigned mism = __ballot_sync(0xFFFFFFFFu, in_draft && tok != am);
         if (n == d && mism) n = i0 + __ffs(mism) - 1;
     }
     if (__any_sync(0xFFFFFFFFu, range_bad)) st |= PLDP_ST_TOKEN_RANGE;
-    const int bonus = static_cast<int>(key_index(__ldcg(keys + n)));
+    const int bonus = n < 32 ? __shfl_sync(0xFFFFFFFFu, am_first, n)
+                             : static_cast<int>(key_index(__ldcg(keys + n)));
     __syncwarp();
     for (int i = lane; i < K1; i += 32) keys[i] = 0ull;
 
@@ -177,7 +183,6 @@ __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
         a.next_token[b] = bonus;
     }
     if (a.seq_len) {
-        const int64_t L = a.seq_len[b];
         int64_t kv = -1;
         if (L < 1 || L > a.T_cap) {
             st |= PLDP_ST_SEQ_LEN;
@@ -188,7 +193,8 @@ __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
             } else {
                 if (a.ids) {
                     int32_t* row = a.ids + b * a.ids_stride + L;
-                    for (int i = lane; i < n; i += 32) row[i] = a.draft[b * a.K + i];
+                    if (lane < n) row[lane] = tok_first;
+                    for (int i = 32 + lane; i < n; i += 32) row[i] = a.draft[b * a.K + i];
                     if (lane == 0) row[n] = bonus;
                 }
                 __syncwarp();
@@ -202,25 +208,52 @@ __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
     }
 }
 
+// Packed key from an ordered value key (see ordered_key) and an index.
+__device__ __forceinline__ unsigned long long pack_ordered(uint32_t okey, uint32_t idx) {
+    return (static_cast<unsigned long long>(okey) << 32) | static_cast<unsigned long long>(0xFFFFFFFFu - idx);
+}
+
 // Segment [s0, s0 + 32 * kSegLoads) of the flattened logits, in 16-byte vectors
-// (nvec of them in all, vrow per row; rows are at least a segment long, and
-// nvec < 2^31 so that 32-bit indices hold): the segment holds the end of row r0
-// and possibly the start of row r0 + 1.
+// (nvec in all, vrow per row, rows at least a segment long, nvec < 2^31 so that
+// 32-bit indices hold).  The segment starts `rem` vectors into row r0.
+//
+// Common case, the segment inside row r0: each lane takes the max of its four
+// vectors, the warp's max comes from one redux over the ordered keys, and only
+// the lane(s) holding it search for the element; a second redux picks the
+// smallest index.  A segment that crosses into row r0 + 1 keeps a running
+// (max, first index) per row and lane.
 template <typename T>
-__device__ __forceinline__ void segment_two_rows(const uint4* __restrict__ p, uint32_t s0, uint32_t nvec,
-                                                 uint32_t vrow, int lane, unsigned long long* __restrict__ keys) {
+__device__ __forceinline__ void segment_argmax(const uint4* __restrict__ p, uint32_t s0, uint32_t nvec,
+                                               uint32_t r0, uint32_t rem, uint32_t vrow, int lane,
+                                               unsigned long long* __restrict__ keys) {
     constexpr uint32_t VW = 16 / sizeof(T);
     constexpr uint32_t seg = 32 * kSegLoads;
-    const uint32_t r0 = s0 / vrow;
-    const uint32_t bnd = (r0 + 1) * vrow;                   // first vector of row r0 + 1
     uint4 x[kSegLoads];
 #pragma unroll
     for (int u = 0; u < kSegLoads; ++u) {
         const uint32_t v = s0 + lane + 32 * u;
         if (v < nvec) x[u] = ld_stream16(p + v);
     }
+    if (rem + seg <= vrow && s0 + seg <= nvec) {               // warp-uniform
+        float m = vmax(x[0], T());
+#pragma unroll
+        for (int u = 1; u < kSegLoads; ++u) m = fmaxf(m, vmax(x[u], T()));
+        const uint32_t ok = ordered_key(m);
+        const uint32_t wk = __reduce_max_sync(0xFFFFFFFFu, ok);
+        uint32_t idx = 0xFFFFFFFFu;
+        if (ok == wk) {
+#pragma unroll
+            for (int u = 0; u < kSegLoads; ++u)
+                if (idx == 0xFFFFFFFFu && vmax(x[u], T()) == m)
+                    idx = (rem + lane + 32 * u) * VW + vfirst(x[u], m, T());
+        }
+        idx = __reduce_min_sync(0xFFFFFFFFu, idx);
+        if (lane == 0) atomicMax(keys + r0, pack_ordered(wk, idx));
+        return;
+    }
+    const uint32_t bnd = s0 - rem + vrow;                      // first vector of row r0 + 1
     float b0 = -INFINITY, b1 = -INFINITY;
-    uint32_t i0 = (s0 - r0 * vrow) * VW, i1 = 0;
+    uint32_t i0 = rem * VW, i1 = 0;
 #pragma unroll
     for (int u = 0; u < kSegLoads; ++u) {
         const uint32_t v = s0 + lane + 32 * u;
@@ -229,7 +262,7 @@ __device__ __forceinline__ void segment_two_rows(const uint4* __restrict__ p, ui
             if (v < bnd) {
                 if (m > b0) {
                     b0 = m;
-                    i0 = (v - r0 * vrow) * VW + vfirst(x[u], m, T());
+                    i0 = (v - (s0 - rem)) * VW + vfirst(x[u], m, T());
                 }
             } else if (m > b1) {
                 b1 = m;
@@ -278,8 +311,18 @@ verify_argmax_kernel(const T* __restrict__ logits, int64_t N, int64_t V, int64_t
         const uint32_t nvec = static_cast<uint32_t>(N / VW), vrow = static_cast<uint32_t>(V / VW);
         const uint32_t stride = static_cast<uint32_t>(W) * seg;
         const uint4* p = reinterpret_cast<const uint4*>(logits);
-        for (uint32_t s0 = static_cast<uint32_t>(w) * seg; s0 < nvec; s0 += stride)
-            segment_two_rows<T>(p, s0, nvec, vrow, lane, keys);
+        const uint32_t dq = stride / vrow, dr = stride - dq * vrow;      // rows and vectors per stride
+        uint32_t s0 = static_cast<uint32_t>(w) * seg;
+        uint32_t r0 = s0 / vrow, rem = s0 - r0 * vrow;
+        for (; s0 < nvec; s0 += stride) {
+            segment_argmax<T>(p, s0, nvec, r0, rem, vrow, lane, keys);
+            r0 += dq;
+            rem += dr;
+            if (rem >= vrow) {
+                rem -= vrow;
+                ++r0;
+            }
+        }
     } else {
         constexpr int64_t SEG = kSegBytes / static_cast<int64_t>(sizeof(T));   // elements per segment
         for (int64_t e0 = w * SEG; e0 < N; e0 += W * SEG) {
