@@ -95,6 +95,17 @@ def barrier(ws):
         dist.barrier()
 
 
+def shard_seed(seed, rank):
+    """Each rank draws its own batch of sequences (weak scaling: independent shards)."""
+    return seed + 7919 * rank
+
+
+def steps_per_second(ws, steps, max_ms):
+    """Whole-job throughput: every rank ran `steps` steps of its own batch in at most
+    `max_ms` device milliseconds (the max over ranks)."""
+    return ws * steps / (max_ms / 1e3)
+
+
 def max_over_ranks(x, ws):
     if ws == 1:
         return x
@@ -284,7 +295,7 @@ def run_ours(args, ws_, rank, local):
     w = workload(args)
     if w.steps <= 1:
         raise SystemExit("the benchmark workload is the sustained decode loop (c5)")
-    w = w.replace(seed=w.seed + 7919 * rank)          # each rank its own shard of sequences
+    w = w.replace(seed=shard_seed(w.seed, rank))      # each rank its own shard of sequences
     K_steps, W_steps = args.steps, args.warmup
     t0 = time.perf_counter()
     loop = wl.DecodeLoop(w, steps=W_steps + K_steps, device=dev)
@@ -338,7 +349,7 @@ def run_ours(args, ws_, rank, local):
         step_ms_total = float(per_k.sum())                    # device ms over K steps
     step_ms_total = max_over_ranks(step_ms_total, ws_)
     ms_per_step = step_ms_total / K_steps
-    value = ws_ * K_steps / (step_ms_total / 1e3)
+    value = steps_per_second(ws_, K_steps, step_ms_total)
     st = path.status.cpu().numpy()
     cand_mean = float(cand_sum) / (K_steps * w.B)
     acc_mean = float(acc_sum) / (K_steps * w.B)
@@ -452,7 +463,7 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     return {"value": round(ws_ * steps / tot, 2), "unit": "steps/s",
             "ms_per_step": round(tot / steps * 1e3, 3),
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(h_res.numel() * 4),
-            "timing": "host wall clock per step: H2D of inputs from pinned memory, the five C-ABI "
+            "timing": "host wall clock per step: H2D of inputs from pinned memory, the step's C-ABI "
                       "calls, D2H of accept/next/seq_len/draft, synchronize"}
 
 
@@ -482,24 +493,40 @@ def oracle_step(orc, ids, L, H, A, logits, w, T_cap):
     return orc.verify_greedy(logits, draft, dl, ids=ids, seq_len=L, kv_keep=True)
 
 
-def cpu_baseline_from_loop(loop, path, w, budget_s=15.0, nseq=4, max_steps=64):
-    """Times the oracle on a bounded sample of the same loop: ``nseq`` sequences for
-    up to ``max_steps`` steps (or ``budget_s`` seconds of oracle time), each from the
-    GPU loop's own pre-step state; scaled to steps/s of the full batch."""
+def cpu_baseline_from_loop(loop, path, w, budget_s=20.0, nseq=64, max_steps=192):
+    """Times the oracle on a bounded sample of the same loop: the first ``nseq``
+    sequences for up to ``max_steps`` steps (or until ``budget_s`` seconds of oracle
+    time), every step from the GPU loop's own pre-step state; scaled to steps/s of the
+    full batch.
+
+    The oracle reads hidden rows and attention values only at the query position and
+    at occurrences of x_t.  The host copies hold exactly those (every other row of the
+    [nseq, T_cap, d] and [nseq, R, T_cap] arrays is a zero page that is never touched,
+    so the sample fits in host memory); logits are copied whole."""
     import oracle
     oracle.build()
     loop.reset()
-    sel = list(range(nseq))
-    Hs = _host(loop.H[sel])
+    nseq = min(nseq, w.B)
+    max_steps = min(max_steps, loop.steps)
+    Hs = np.zeros((nseq, loop.T_cap, w.d), np.uint16)       # zero pages until written
+    As = np.zeros((nseq, w.R, loop.T_cap), np.uint16)
     spent, n_steps = 0.0, 0
     for s in range(max_steps):
         loop.step_inputs(s)
-        ids = _host(loop.ids[sel]).copy()
-        L = _host(loop.seq_len[sel]).copy()
-        A = _host(loop.A[sel])
-        lg = _host(loop.logits[sel])
+        ids = _host(loop.ids[:nseq]).copy()
+        L = _host(loop.seq_len[:nseq]).copy()
+        for b in range(nseq):
+            t = int(L[b]) - 1
+            if t < 1:
+                continue
+            occ = np.nonzero(ids[b, :t] == ids[b, t])[0]
+            rows = np.unique(np.concatenate([occ[occ >= 1] - 1, [t - 1]]))
+            Hs[b, rows] = _host(loop.H[b, torch.from_numpy(rows).to(loop.device)])
+            if occ.size:
+                As[b][:, occ] = _host(loop.A[b][:, torch.from_numpy(occ).to(loop.device)])
+        lg = _host(loop.logits[:nseq])
         t0 = time.perf_counter()
-        oracle_step(oracle, ids, L, Hs, A, lg, w, loop.T_cap)
+        oracle_step(oracle, ids, L, Hs, As, lg, w, loop.T_cap)
         spent += time.perf_counter() - t0
         n_steps += 1
         path.run()                      # advance the GPU loop to the next state
@@ -508,8 +535,9 @@ def cpu_baseline_from_loop(loop, path, w, budget_s=15.0, nseq=4, max_steps=64):
     per_seq_step = spent / (n_steps * nseq)
     return {"value": round(1.0 / (per_seq_step * w.B), 4), "unit": "steps/s", "cores": 1,
             "kind": "oracle",
-            "sample": f"{nseq} of {w.B} sequences x {n_steps} steps of the same loop "
-                      f"({spent:.1f} s of single-threaded oracle time), scaled to the full batch"}
+            "sample": f"{nseq} of {w.B} sequences x {n_steps} consecutive steps of the same loop "
+                      f"({spent:.1f} s of single-threaded oracle time on the host), scaled to the full "
+                      f"batch of {w.B}"}
 
 
 # ----------------------------------------------------------------------------

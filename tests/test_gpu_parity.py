@@ -185,9 +185,12 @@ def test_extract_draft(lib, K):
 # ----------------------------------------------------------------------------
 # verification
 # ----------------------------------------------------------------------------
+# V * sizeof(dtype): >= 2 KB and a multiple of 16 bytes takes the streaming path (32000,
+# 1000 f32, 128256); a multiple of 16 bytes under 2 KB takes the short-row path (1000 and
+# 64 bf16); anything else takes element loads (1001, 999, 7).
 @pytest.mark.parametrize("V,dtype", [(32000, torch.bfloat16), (1000, torch.float32),
                                      (1001, torch.bfloat16), (999, torch.float32), (7, torch.bfloat16),
-                                     (128256, torch.bfloat16)])
+                                     (128256, torch.bfloat16), (1000, torch.bfloat16), (64, torch.bfloat16)])
 @pytest.mark.parametrize("K", [1, 10, 40])
 def test_verify_greedy(lib, V, dtype, K):
     rng = np.random.default_rng(V + K)

@@ -302,6 +302,7 @@ class DecodeLoop:
                  with_hidden: bool = True, with_attention: bool = True):
         self.w = w
         self.seed = w.seed if seed is None else seed
+        self.steps = steps
         self.T_cap = w.t_cap(steps)
         self.device = device
         gt, src = token_streams(w, self.T_cap, self.seed)
