@@ -72,8 +72,10 @@ def _configure(lib):
                                          P, P, P, P]
     lib.pldpo_extract_draft.argtypes = [P, i64, P, i64, P, i32, i32, P, P]
     lib.pldpo_verify_greedy.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64, P, i64, P, P]
+    lib.pldpo_verify_sample.argtypes = [P, i32, i32, i32, i32, ctypes.c_double, P, P, P, P, P, P, P, i64,
+                                        P, i64, P, P]
     for f in ("pldpo_find_candidates", "pldpo_rank_hidden", "pldpo_rank_attention",
-              "pldpo_extract_draft", "pldpo_verify_greedy"):
+              "pldpo_extract_draft", "pldpo_verify_greedy", "pldpo_verify_sample"):
         getattr(lib, f).restype = ctypes.c_int
 
 
@@ -217,6 +219,39 @@ def verify_greedy(logits, draft, draft_len, ids=None, seq_len=None, T_cap=None, 
                                        _ptr(seq_len), int(T_cap or 0), _ptr(kv), _ptr(st)),
            "verify_greedy")
     return dict(argmax=argmax, accept_len=acc, next_token=nxt, kv_keep_len=kv, status=st)
+
+
+def verify_sample(logits, uniforms, draft, draft_len, temperature=1.0, ids=None, seq_len=None,
+                  T_cap=None, kv_keep=False):
+    """Sec. 4.4 with sampling at ``temperature``: position i of sequence b draws the
+    smallest v whose cumulative softmax(logits / T) probability exceeds
+    uniforms[b, i] (float32 [B, K+1]).  Bookkeeping as verify_greedy.  Returns
+    dict(sampled, accept_len, next_token, kv_keep_len, status)."""
+    logits, dt = _elem(logits)
+    B, K1, V = logits.shape
+    K = K1 - 1
+    draft, draft_len = _i32(draft), _i32(draft_len)
+    assert draft.shape == (B, K)
+    u = np.ascontiguousarray(uniforms, dtype=np.float32)
+    assert u.shape == (B, K1)
+    sampled = np.zeros((B, K1), np.int32)
+    acc = np.zeros(B, np.int32)
+    nxt = np.zeros(B, np.int32)
+    st = np.zeros(B, np.uint32)
+    kv = np.zeros(B, np.int32) if kv_keep else None
+    stride = 0
+    if ids is not None:
+        assert ids.dtype == np.int32 and ids.flags.c_contiguous
+        T_cap, stride = ids.shape[1], ids.shape[1]
+    if seq_len is not None:
+        assert seq_len.dtype == np.int32 and seq_len.flags.c_contiguous
+        if T_cap is None:
+            raise ValueError("seq_len bookkeeping needs T_cap (or ids)")
+    _check(_load().pldpo_verify_sample(_ptr(logits), dt, B, K, V, float(temperature), _ptr(u), _ptr(draft),
+                                       _ptr(draft_len), _ptr(sampled), _ptr(acc), _ptr(nxt), _ptr(ids), stride,
+                                       _ptr(seq_len), int(T_cap or 0), _ptr(kv), _ptr(st)),
+           "verify_sample")
+    return dict(sampled=sampled, accept_len=acc, next_token=nxt, kv_keep_len=kv, status=st)
 
 
 def bf16_bits(x):

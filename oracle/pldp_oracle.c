@@ -263,6 +263,50 @@ int pldpo_extract_draft(const int32_t* ids, int64_t ids_stride, const int32_t* s
     return 0;
 }
 
+/* Acceptance and bookkeeping shared by both verifications, for sequence b
+ * whose K+1 target tokens (argmax or sampled) are tok[0..K]:
+ * n = first i < d with draft_i != tok_i (else d), bonus = tok_n, then the
+ * optional append to ids / seq_len and kv_keep_len = L + n.  Sec. 4.4. */
+static void orc_accept(int b, int K, int V, const int32_t* tok, const int32_t* draft,
+                       const int32_t* draft_len, int32_t* accept_len, int32_t* next_token,
+                       int32_t* ids, int64_t ids_stride, int32_t* seq_len, int64_t T_cap,
+                       int32_t* kv_keep_len, uint32_t* status) {
+    int64_t d = draft_len[b];
+    if (d < 0 || d > K) {
+        if (status) status[b] |= ORC_ST_DRAFT_LEN;
+        d = d < 0 ? 0 : K;
+    }
+    for (int64_t i = 0; i < d; ++i) {
+        int32_t t = draft[(int64_t)b * K + i];
+        if ((t < 0 || t >= V) && status) status[b] |= ORC_ST_TOKEN_RANGE;
+    }
+    int64_t n = d;
+    for (int64_t i = 0; i < d; ++i) {
+        if (draft[(int64_t)b * K + i] != tok[i]) { n = i; break; }
+    }
+    int32_t bonus = tok[n];
+    accept_len[b] = (int32_t)n;
+    next_token[b] = bonus;
+    if (!seq_len) return;
+    int64_t L = seq_len[b];
+    if (L < 1 || L > T_cap) {
+        if (status) status[b] |= ORC_ST_SEQ_LEN;
+        if (kv_keep_len) kv_keep_len[b] = -1;
+        return;
+    }
+    if (kv_keep_len) kv_keep_len[b] = (int32_t)(L + n);
+    if (L + n + 1 > T_cap) {
+        if (status) status[b] |= ORC_ST_CAPACITY;
+        return;
+    }
+    if (ids) {
+        int32_t* x = ids + (int64_t)b * ids_stride;
+        for (int64_t i = 0; i < n; ++i) x[L + i] = draft[(int64_t)b * K + i];
+        x[L + n] = bonus;
+    }
+    seq_len[b] = (int32_t)(L + n + 1);
+}
+
 /* --------------------------------------------------------------------------
  * Greedy verification (Sec. 4.4 with T = 0, and Sec. 3: one forward pass on
  * the draft gives K+1 distributions).  Row i of logits[b] is the target
@@ -299,42 +343,71 @@ int pldpo_verify_greedy(const void* logits, int dtype, int B, int K, int V,
             av[i] = bi;
             if (argmax) argmax[(int64_t)b * (K + 1) + i] = bi;
         }
-        int64_t d = draft_len[b];
-        if (d < 0 || d > K) {
-            if (status) status[b] |= ORC_ST_DRAFT_LEN;
-            d = d < 0 ? 0 : K;
-        }
-        for (int64_t i = 0; i < d; ++i) {
-            int32_t tok = draft[(int64_t)b * K + i];
-            if ((tok < 0 || tok >= V) && status) status[b] |= ORC_ST_TOKEN_RANGE;
-        }
-        int64_t n = d;
-        for (int64_t i = 0; i < d; ++i) {
-            if (draft[(int64_t)b * K + i] != av[i]) { n = i; break; }
-        }
-        int32_t bonus = av[n];
-        accept_len[b] = (int32_t)n;
-        next_token[b] = bonus;
-        if (!seq_len) continue;
-        int64_t L = seq_len[b];
-        if (L < 1 || L > T_cap) {
-            if (status) status[b] |= ORC_ST_SEQ_LEN;
-            if (kv_keep_len) kv_keep_len[b] = -1;
-            continue;
-        }
-        if (kv_keep_len) kv_keep_len[b] = (int32_t)(L + n);
-        if (L + n + 1 > T_cap) {
-            if (status) status[b] |= ORC_ST_CAPACITY;
-            continue;
-        }
-        if (ids) {
-            int32_t* x = ids + (int64_t)b * ids_stride;
-            for (int64_t i = 0; i < n; ++i) x[L + i] = draft[(int64_t)b * K + i];
-            x[L + n] = bonus;
-        }
-        seq_len[b] = (int32_t)(L + n + 1);
+        orc_accept(b, K, V, av, draft, draft_len, accept_len, next_token, ids, ids_stride,
+                   seq_len, T_cap, kv_keep_len, status);
     }
     free(av);
+    return 0;
+}
+
+/*
+ * Sampling verification -- Sec. 4.4 at temperature T > 0 (the paper's sampled
+ * runs use T = 1, Table 2): at each of the K+1 positions a token is drawn from
+ * p = softmax(logits / T), and the draft is accepted up to the first position
+ * whose drawn token differs from it; the token drawn there is the bonus.  For a
+ * draft that is a single token per position (as PLD+'s is), this accepts token
+ * i with probability p(draft_i) and, on a rejection, draws the bonus from p
+ * restricted to the other tokens: exactly what sampling from the target alone
+ * would emit.
+ *
+ * The random numbers are the caller's: position i of sequence b takes
+ * u = uniforms[b, i] and draws the smallest v whose cumulative probability
+ * sum_{v' <= v} p_v' exceeds u (inverse-CDF sampling).
+ * READING: u outside [0, 1) is clamped into it; the paper does not say how its
+ * samples are drawn, only that they are.
+ * Finite logits only.  Probabilities are carried in double precision: with
+ * m the row maximum, w_v = exp((l_v - m) / T), Z = sum w_v, and the draw is the
+ * first v with sum_{v' <= v} w_v' > u * Z.
+ */
+int pldpo_verify_sample(const void* logits, int dtype, int B, int K, int V, double temperature,
+                        const float* uniforms, const int32_t* draft, const int32_t* draft_len,
+                        int32_t* sampled, int32_t* accept_len, int32_t* next_token,
+                        int32_t* ids, int64_t ids_stride, int32_t* seq_len, int64_t T_cap,
+                        int32_t* kv_keep_len, uint32_t* status) {
+    if (B < 0 || K < 1 || V < 1 || (dtype != ORC_F32 && dtype != ORC_BF16)) return 1;
+    if (!(temperature > 0.0) || isinf(temperature)) return 1;
+    if ((ids || kv_keep_len) && !seq_len) return 1;
+    int32_t* yv = (int32_t*)malloc(sizeof(int32_t) * (size_t)(K + 1));
+    if (!yv) return 2;
+    for (int b = 0; b < B; ++b) {
+        for (int i = 0; i <= K; ++i) {
+            int64_t row = ((int64_t)b * (K + 1) + i) * (int64_t)V;
+            double m = orc_load(logits, dtype, row);
+            for (int64_t v = 1; v < V; ++v) {
+                double x = orc_load(logits, dtype, row + v);
+                if (x > m) m = x;
+            }
+            double Z = 0.0;
+            for (int64_t v = 0; v < V; ++v) Z += exp((orc_load(logits, dtype, row + v) - m) / temperature);
+            double u = (double)uniforms[(int64_t)b * (K + 1) + i];
+            if (!(u >= 0.0)) u = 0.0;                                 /* also NaN */
+            if (u >= 1.0) u = nextafter(1.0, 0.0);
+            double target = u * Z, c = 0.0;
+            int32_t y = -1, last_pos = 0;
+            for (int64_t v = 0; v < V; ++v) {
+                double w = exp((orc_load(logits, dtype, row + v) - m) / temperature);
+                if (w > 0.0) last_pos = (int32_t)v;
+                c += w;
+                if (c > target) { y = (int32_t)v; break; }
+            }
+            if (y < 0) y = last_pos;     /* unreachable: the sum ends at Z > u * Z */
+            yv[i] = y;
+            if (sampled) sampled[(int64_t)b * (K + 1) + i] = y;
+        }
+        orc_accept(b, K, V, yv, draft, draft_len, accept_len, next_token, ids, ids_stride,
+                   seq_len, T_cap, kv_keep_len, status);
+    }
+    free(yv);
     return 0;
 }
 

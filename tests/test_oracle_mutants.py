@@ -56,12 +56,22 @@ MUTANTS = [
     ("argmax keeps the last of equal maxima",
      "if (x > best) { best = x; bi = (int32_t)v; }", "if (x >= best) { best = x; bi = (int32_t)v; }"),
     ("bonus token from the row after the whole draft",
-     "int32_t bonus = av[n];", "int32_t bonus = av[d];"),
+     "int32_t bonus = tok[n];", "int32_t bonus = tok[d];"),
     ("kv_keep counts the bonus token",
      "kv_keep_len[b] = (int32_t)(L + n);", "kv_keep_len[b] = (int32_t)(L + n + 1);"),
     ("accept ignores the first draft token",
-     "for (int64_t i = 0; i < d; ++i) {\n            if (draft[(int64_t)b * K + i] != av[i]) { n = i; break; }",
-     "for (int64_t i = 1; i < d; ++i) {\n            if (draft[(int64_t)b * K + i] != av[i]) { n = i; break; }"),
+     "for (int64_t i = 0; i < d; ++i) {\n        if (draft[(int64_t)b * K + i] != tok[i]) { n = i; break; }",
+     "for (int64_t i = 1; i < d; ++i) {\n        if (draft[(int64_t)b * K + i] != tok[i]) { n = i; break; }"),
+    ("sampling draws where the cumulative sum only reaches u",
+     "if (c > target) { y = (int32_t)v; break; }", "if (c >= target) { y = (int32_t)v; break; }"),
+    ("sampling multiplies by the temperature",
+     "double w = exp((orc_load(logits, dtype, row + v) - m) / temperature);",
+     "double w = exp((orc_load(logits, dtype, row + v) - m) * temperature);"),
+    ("sampling takes the next position's uniform",
+     "double u = (double)uniforms[(int64_t)b * (K + 1) + i];",
+     "double u = (double)uniforms[(int64_t)b * (K + 1) + (i + 1) % (K + 1)];"),
+    ("sampling bonus from the argmax instead of the draw",
+     "yv[i] = y;", "yv[i] = (i == K) ? 0 : y;"),
 ]
 
 

@@ -9,12 +9,17 @@
 * Attention ranking (Eq. 2): ``numpy`` max/sum over the selected rows.
 * Verification (Sec. 4.4): ``numpy.argmax`` (documented first occurrence) and
   the accept-length invariants.
+* Sampling verification (Sec. 4.4 at T > 0): ``scipy.special.softmax`` and
+  ``numpy.searchsorted`` over a grid of uniforms (inverse-CDF sampling), the
+  low-temperature limit (argmax), equal logits (floor(u V)), zero-probability
+  tokens, and the acceptance rate p(draft token) that makes the step lossless.
 """
 import itertools
 
 import numpy as np
 import pytest
 from scipy.spatial.distance import cosine as scipy_cosine
+from scipy.special import softmax as scipy_softmax
 
 
 # ----------------------------------------------------------------------------
@@ -247,3 +252,110 @@ def test_verify_matches_numpy_argmax_and_invariants(orc, bf16):
         else:
             assert lens[b] == lens0[b] and out["status"][b] == orc.ST_CAPACITY
             assert np.array_equal(ids[b], ids0[b])
+
+
+# ----------------------------------------------------------------------------
+# sampling verification
+# ----------------------------------------------------------------------------
+def _grid_draws(orc, logits_row, T, us):
+    """Draws of the oracle for one logits row under each uniform in ``us``
+    (one sequence per uniform, K = 1; row 1 gets the uniform reversed)."""
+    N, V = len(us), logits_row.size
+    logits = np.broadcast_to(logits_row.astype(np.float32), (N, 2, V)).copy()
+    u = np.stack([us, us[::-1]], axis=1).astype(np.float32)
+    out = orc.verify_sample(logits, u, np.zeros((N, 1), np.int32), np.zeros(N, np.int32), temperature=T)
+    return out["sampled"][:, 0], out["sampled"][:, 1][::-1]
+
+
+@pytest.mark.parametrize("T", [1.0, 0.5, 2.0])
+def test_sample_is_inverse_cdf_of_softmax(orc, T):
+    rng = np.random.default_rng(int(T * 10))
+    row = rng.normal(0, 1.5, size=7).astype(np.float32)
+    cdf = np.cumsum(scipy_softmax(row.astype(np.float64) / T))
+    us = ((np.arange(4000) + 0.5) / 4000).astype(np.float32)
+    keep = np.min(np.abs(us.astype(np.float64)[:, None] - cdf[None, :]), axis=1) > 1e-9
+    want = np.searchsorted(cdf, us.astype(np.float64), side="right")   # smallest v with cdf_v > u
+    got0, got1 = _grid_draws(orc, row, T, us)
+    assert np.array_equal(got0[keep], want[keep]) and np.array_equal(got1[keep], want[keep])
+    # the frequencies over the grid are the probabilities
+    freq = np.bincount(got0, minlength=7) / us.size
+    assert np.allclose(freq, np.diff(np.concatenate([[0.0], cdf])), atol=1.0 / us.size)
+
+
+def test_sample_hand_worked(orc):
+    # logits ln 1, ln 2, ln 3 at T = 1: p = 1/6, 2/6, 3/6, cumulative 1/6, 1/2, 1
+    row = np.log(np.array([1.0, 2.0, 3.0])).astype(np.float32)
+    us = np.array([0.0, 0.1, 0.17, 0.3, 0.49, 0.51, 0.99], np.float32)
+    got, _ = _grid_draws(orc, row, 1.0, us)
+    assert got.tolist() == [0, 0, 1, 1, 1, 2, 2]
+
+
+def test_sample_low_temperature_is_argmax(orc):
+    rng = np.random.default_rng(5)
+    row = (rng.permutation(40) * 0.05).astype(np.float32)            # distinct, gaps >= 0.05
+    us = np.linspace(1e-6, 0.999, 300).astype(np.float32)       # u = 0 draws the first p > 0
+    got, _ = _grid_draws(orc, row, 1e-3, us)
+    assert (got == np.argmax(row)).all()
+
+
+def test_sample_equal_logits_is_floor_uV(orc):
+    V = 12
+    us = ((np.arange(600) + 0.25) / 600).astype(np.float32)
+    got, _ = _grid_draws(orc, np.full(V, 0.7, np.float32), 1.0, us)
+    want = np.floor(us.astype(np.float64) * V).astype(int)
+    near = np.abs(us.astype(np.float64) * V - np.round(us.astype(np.float64) * V)) < 1e-6
+    assert np.array_equal(got[~near], want[~near])
+
+
+def test_sample_never_draws_zero_probability(orc):
+    row = np.array([-1000.0, 0.0, -1000.0, 0.5, -1000.0], np.float32)
+    us = np.array([0.0, 1e-12, 0.3, 0.999999], np.float32)
+    got, _ = _grid_draws(orc, row, 1.0, us)
+    assert set(got.tolist()) <= {1, 3} and got[0] == 1
+
+
+def test_sample_acceptance_rate_is_p_of_draft(orc):
+    """The draft token is accepted exactly when the draw equals it, so over a grid of
+    uniforms the accepted fraction is p(draft); on a rejection the bonus is the draw
+    (never the draft token), and with every position accepted the bonus is the draw
+    at position K."""
+    row = np.array([0.3, -0.2, 1.1, 0.0], np.float32)
+    p = scipy_softmax(row.astype(np.float64))
+    N = 5000
+    us = ((np.arange(N) + 0.5) / N).astype(np.float32)
+    for tok in range(4):
+        logits = np.broadcast_to(row, (N, 2, 4)).copy()
+        u = np.stack([us, us[::-1]], axis=1)
+        draft = np.full((N, 1), tok, np.int32)
+        out = orc.verify_sample(logits, u, draft, np.ones(N, np.int32))
+        acc = out["accept_len"]
+        assert abs(acc.mean() - p[tok]) <= 2.0 / N
+        rej = acc == 0
+        assert (out["next_token"][rej] != tok).all()
+        assert np.array_equal(out["next_token"][rej], out["sampled"][rej, 0])
+        assert np.array_equal(out["next_token"][~rej], out["sampled"][~rej, 1])
+
+
+def test_sample_bookkeeping_matches_greedy_rules(orc):
+    rng = np.random.default_rng(77)
+    B, K, V, T_cap = 32, 5, 9, 16
+    logits = rng.normal(0, 2, size=(B, K + 1, V)).astype(np.float32)
+    u = rng.random((B, K + 1)).astype(np.float32)
+    first = orc.verify_sample(logits, u, np.zeros((B, K), np.int32), np.zeros(B, np.int32))
+    y = first["sampled"]
+    draft = np.where(rng.random((B, K)) < 0.7, y[:, :K], rng.integers(0, V, size=(B, K))).astype(np.int32)
+    dlen = rng.integers(0, K + 1, size=B).astype(np.int32)
+    ids = rng.integers(0, V, size=(B, T_cap)).astype(np.int32)
+    lens = rng.integers(1, T_cap + 1, size=B).astype(np.int32)
+    ids0, lens0 = ids.copy(), lens.copy()
+    out = orc.verify_sample(logits, u, draft, dlen, ids=ids, seq_len=lens, kv_keep=True)
+    assert np.array_equal(out["sampled"], y)
+    for b in range(B):
+        mism = [i for i in range(dlen[b]) if draft[b, i] != y[b, i]]
+        n = mism[0] if mism else dlen[b]
+        assert out["accept_len"][b] == n and out["next_token"][b] == y[b, n]
+        assert out["kv_keep_len"][b] == lens0[b] + n
+        if lens0[b] + n + 1 <= T_cap:
+            assert ids[b, lens0[b]:lens[b]].tolist() == list(draft[b, :n]) + [y[b, n]]
+        else:
+            assert out["status"][b] == orc.ST_CAPACITY and np.array_equal(ids[b], ids0[b])
