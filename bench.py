@@ -62,6 +62,8 @@ def parse():
     ap.add_argument("--separate", action="store_true",
                     help="draft with the four separate calls instead of the fused launch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sample", action="store_true",
+                    help="skip the separate timing of sampling verification (T = 1) on the same logits")
     ap.add_argument("--ref-seqs", type=int, default=2, help="sequences per oracle step (reference arm)")
     ap.add_argument("--batch", type=int, default=None, help="override the batch (not the headline)")
     ap.add_argument("--hidden-width", type=int, default=None,
@@ -414,11 +416,51 @@ def run_ours(args, ws_, rank, local):
                   "lossless_vs_ground_truth": lossless, "setup_s": round(setup_s, 1),
                   "timed_loop_wall_s": round(wall, 3)},
     }
+    if not args.no_sample:
+        out["sampling_verify"] = time_sampling_verify(pk, loop, w, flush_l2, peak)
     if not args.no_e2e:
         out["e2e"] = run_e2e(pk, loop, path, K_steps, W_steps, ws_)
     if rank == 0 and ws_ == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline_from_loop(loop, path, w)
     return out
+
+
+def time_sampling_verify(pk, loop, w, flush_l2, peak, calls=64, warm=4, temperature=1.0):
+    """Sampling verification (Sec. 4.4 at T = 1) on the loop's logits [B, K+1, V]:
+    the same bytes as greedy verification, timed per call with CUDA events, L2
+    flushed before each call, no bookkeeping (the loop state is left alone)."""
+    dev = loop.device
+    B, K1 = w.B, w.K + 1
+    gen = torch.Generator(device=dev).manual_seed(w.seed + 17)
+    u = torch.rand((B, K1), generator=gen, device=dev)
+    ws = torch.empty(pk.pldp_verify_sample_workspace_size(B, w.K, w.V, loop.logits.dtype), dtype=torch.uint8,
+                     device=dev)
+    acc, nxt = torch.zeros(B, dtype=torch.int32, device=dev), torch.zeros(B, dtype=torch.int32, device=dev)
+    sampled = torch.zeros((B, K1), dtype=torch.int32, device=dev)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(calls)]
+    s = torch.cuda.current_stream()
+    for i in range(warm + calls):
+        flush_l2(i)
+        if i >= warm:
+            ev[i - warm][0].record(s)
+        pk.pldp_verify_sample(loop.logits, u, path_draft(loop, w), torch.full((B,), w.K, dtype=torch.int32,
+                              device=dev), acc, nxt, ws, temperature=temperature, sampled=sampled)
+        if i >= warm:
+            ev[i - warm][1].record(s)
+    torch.cuda.synchronize()
+    us = float(np.mean([a.elapsed_time(b) for a, b in ev])) * 1e3
+    by = 2.0 * B * K1 * w.V
+    return {"temperature": temperature, "calls": calls, "us_per_call": round(us, 2),
+            "achieved_gbs": round(by / (us * 1e-6) / 1e9, 1), "peak_gbs": peak,
+            "frac": round(by / (us * 1e-6) / 1e9 / peak, 4), "algorithmic_bytes": by,
+            "launches_per_call": 2,
+            "timing": "CUDA events around each pldp_verify_sample call, L2 flushed before each"}
+
+
+def path_draft(loop, w):
+    """A draft for timing: the ground-truth continuation of every sequence."""
+    pos = loop.seq_len.long()[:, None] + torch.arange(w.K, device=loop.device)[None]
+    return loop.gt.gather(1, pos.clamp(max=loop.gt.shape[1] - 1)).to(torch.int32).contiguous()
 
 
 def run_e2e(pk, loop, path, K_steps, W_steps, ws_):

@@ -306,6 +306,46 @@ PLDP_API pldp_status pldp_verify_greedy(const void* logits, pldp_dtype dtype, in
                                         size_t workspace_bytes, void* stream);
 
 /*
+ * Sampling verification -- Sec. 4.4 at temperature T > 0 (the paper's sampled
+ * runs use T = 1, Table 2).  Position i of sequence b draws
+ *   y_i = the smallest v with sum_{v' <= v} p_v' > u[b, i],
+ *         p = softmax(logits[b, i] / T)                  (inverse-CDF sampling)
+ * from the caller's uniform u[b, i]; then, as for greedy verification,
+ *   n = first i < draft_len[b] with draft[b, i] != y_i, else draft_len[b];
+ *   bonus = y_n.
+ * For a draft with one token per position (PLD+'s draft) this accepts draft_i
+ * with probability p(draft_i) and on a rejection draws the bonus from p
+ * restricted to the other tokens: the step emits exactly what sampling from the
+ * target alone would.  The random numbers are inputs: the same uniforms give
+ * the same draws.
+ *
+ *  logits        dtype [B, K+1, V], contiguous, finite.  Fast path when logits is
+ *                16-byte aligned and V * sizeof(dtype) is a multiple of 16.
+ *  temperature   T > 0, finite (else PLDP_ERR_INVALID_ARG).
+ *  uniforms      float [B, K+1]; values outside [0, 1) are clamped into it.
+ *  sampled       int32 [B, K+1] out or NULL: every y_i.
+ *  draft, draft_len, accept_len, next_token, ids, ids_stride, seq_len, T_cap,
+ *  kv_keep_len, status   as pldp_verify_greedy.
+ *  workspace     device scratch of pldp_verify_sample_workspace_size(B, K, V, dtype)
+ *                bytes, 16-byte aligned (no zeroing needed).
+ * Probabilities are computed in fp32 (per-2 KB-piece maxima and sums of
+ * exp2(log2(e) (l - max) / T)); a draw can differ from the exact draw only when
+ * u lies within fp32 rounding (~1e-6) of a boundary of the cumulative
+ * distribution.  K + 1 <= 12288.
+ */
+PLDP_API pldp_status pldp_verify_sample(const void* logits, pldp_dtype dtype, int B, int K, int V,
+                                        float temperature, const float* uniforms,
+                                        const int32_t* draft, const int32_t* draft_len,
+                                        int32_t* sampled, int32_t* accept_len,
+                                        int32_t* next_token, int32_t* ids, int64_t ids_stride,
+                                        int32_t* seq_len, int64_t T_cap, int32_t* kv_keep_len,
+                                        uint32_t* status, void* workspace,
+                                        size_t workspace_bytes, void* stream);
+
+/* Bytes of workspace pldp_verify_sample needs (0 if invalid). */
+PLDP_API size_t pldp_verify_sample_workspace_size(int B, int K, int V, pldp_dtype dtype);
+
+/*
  * Greedy verification without a caller workspace.  The paper has no counterpart:
  * this is a deployment convenience.  Same arguments, results and status bits as
  * pldp_verify_greedy, minus the workspace.

@@ -119,6 +119,11 @@ def _load():
             lib.pldp_verify_greedy_noalloc.restype = ctypes.c_int
             lib.pldp_verify_workspace_size.argtypes = [i32, i32, i32]
             lib.pldp_verify_workspace_size.restype = sz
+            lib.pldp_verify_sample.argtypes = [P, i32, i32, i32, i32, f32, P, P, P, P, P, P, P, i64, P,
+                                               i64, P, P, P, sz, P]
+            lib.pldp_verify_sample.restype = ctypes.c_int
+            lib.pldp_verify_sample_workspace_size.argtypes = [i32, i32, i32, i32]
+            lib.pldp_verify_sample_workspace_size.restype = sz
             lib.pldp_last_error.argtypes = []
             lib.pldp_last_error.restype = ctypes.c_char_p
             lib.pldp_version.argtypes = []
@@ -315,6 +320,37 @@ def pldp_verify_greedy(logits, draft, draft_len, accept_len, next_token, workspa
         _dense(logits, "logits"), _code(logits.dtype), B, K, V, _dense(draft, "draft", torch.int32),
         _dense(draft_len, "draft_len", torch.int32),
         _dense(argmax, "argmax", torch.int32, allow_none=True),
+        _dense(accept_len, "accept_len", torch.int32), _dense(next_token, "next_token", torch.int32),
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True), T_cap,
+        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True),
+        _dense(status, "status", None, allow_none=True), _dense(workspace, "workspace"),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def pldp_verify_sample_workspace_size(B, K, V, dtype=torch.bfloat16) -> int:
+    return int(_load().pldp_verify_sample_workspace_size(B, K, V, _code(dtype)))
+
+
+def pldp_verify_sample(logits, uniforms, draft, draft_len, accept_len, next_token, workspace,
+                       temperature=1.0, sampled=None, ids=None, seq_len=None, kv_keep_len=None,
+                       status=None, T_cap=None, stream=None):
+    """Sec. 4.4 with sampling at ``temperature``: position i of sequence b draws the
+    smallest v whose cumulative softmax(logits / T) probability exceeds uniforms[b, i]
+    (float32 [B, K+1] CUDA tensor); acceptance and bookkeeping as pldp_verify_greedy.
+    workspace: uint8 CUDA tensor of pldp_verify_sample_workspace_size(B, K, V, dtype) bytes."""
+    B, K1, V = logits.shape
+    K = K1 - 1
+    if draft.shape != (B, K):
+        raise ValueError("draft must be [B, K] with K = logits.shape[1] - 1")
+    if uniforms.shape != (B, K1):
+        raise ValueError("uniforms must be [B, K+1]")
+    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids")
+    if T_cap is None:
+        T_cap = T
+    _check("pldp_verify_sample", _load().pldp_verify_sample(
+        _dense(logits, "logits"), _code(logits.dtype), B, K, V, float(temperature),
+        _dense(uniforms, "uniforms", torch.float32), _dense(draft, "draft", torch.int32),
+        _dense(draft_len, "draft_len", torch.int32), _dense(sampled, "sampled", torch.int32, allow_none=True),
         _dense(accept_len, "accept_len", torch.int32), _dense(next_token, "next_token", torch.int32),
         p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True), T_cap,
         _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True),

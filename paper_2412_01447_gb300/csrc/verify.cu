@@ -142,14 +142,31 @@ struct VerifyArgs {
     int B, K, V;
 };
 
-// Accept/bonus/append for sequence b, by one warp, once the row keys are final.
-// Everything it reads is requested up front (one round trip when K < 32).
-__device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
+// Where the finish reads the K+1 target tokens of a sequence: the greedy row keys
+// (argmax packed in the low word; the keys are returned to zero afterwards) or
+// the draws of sampling verification, staged in shared memory.
+struct KeyTokens {
+    unsigned long long* keys;   // [K+1] of this sequence
+    __device__ __forceinline__ int at(int i) const { return static_cast<int>(key_index(__ldcg(keys + i))); }
+    __device__ __forceinline__ void release(int K1, int lane) const {
+        for (int i = lane; i < K1; i += 32) keys[i] = 0ull;
+    }
+};
+struct SharedTokens {
+    const int32_t* tok;          // shared memory, [K+1]
+    __device__ __forceinline__ int at(int i) const { return tok[i]; }
+    __device__ __forceinline__ void release(int, int) const {}
+};
+
+// Accept/bonus/append for sequence b, by one warp, once its K+1 target tokens are
+// final.  Everything it reads is requested up front (one round trip when K < 32).
+// Sec. 4.4: n = first i < d with draft_i != target_i (else d), bonus = target_n.
+template <typename Src>
+__device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane, const Src& src) {
     const int K1 = a.K + 1;
-    unsigned long long* keys = a.row_keys + b * K1;
     const int d_in = a.draft_len[b];
     const int64_t L = a.seq_len ? a.seq_len[b] : 0;
-    const unsigned long long k_first = lane < K1 ? __ldcg(keys + lane) : 0ull;
+    const int t_first = lane < K1 ? src.at(lane) : 0;
     const int tok_first = lane < a.K ? a.draft[b * a.K + lane] : 0;
     uint32_t st = 0;
     int d = d_in;
@@ -159,13 +176,10 @@ __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
     }
     int n = d;
     bool range_bad = false;
-    int am_first = 0;
     for (int i0 = 0; i0 < K1; i0 += 32) {
         const int i = i0 + lane;
-        const unsigned long long kk = i0 == 0 ? k_first : (i < K1 ? __ldcg(keys + i) : 0ull);
+        const int am = i0 == 0 ? t_first : (i < K1 ? src.at(i) : 0);
         const int tok = i0 == 0 ? tok_first : (i < a.K ? a.draft[b * a.K + i] : 0);
-        const int am = static_cast<int>(key_index(kk));
-        if (i0 == 0) am_first = am;
         if (i < K1 && a.argmax) a.argmax[b * K1 + i] = am;
         const bool in_draft = i < d;
         range_bad |= in_draft && (tok < 0 || tok >= a.V);
@@ -173,10 +187,9 @@ __device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane) {
         if (n == d && mism) n = i0 + __ffs(mism) - 1;
     }
     if (__any_sync(0xFFFFFFFFu, range_bad)) st |= PLDP_ST_TOKEN_RANGE;
-    const int bonus = n < 32 ? __shfl_sync(0xFFFFFFFFu, am_first, n)
-                             : static_cast<int>(key_index(__ldcg(keys + n)));
+    const int bonus = n < 32 ? __shfl_sync(0xFFFFFFFFu, t_first, n) : src.at(n);
     __syncwarp();
-    for (int i = lane; i < K1; i += 32) keys[i] = 0ull;
+    src.release(K1, lane);
 
     if (lane == 0) {
         a.accept_len[b] = n;
@@ -336,7 +349,7 @@ verify_argmax_kernel(const T* __restrict__ logits, int64_t N, int64_t V, int64_t
 __global__ void __launch_bounds__(kThreads) verify_finish_kernel(VerifyArgs a) {
     pdl_enter();                                           // the pass's keys are final
     const int64_t b = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
-    if (b < a.B) finish_sequence(a, b, threadIdx.x & 31);
+    if (b < a.B) finish_sequence(a, b, threadIdx.x & 31, KeyTokens{a.row_keys + b * (a.K + 1)});
 }
 
 size_t keys_bytes(int B, int K) {
@@ -467,6 +480,354 @@ extern "C" PLDP_API pldp_status pldp_verify_greedy(
                                      ids_stride, seq_len, T_cap, kv_keep_len, status);
     return launch_verify(logits, dtype, a, workspace, static_cast<cudaStream_t>(stream),
                          "verify_greedy");
+}
+
+// ---------------------------------------------------------------------------
+// Sampling verification (Sec. 4.4 at temperature T > 0).
+//
+// Position i of sequence b draws the smallest v whose cumulative probability
+// under p = softmax(logits[b, i] / T) exceeds the caller's uniform u[b, i]
+// (inverse-CDF sampling); the draft is then accepted up to the first position
+// whose draw differs from it, and the draw there is the bonus -- for a
+// single-token-per-position draft this is exactly what sampling from the target
+// would emit.
+//
+// 1. A stats pass streams the logits once, in the same moving-window order as
+//    the greedy pass, over units of (row, 2 KB piece): per piece the max M_k and
+//    S_k = sum 2^((l - M_k) log2(e) / T).  No atomics: each piece has its slot.
+// 2. One CTA per sequence, one warp per row: the piece weights
+//    W_k = S_k 2^((M_k - M) log2(e) / T) against the row max M give the total Z
+//    (a warp scan over the pieces, run twice in the same order, so the second
+//    run's crossing of u Z always exists), which picks the piece; the warp then
+//    rereads that one piece and finds the element where the running sum of its
+//    weights passes the same fraction of the piece.  fp32 throughout: a draw can
+//    differ from the exact one only when u lies within rounding (~1e-6) of a
+//    boundary of the cumulative distribution.
+// ---------------------------------------------------------------------------
+namespace pldp {
+namespace {
+
+constexpr int64_t kPieceBytes = 2048;
+
+struct SampleArgs {
+    VerifyArgs v;                   // draft, bookkeeping; v.argmax receives the draws
+    const float* uniforms;          // [B*(K+1)]
+    const float2* stats;            // [rows * npieces]: (M_k, S_k)
+    float c;                        // log2(e) / T
+    int npieces;                    // pieces per row
+    int P;                          // elements per piece
+};
+
+__device__ __forceinline__ float ex2_approx(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// The elements of one 16-byte vector as floats.
+__device__ __forceinline__ void unpack(const uint4& x, float (&e)[8], __nv_bfloat16) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        e[2 * k] = __uint_as_float(w[k] << 16);
+        e[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+    }
+}
+__device__ __forceinline__ void unpack(const uint4& x, float (&e)[8], float) {
+    e[0] = __uint_as_float(x.x);
+    e[1] = __uint_as_float(x.y);
+    e[2] = __uint_as_float(x.z);
+    e[3] = __uint_as_float(x.w);
+}
+
+__device__ __forceinline__ float warp_max_f(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+    return v;
+}
+
+// 1. per-piece (max, sum of weights).  Units u = row * npieces + piece, warp w of W
+// takes units w, w + W, ...; piece k of row r covers elements [k P, min((k+1) P, V)).
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads, VEC ? kPassBlocksPerSm : 4)
+sample_stats_kernel(const T* __restrict__ logits, int64_t V, int64_t rows, int npieces, int P, float c,
+                    int64_t W, float2* __restrict__ stats) {
+    pdl_enter();
+    const int lane = threadIdx.x & 31;
+    const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
+    const int64_t units = rows * npieces;
+    int64_t r = w / npieces, k = w - r * npieces;
+    const int64_t dr = W / npieces, dk = W - dr * npieces;
+    for (int64_t u = w; u < units; u += W) {
+        const int64_t e0 = static_cast<int64_t>(k) * P;
+        const int64_t n = (V - e0 < P) ? V - e0 : P;            // elements in this piece
+        const T* piece = logits + r * V + e0;
+        float m = -INFINITY, sum = 0.f, M;
+        if constexpr (VEC) {
+            // whole 16-byte vectors: V, hence every piece length, is a multiple of one
+            constexpr int VW = 16 / static_cast<int>(sizeof(T));
+            const uint4* pv = reinterpret_cast<const uint4*>(piece);
+            uint4 raw[kSegLoads];
+#pragma unroll
+            for (int q = 0; q < kSegLoads; ++q) {
+                const int vi = lane + 32 * q;
+                if (static_cast<int64_t>(vi) * VW < n) raw[q] = ld_stream16(pv + vi);
+            }
+#pragma unroll
+            for (int q = 0; q < kSegLoads; ++q)
+                if (static_cast<int64_t>(lane + 32 * q) * VW < n) m = fmaxf(m, vmax(raw[q], T()));
+            M = warp_max_f(m);
+            if (M > -INFINITY) {
+                const float mc = M * c;
+#pragma unroll
+                for (int q = 0; q < kSegLoads; ++q) {
+                    if (static_cast<int64_t>(lane + 32 * q) * VW >= n) continue;
+                    float e[8];
+                    unpack(raw[q], e, T());
+#pragma unroll
+                    for (int j = 0; j < VW; ++j) sum += ex2_approx(fmaf(e[j], c, -mc));
+                }
+            }
+        } else {
+            constexpr int PER = static_cast<int>(kPieceBytes / sizeof(T)) / 32;
+            float x[PER];
+#pragma unroll
+            for (int q = 0; q < PER; ++q) {
+                const int ei = lane + 32 * q;
+                x[q] = ei < n ? to_f32(piece[ei]) : -INFINITY;
+                m = fmaxf(m, x[q]);
+            }
+            M = warp_max_f(m);
+            if (M > -INFINITY) {
+                const float mc = M * c;
+#pragma unroll
+                for (int q = 0; q < PER; ++q)
+                    if (x[q] > -INFINITY) sum += ex2_approx(fmaf(x[q], c, -mc));
+            }
+        }
+        sum = warp_sum(sum);
+        if (lane == 0) stats[u] = make_float2(M, sum);
+        r += dr;
+        k += dk;
+        if (k >= npieces) {
+            k -= npieces;
+            ++r;
+        }
+    }
+}
+
+// Weight of piece k of a row against the row max M (0 for an empty piece).
+__device__ __forceinline__ float piece_weight(const float2* st, int k, int npieces, float Mc, float c) {
+    if (k >= npieces) return 0.f;
+    const float2 s = __ldcg(st + k);
+    return s.x > -INFINITY ? s.y * ex2_approx(fmaf(s.x, c, -Mc)) : 0.f;
+}
+
+__device__ __forceinline__ float warp_incl_scan(float v, int lane) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const float t = __shfl_up_sync(0xFFFFFFFFu, v, o);
+        if (lane >= o) v += t;
+    }
+    return v;
+}
+
+// The draw of row r (one warp).
+template <typename T, bool VEC>
+__device__ int sample_row(const T* __restrict__ logits, const SampleArgs& a, int64_t r, int lane) {
+    const int64_t V = a.v.V;
+    const int np = a.npieces;
+    const float2* st = a.stats + r * np;
+    float m = -INFINITY;
+    for (int k = lane; k < np; k += 32) m = fmaxf(m, __ldcg(st + k).x);
+    const float M = warp_max_f(m);
+    const float Mc = M * a.c;
+    // the total, then the first piece whose running total passes u Z (same sums, same order)
+    float base = 0.f;
+    for (int k0 = 0; k0 < np; k0 += 32) {
+        const float incl = warp_incl_scan(piece_weight(st, k0 + lane, np, Mc, a.c), lane);
+        base += __shfl_sync(0xFFFFFFFFu, incl, 31);
+    }
+    float u = a.uniforms[r];
+    if (!(u >= 0.f)) u = 0.f;
+    if (u >= 1.f) u = __uint_as_float(0x3F7FFFFFu);               // largest float below 1
+    const float target = u * base;
+    int ks = -1;
+    float before = 0.f, wk = 0.f;
+    float run = 0.f;
+    for (int k0 = 0; k0 < np && ks < 0; k0 += 32) {
+        const float wv = piece_weight(st, k0 + lane, np, Mc, a.c);
+        const float incl = warp_incl_scan(wv, lane);
+        const unsigned hit = __ballot_sync(0xFFFFFFFFu, run + incl > target && k0 + lane < np);
+        if (hit) {
+            const int f = __ffs(hit) - 1;
+            ks = k0 + f;
+            before = run + __shfl_sync(0xFFFFFFFFu, incl - wv, f);
+            wk = __shfl_sync(0xFFFFFFFFu, wv, f);
+        }
+        run += __shfl_sync(0xFFFFFFFFu, incl, 31);
+    }
+    if (ks < 0) {                                                 // rounding: the last piece with weight
+        ks = np - 1;
+        for (; ks > 0; --ks)
+            if (piece_weight(st, ks, np, Mc, a.c) > 0.f) break;
+        wk = piece_weight(st, ks, np, Mc, a.c);
+        before = target;
+    }
+    float f = wk > 0.f ? (target - before) / wk : 0.f;            // fraction of the piece to pass
+    f = fminf(fmaxf(f, 0.f), __uint_as_float(0x3F7FFFFFu));
+    // the piece, lane L holding its elements [L E, (L+1) E) in index order
+    constexpr int E = static_cast<int>(kPieceBytes / sizeof(T)) / 32;
+    const int64_t e0 = static_cast<int64_t>(ks) * a.P;
+    const int64_t n = (V - e0 < a.P) ? V - e0 : a.P;
+    const T* piece = logits + r * V + e0;
+    const float Mk = __ldcg(st + ks).x, Mkc = Mk * a.c;
+    float x[E];
+    if constexpr (VEC) {
+        constexpr int VW = 16 / static_cast<int>(sizeof(T));
+        const uint4* pv = reinterpret_cast<const uint4*>(piece) + lane * (E / VW);
+#pragma unroll
+        for (int q = 0; q < E / VW; ++q) {
+            const int64_t ei = static_cast<int64_t>(lane) * E + q * VW;
+            uint4 raw = make_uint4(0u, 0u, 0u, 0u);
+            if (ei < n) raw = __ldcg(pv + q);
+            float e[8];
+            unpack(raw, e, T());
+#pragma unroll
+            for (int j = 0; j < VW; ++j) x[q * VW + j] = ei + j < n ? e[j] : -INFINITY;
+        }
+    } else {
+#pragma unroll
+        for (int q = 0; q < E; ++q) {
+            const int64_t ei = static_cast<int64_t>(lane) * E + q;
+            x[q] = ei < n ? to_f32(piece[ei]) : -INFINITY;
+        }
+    }
+    float ls = 0.f;
+#pragma unroll
+    for (int j = 0; j < E; ++j) ls += x[j] > -INFINITY ? ex2_approx(fmaf(x[j], a.c, -Mkc)) : 0.f;
+    const float incl = warp_incl_scan(ls, lane);
+    const float tot = __shfl_sync(0xFFFFFFFFu, incl, 31);
+    const float tgt = f * tot;
+    const unsigned hit = __ballot_sync(0xFFFFFFFFu, incl > tgt && ls > 0.f);
+    const unsigned has = __ballot_sync(0xFFFFFFFFu, ls > 0.f);
+    // the lane where the running sum passes the target; if rounding hides it, the
+    // last lane holding weight (its last element with weight is then drawn)
+    const int L0 = hit ? __ffs(hit) - 1 : (has ? 31 - __clz(has) : 0);
+    int y = -1;
+    if (lane == L0) {
+        float acc = incl - ls;
+        int last = -1;
+#pragma unroll
+        for (int j = 0; j < E; ++j) {
+            const float wv = x[j] > -INFINITY ? ex2_approx(fmaf(x[j], a.c, -Mkc)) : 0.f;
+            if (wv > 0.f) last = j;
+            acc += wv;
+            if (y < 0 && acc > tgt) y = j;
+        }
+        if (y < 0) y = last;                                      // rounding inside the lane
+        if (y < 0) y = 0;
+        y = static_cast<int>(static_cast<int64_t>(L0) * E + y + e0);
+    }
+    return __shfl_sync(0xFFFFFFFFu, y, L0);
+}
+
+// 2. draws and acceptance: one CTA per sequence, warp w draws rows w, w + 8, ...
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads) sample_finish_kernel(const T* __restrict__ logits, SampleArgs a) {
+    extern __shared__ int32_t draws[];                           // [K+1]
+    pdl_enter();
+    const int64_t b = blockIdx.x;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int K1 = a.v.K + 1;
+    for (int i = warp; i < K1; i += kWarps) {
+        const int y = sample_row<T, VEC>(logits, a, b * K1 + i, lane);
+        if (lane == 0) draws[i] = y;
+    }
+    __syncthreads();
+    if (warp == 0) finish_sequence(a.v, b, lane, SharedTokens{draws});
+}
+
+int sample_pieces(int V, size_t es) {
+    const int64_t P = kPieceBytes / static_cast<int64_t>(es);
+    return static_cast<int>((V + P - 1) / P);
+}
+
+template <typename T, bool VEC>
+pldp_status launch_sample_t(const void* logits, SampleArgs a, cudaStream_t s) {
+    const int64_t rows = static_cast<int64_t>(a.v.B) * (a.v.K + 1);
+    const int64_t units = rows * a.npieces;
+    const void* fn = reinterpret_cast<const void*>(&sample_stats_kernel<T, VEC>);
+    int64_t blocks = static_cast<int64_t>(resident_blocks(fn, kThreads, 0)) * kPassWaves;
+    const int64_t need = (units + kWarps - 1) / kWarps;
+    if (blocks > need) blocks = need;
+    if (blocks < 1) blocks = 1;
+    cudaError_t e = launch_pdl(sample_stats_kernel<T, VEC>, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0,
+                               s, 0, static_cast<const T*>(logits), static_cast<int64_t>(a.v.V), rows, a.npieces,
+                               a.P, a.c, blocks * kWarps, const_cast<float2*>(a.stats));
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "verify_sample: launch failed: %s", cudaGetErrorString(e));
+    const size_t smem = static_cast<size_t>(a.v.K + 1) * sizeof(int32_t);
+    if (smem > 48 * 1024) {
+        e = cudaFuncSetAttribute(sample_finish_kernel<T, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 static_cast<int>(smem));
+        if (e != cudaSuccess)
+            return fail(PLDP_ERR_CUDA, "verify_sample: shared memory attribute: %s", cudaGetErrorString(e));
+    }
+    e = launch_pdl(sample_finish_kernel<T, VEC>, dim3(static_cast<unsigned>(a.v.B)), dim3(kThreads), smem, s, 0,
+                   static_cast<const T*>(logits), a);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "verify_sample: launch failed: %s", cudaGetErrorString(e));
+    return PLDP_OK;
+}
+
+}  // namespace
+}  // namespace pldp
+
+extern "C" PLDP_API size_t pldp_verify_sample_workspace_size(int B, int K, int V, pldp_dtype dtype) {
+    if (B < 0 || K < 1 || V < 1 || (dtype != PLDP_F32 && dtype != PLDP_BF16)) return 0;
+    const size_t es = dtype == PLDP_F32 ? 4 : 2;
+    const size_t bytes = static_cast<size_t>(B) * (K + 1) * sample_pieces(V, es) * sizeof(float2);
+    return (bytes + 255) / 256 * 256;
+}
+
+extern "C" PLDP_API pldp_status pldp_verify_sample(
+    const void* logits, pldp_dtype dtype, int B, int K, int V, float temperature, const float* uniforms,
+    const int32_t* draft, const int32_t* draft_len, int32_t* sampled, int32_t* accept_len, int32_t* next_token,
+    int32_t* ids, int64_t ids_stride, int32_t* seq_len, int64_t T_cap, int32_t* kv_keep_len, uint32_t* status,
+    void* workspace, size_t workspace_bytes, void* stream) {
+    if (B < 0) return fail(PLDP_ERR_INVALID_ARG, "verify_sample: B < 0");
+    if (K < 1) return fail(PLDP_ERR_INVALID_ARG, "verify_sample: K < 1");
+    if (V < 1) return fail(PLDP_ERR_INVALID_ARG, "verify_sample: V < 1");
+    if (dtype != PLDP_F32 && dtype != PLDP_BF16)
+        return fail(PLDP_ERR_UNSUPPORTED, "verify_sample: unsupported dtype %d", (int)dtype);
+    if (!(temperature > 0.f) || isinf(temperature))
+        return fail(PLDP_ERR_INVALID_ARG, "verify_sample: temperature must be positive and finite");
+    if ((ids || kv_keep_len) && !seq_len)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_sample: ids/kv_keep_len need seq_len");
+    if (seq_len && (T_cap < 0 || T_cap > INT32_MAX)) return fail(PLDP_ERR_INVALID_ARG, "verify_sample: bad T_cap");
+    if (ids && ids_stride < T_cap) return fail(PLDP_ERR_INVALID_ARG, "verify_sample: ids_stride < T_cap");
+    if (static_cast<int64_t>(K) + 1 > 12288) return fail(PLDP_ERR_UNSUPPORTED, "verify_sample: K > 12287");
+    if (B == 0) return PLDP_OK;
+    if (!logits || !uniforms || !draft || !draft_len || !accept_len || !next_token)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_sample: null pointer");
+    const size_t need = pldp_verify_sample_workspace_size(B, K, V, dtype);
+    if (!workspace || workspace_bytes < need)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_sample: workspace needs %zu bytes", need);
+    if (!aligned16(workspace)) return fail(PLDP_ERR_INVALID_ARG, "verify_sample: workspace not 16-byte aligned");
+
+    const size_t es = dtype == PLDP_F32 ? 4 : 2;
+    SampleArgs a = {};
+    a.v = verify_args(B, K, V, draft, draft_len, sampled, accept_len, next_token, ids, ids_stride, seq_len, T_cap,
+                      kv_keep_len, status);
+    a.uniforms = uniforms;
+    a.stats = static_cast<const float2*>(workspace);
+    a.c = 1.4426950408889634f / temperature;                      // log2(e) / T
+    a.npieces = sample_pieces(V, es);
+    a.P = static_cast<int>(kPieceBytes / static_cast<int64_t>(es));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const bool vec = aligned16(logits) && (static_cast<size_t>(V) * es) % 16 == 0;
+    if (dtype == PLDP_BF16)
+        return vec ? launch_sample_t<__nv_bfloat16, true>(logits, a, s) : launch_sample_t<__nv_bfloat16, false>(logits, a, s);
+    return vec ? launch_sample_t<float, true>(logits, a, s) : launch_sample_t<float, false>(logits, a, s);
 }
 
 // ---------------------------------------------------------------------------

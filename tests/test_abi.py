@@ -88,6 +88,21 @@ def test_host_argument_checks(so):
     bad[16] = ctypes.c_void_p(256); bad[17] = 8
     assert lib.pldp_verify_greedy(*bad) == 1
     assert "workspace" in pk.pldp_last_error()
+    # verify_sample: temperature not positive/finite, K < 1, workspace too small
+    sm = [null, 1, 2, 4, 100, 1.0, null, null, null, null, null, null, null, 0, null, 0, null, null, null, 0,
+          null]
+    for t in (0.0, -1.0, float("inf"), float("nan")):
+        bad = list(sm); bad[5] = t
+        assert lib.pldp_verify_sample(*bad) == 1 and "temperature" in pk.pldp_last_error()
+    bad = list(sm); bad[3] = 0
+    assert lib.pldp_verify_sample(*bad) == 1
+    bad = list(sm)
+    for k in (0, 6, 7, 8, 10, 11):
+        bad[k] = ctypes.c_void_p(256)
+    bad[18] = ctypes.c_void_p(256); bad[19] = 8
+    assert lib.pldp_verify_sample(*bad) == 1 and "workspace" in pk.pldp_last_error()
+    assert lib.pldp_verify_sample_workspace_size(2, 4, 100, 7) == 0
+    assert lib.pldp_verify_sample_workspace_size(128, 12, 128256, 1) == 128 * 13 * 126 * 8
 
 
 def test_python_binding_refuses_cpu_tensors():
