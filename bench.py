@@ -437,14 +437,15 @@ def time_sampling_verify(pk, loop, w, flush_l2, peak, calls=64, warm=4, temperat
                      device=dev)
     acc, nxt = torch.zeros(B, dtype=torch.int32, device=dev), torch.zeros(B, dtype=torch.int32, device=dev)
     sampled = torch.zeros((B, K1), dtype=torch.int32, device=dev)
+    draft = path_draft(loop, w)
+    dlen = torch.full((B,), w.K, dtype=torch.int32, device=dev)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(calls)]
     s = torch.cuda.current_stream()
     for i in range(warm + calls):
         flush_l2(i)
         if i >= warm:
             ev[i - warm][0].record(s)
-        pk.pldp_verify_sample(loop.logits, u, path_draft(loop, w), torch.full((B,), w.K, dtype=torch.int32,
-                              device=dev), acc, nxt, ws, temperature=temperature, sampled=sampled)
+        pk.pldp_verify_sample(loop.logits, u, draft, dlen, acc, nxt, ws, temperature=temperature, sampled=sampled)
         if i >= warm:
             ev[i - warm][1].record(s)
     torch.cuda.synchronize()

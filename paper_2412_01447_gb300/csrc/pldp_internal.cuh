@@ -134,6 +134,13 @@ __device__ __forceinline__ void pdl_enter() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// The wait alone: the next kernel is then scheduled only as this grid's CTAs
+// finish, for a kernel whose dependent is heavy enough (registers, threads) to
+// crowd out this grid's last CTAs if it were resident early.
+__device__ __forceinline__ void pdl_wait_only() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
 // Launches `kernel` with programmatic stream serialisation (and an optional
 // cluster shape, cluster_x > 0).
 template <typename... KArgs, typename... Args>

@@ -552,7 +552,7 @@ template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads, VEC ? kPassBlocksPerSm : 4)
 sample_stats_kernel(const T* __restrict__ logits, int64_t V, int64_t rows, int npieces, int P, float c,
                     int64_t W, float2* __restrict__ stats) {
-    pdl_enter();
+    pdl_wait_only();                        // the finish (a full SM per CTA) starts as this grid ends
     const int lane = threadIdx.x & 31;
     const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
     const int64_t units = rows * npieces;
@@ -632,56 +632,109 @@ __device__ __forceinline__ float warp_incl_scan(float v, int lane) {
     return v;
 }
 
+// Piece k* of row r, where the running total of the piece weights first passes
+// u Z: the total is summed, then the crossing found, by the same warp scans in the
+// same order, so the crossing exists.  The row's stats are held in registers
+// (up to 32 * kStatRegs pieces) or, beyond that, reread per scan.
+constexpr int kStatRegs = 4;
+
+struct PiecePick {
+    int k;          // the piece
+    float before;   // running total before it
+    float w;        // its weight
+    float target;   // u Z
+    float Mk;       // its max
+};
+
+__device__ __forceinline__ PiecePick pick_piece(const float2* __restrict__ st, int np, float c, float u, int lane) {
+    PiecePick pk = {-1, 0.f, 0.f, 0.f, 0.f};
+    if (np <= 32 * kStatRegs) {
+        float2 sv[kStatRegs];
+        float m = -INFINITY;
+#pragma unroll
+        for (int q = 0; q < kStatRegs; ++q) {
+            const int k = lane + 32 * q;
+            sv[q] = k < np ? __ldcg(st + k) : make_float2(-INFINITY, 0.f);
+            m = fmaxf(m, sv[q].x);
+        }
+        const float Mc = warp_max_f(m) * c;
+        float wv[kStatRegs], incl[kStatRegs], total = 0.f;
+#pragma unroll
+        for (int q = 0; q < kStatRegs; ++q) {
+            wv[q] = sv[q].x > -INFINITY ? sv[q].y * ex2_approx(fmaf(sv[q].x, c, -Mc)) : 0.f;
+            incl[q] = warp_incl_scan(wv[q], lane);
+            total += __shfl_sync(0xFFFFFFFFu, incl[q], 31);
+        }
+        pk.target = u * total;
+        float run = 0.f;
+#pragma unroll
+        for (int q = 0; q < kStatRegs; ++q) {
+            const unsigned hit = __ballot_sync(0xFFFFFFFFu, run + incl[q] > pk.target && lane + 32 * q < np);
+            if (pk.k < 0 && hit) {
+                const int f = __ffs(hit) - 1;
+                pk.k = 32 * q + f;
+                pk.before = run + __shfl_sync(0xFFFFFFFFu, incl[q] - wv[q], f);
+                pk.w = __shfl_sync(0xFFFFFFFFu, wv[q], f);
+                pk.Mk = __shfl_sync(0xFFFFFFFFu, sv[q].x, f);
+            }
+            run += __shfl_sync(0xFFFFFFFFu, incl[q], 31);
+        }
+    } else {
+        float m = -INFINITY;
+        for (int k = lane; k < np; k += 32) m = fmaxf(m, __ldcg(st + k).x);
+        const float Mc = warp_max_f(m) * c;
+        float total = 0.f;
+        for (int k0 = 0; k0 < np; k0 += 32) {
+            const float incl = warp_incl_scan(piece_weight(st, k0 + lane, np, Mc, c), lane);
+            total += __shfl_sync(0xFFFFFFFFu, incl, 31);
+        }
+        pk.target = u * total;
+        float run = 0.f;
+        for (int k0 = 0; k0 < np && pk.k < 0; k0 += 32) {
+            const float wv = piece_weight(st, k0 + lane, np, Mc, c);
+            const float incl = warp_incl_scan(wv, lane);
+            const unsigned hit = __ballot_sync(0xFFFFFFFFu, run + incl > pk.target && k0 + lane < np);
+            if (hit) {
+                const int f = __ffs(hit) - 1;
+                pk.k = k0 + f;
+                pk.before = run + __shfl_sync(0xFFFFFFFFu, incl - wv, f);
+                pk.w = __shfl_sync(0xFFFFFFFFu, wv, f);
+                pk.Mk = __ldcg(st + pk.k).x;
+            }
+            run += __shfl_sync(0xFFFFFFFFu, incl, 31);
+        }
+    }
+    return pk;
+}
+
 // The draw of row r (one warp).
 template <typename T, bool VEC>
 __device__ int sample_row(const T* __restrict__ logits, const SampleArgs& a, int64_t r, int lane) {
     const int64_t V = a.v.V;
     const int np = a.npieces;
     const float2* st = a.stats + r * np;
-    float m = -INFINITY;
-    for (int k = lane; k < np; k += 32) m = fmaxf(m, __ldcg(st + k).x);
-    const float M = warp_max_f(m);
-    const float Mc = M * a.c;
-    // the total, then the first piece whose running total passes u Z (same sums, same order)
-    float base = 0.f;
-    for (int k0 = 0; k0 < np; k0 += 32) {
-        const float incl = warp_incl_scan(piece_weight(st, k0 + lane, np, Mc, a.c), lane);
-        base += __shfl_sync(0xFFFFFFFFu, incl, 31);
-    }
     float u = a.uniforms[r];
     if (!(u >= 0.f)) u = 0.f;
     if (u >= 1.f) u = __uint_as_float(0x3F7FFFFFu);               // largest float below 1
-    const float target = u * base;
-    int ks = -1;
-    float before = 0.f, wk = 0.f;
-    float run = 0.f;
-    for (int k0 = 0; k0 < np && ks < 0; k0 += 32) {
-        const float wv = piece_weight(st, k0 + lane, np, Mc, a.c);
-        const float incl = warp_incl_scan(wv, lane);
-        const unsigned hit = __ballot_sync(0xFFFFFFFFu, run + incl > target && k0 + lane < np);
-        if (hit) {
-            const int f = __ffs(hit) - 1;
-            ks = k0 + f;
-            before = run + __shfl_sync(0xFFFFFFFFu, incl - wv, f);
-            wk = __shfl_sync(0xFFFFFFFFu, wv, f);
-        }
-        run += __shfl_sync(0xFFFFFFFFu, incl, 31);
+    PiecePick pk = pick_piece(st, np, a.c, u, lane);
+    if (pk.k < 0) {                                               // rounding: the last piece with weight
+        int k = np - 1;
+        for (; k > 0; --k)
+            if (__ldcg(st + k).y > 0.f) break;
+        pk.k = k;
+        pk.before = pk.target;
+        pk.w = 1.f;
+        pk.Mk = __ldcg(st + k).x;
     }
-    if (ks < 0) {                                                 // rounding: the last piece with weight
-        ks = np - 1;
-        for (; ks > 0; --ks)
-            if (piece_weight(st, ks, np, Mc, a.c) > 0.f) break;
-        wk = piece_weight(st, ks, np, Mc, a.c);
-        before = target;
-    }
-    float f = wk > 0.f ? (target - before) / wk : 0.f;            // fraction of the piece to pass
+    float f = pk.w > 0.f ? (pk.target - pk.before) / pk.w : 0.f;  // fraction of the piece to pass
     f = fminf(fmaxf(f, 0.f), __uint_as_float(0x3F7FFFFFu));
+    const int ks = pk.k;
     // the piece, lane L holding its elements [L E, (L+1) E) in index order
     constexpr int E = static_cast<int>(kPieceBytes / sizeof(T)) / 32;
     const int64_t e0 = static_cast<int64_t>(ks) * a.P;
     const int64_t n = (V - e0 < a.P) ? V - e0 : a.P;
     const T* piece = logits + r * V + e0;
-    const float Mk = __ldcg(st + ks).x, Mkc = Mk * a.c;
+    const float Mkc = pk.Mk * a.c;
     float x[E];
     if constexpr (VEC) {
         constexpr int VW = 16 / static_cast<int>(sizeof(T));
@@ -732,15 +785,18 @@ __device__ int sample_row(const T* __restrict__ logits, const SampleArgs& a, int
     return __shfl_sync(0xFFFFFFFFu, y, L0);
 }
 
-// 2. draws and acceptance: one CTA per sequence, warp w draws rows w, w + 8, ...
+// 2. draws and acceptance: one CTA per sequence, warp w draws rows w, w + 16, ...
+constexpr int kFinishWarps = 16;
+
 template <typename T, bool VEC>
-__global__ void __launch_bounds__(kThreads) sample_finish_kernel(const T* __restrict__ logits, SampleArgs a) {
+__global__ void __launch_bounds__(32 * kFinishWarps, 1) sample_finish_kernel(const T* __restrict__ logits,
+                                                                            SampleArgs a) {
     extern __shared__ int32_t draws[];                           // [K+1]
     pdl_enter();
     const int64_t b = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int K1 = a.v.K + 1;
-    for (int i = warp; i < K1; i += kWarps) {
+    for (int i = warp; i < K1; i += kFinishWarps) {
         const int y = sample_row<T, VEC>(logits, a, b * K1 + i, lane);
         if (lane == 0) draws[i] = y;
     }
@@ -773,7 +829,7 @@ pldp_status launch_sample_t(const void* logits, SampleArgs a, cudaStream_t s) {
         if (e != cudaSuccess)
             return fail(PLDP_ERR_CUDA, "verify_sample: shared memory attribute: %s", cudaGetErrorString(e));
     }
-    e = launch_pdl(sample_finish_kernel<T, VEC>, dim3(static_cast<unsigned>(a.v.B)), dim3(kThreads), smem, s, 0,
+    e = launch_pdl(sample_finish_kernel<T, VEC>, dim3(static_cast<unsigned>(a.v.B)), dim3(32 * kFinishWarps), smem, s, 0,
                    static_cast<const T*>(logits), a);
     if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "verify_sample: launch failed: %s", cudaGetErrorString(e));
     return PLDP_OK;
