@@ -72,10 +72,12 @@ def _configure(lib):
                                          P, P, P, P]
     lib.pldpo_extract_draft.argtypes = [P, i64, P, i64, P, i32, i32, P, P]
     lib.pldpo_verify_greedy.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64, P, i64, P, P]
+    lib.pldpo_rank_hidden_avg.argtypes = [P, i32, i64, i64, i32, P, i32, i64, P, P, i32, ctypes.c_double, P, P,
+                                          P, P]
     lib.pldpo_verify_sample.argtypes = [P, i32, i32, i32, i32, ctypes.c_double, P, P, P, P, P, P, P, i64,
                                         P, i64, P, P]
     for f in ("pldpo_find_candidates", "pldpo_rank_hidden", "pldpo_rank_attention",
-              "pldpo_extract_draft", "pldpo_verify_greedy", "pldpo_verify_sample"):
+              "pldpo_extract_draft", "pldpo_verify_greedy", "pldpo_verify_sample", "pldpo_rank_hidden_avg"):
         getattr(lib, f).restype = ctypes.c_int
 
 
@@ -156,6 +158,23 @@ def rank_hidden(H, seq_len, cand_pos, cand_count, threshold=-np.inf, status=None
     _check(_load().pldpo_rank_hidden(_ptr(H), dt, d, T_cap * d, _ptr(seq_len), B, T_cap, _ptr(cand_pos),
                                      _ptr(cand_count), C_cap, float(threshold), _ptr(scores),
                                      _ptr(best), _ptr(bs), _ptr(status)), "rank_hidden")
+    return scores, best, bs
+
+
+def rank_hidden_avg(H, seq_len, cand_pos, cand_count, m, threshold=-np.inf, status=None):
+    """App. B.2: Eq. 3 on window means of the m rows ending at each position.
+    Same shapes and returns as rank_hidden."""
+    H, dt = _elem(H)
+    B, T_cap, d = H.shape
+    cand_pos = _i32(cand_pos)
+    C_cap = cand_pos.shape[1]
+    seq_len, cand_count = _i32(seq_len), _i32(cand_count)
+    scores = np.full((B, C_cap), np.nan)
+    best = np.zeros(B, np.int32)
+    bs = np.zeros(B)
+    _check(_load().pldpo_rank_hidden_avg(_ptr(H), dt, d, T_cap * d, int(m), _ptr(seq_len), B, T_cap,
+                                         _ptr(cand_pos), _ptr(cand_count), C_cap, float(threshold),
+                                         _ptr(scores), _ptr(best), _ptr(bs), _ptr(status)), "rank_hidden_avg")
     return scores, best, bs
 
 

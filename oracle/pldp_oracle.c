@@ -176,6 +176,75 @@ int pldpo_rank_hidden(const void* H, int dtype, int64_t d, int64_t seq_stride,
 }
 
 /* --------------------------------------------------------------------------
+ * Ranking by averaged hidden states -- the variant of Eq. 3 studied in App. B.2:
+ * every hidden state is replaced by the mean of the m rows ending at it,
+ *     Hbar_p = mean(H_{max(0, p-m+1)}, ..., H_p),
+ * and candidate j scores cos(Hbar_{j-1}, Hbar_{t-1}).  m = 1 is Eq. 3.
+ * READING: the printed formula averages H_1..H_m, the same rows for every
+ * position; it is read as the window of the m positions ending at the position
+ * averaged, cut at position 0 (fewer rows near the start).
+ * Eligibility, zero norms, ties, the threshold and scores as pldpo_rank_hidden.
+ * ------------------------------------------------------------------------ */
+static void orc_window_mean(const void* H, int dtype, int64_t base, int64_t p, int m, int64_t d,
+                            double* out) {
+    int64_t lo = p - m + 1;
+    if (lo < 0) lo = 0;
+    for (int64_t k = 0; k < d; ++k) out[k] = 0.0;
+    for (int64_t r = lo; r <= p; ++r)
+        for (int64_t k = 0; k < d; ++k) out[k] += orc_load(H, dtype, base + r * d + k);
+    for (int64_t k = 0; k < d; ++k) out[k] /= (double)(p - lo + 1);
+}
+
+int pldpo_rank_hidden_avg(const void* H, int dtype, int64_t d, int64_t seq_stride, int m,
+                          const int32_t* seq_len, int B, int64_t T_cap,
+                          const int32_t* cand_pos, const int32_t* cand_count, int C_cap,
+                          double threshold, double* scores,
+                          int32_t* best_pos, double* best_score, uint32_t* status) {
+    if (B < 0 || d < 1 || m < 1 || C_cap < 0 || (dtype != ORC_F32 && dtype != ORC_BF16)) return 1;
+    double* qv = (double*)malloc(sizeof(double) * (size_t)d);
+    double* cv = (double*)malloc(sizeof(double) * (size_t)d);
+    if (!qv || !cv) { free(qv); free(cv); return 2; }
+    for (int b = 0; b < B; ++b) {
+        if (seq_len[b] < 0 || seq_len[b] > T_cap) {         /* sequence skipped */
+            if (status) status[b] |= ORC_ST_SEQ_LEN;
+            best_pos[b] = -1;
+            if (best_score) best_score[b] = -INFINITY;
+            continue;
+        }
+        int64_t t = (int64_t)seq_len[b] - 1;
+        int64_t n = cand_count[b] < 0 ? 0 : cand_count[b];
+        if (n > C_cap) n = C_cap;
+        int64_t base = (int64_t)b * seq_stride;
+        if (t >= 1) orc_window_mean(H, dtype, base, t - 1, m, d, qv);     /* Hbar_{t-1} */
+        int32_t bj = -1;
+        double bs = -INFINITY;
+        for (int64_t i = 0; i < n; ++i) {
+            int64_t j = cand_pos[(int64_t)b * C_cap + i];
+            double s = -INFINITY;
+            if (j >= 1 && j < t) {
+                orc_window_mean(H, dtype, base, j - 1, m, d, cv);         /* Hbar_{j-1} */
+                double dot = 0.0, na = 0.0, nq = 0.0;
+                for (int64_t k = 0; k < d; ++k) {
+                    dot += cv[k] * qv[k];
+                    na += cv[k] * cv[k];
+                    nq += qv[k] * qv[k];
+                }
+                s = (na == 0.0 || nq == 0.0) ? 0.0 : dot / sqrt(na * nq);
+            }
+            if (scores) scores[(int64_t)b * C_cap + i] = s;
+            if (j >= 1 && j < t && threshold < s) {           /* eligible: the smallest j wins a tie */
+                if (bj < 0 || s > bs || (s == bs && j < bj)) { bs = s; bj = (int32_t)j; }
+            }
+        }
+        best_pos[b] = bj;
+        if (best_score) best_score[b] = bj >= 0 ? bs : -INFINITY;
+    }
+    free(qv);
+    free(cv);
+    return 0;
+}
+
+/* --------------------------------------------------------------------------
  * Ranking by attentions.  Eq. 2 (Sec. 4.2.1):
  *     j* = argmax_{j in P} max_{l in L*, g in G*} A^{(l,g)}_{t-1}
  * A holds, per sequence, the attention-probability rows of query t-1 for the

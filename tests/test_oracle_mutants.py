@@ -62,6 +62,13 @@ MUTANTS = [
     ("accept ignores the first draft token",
      "for (int64_t i = 0; i < d; ++i) {\n        if (draft[(int64_t)b * K + i] != tok[i]) { n = i; break; }",
      "for (int64_t i = 1; i < d; ++i) {\n        if (draft[(int64_t)b * K + i] != tok[i]) { n = i; break; }"),
+    ("averaged-ranking tie goes to the larger position",
+     "/* eligible: the smallest j wins a tie */\n                if (bj < 0 || s > bs || (s == bs && j < bj))",
+     "/* eligible: the smallest j wins a tie */\n                if (bj < 0 || s > bs || (s == bs && j > bj))"),
+    ("averaging window one row too long",
+     "int64_t lo = p - m + 1;\n    if (lo < 0) lo = 0;", "int64_t lo = p - m;\n    if (lo < 0) lo = 0;"),
+    ("averaging window misses the row averaged",
+     "for (int64_t r = lo; r <= p; ++r)", "for (int64_t r = lo; r < p; ++r)"),
     ("sampling draws where the cumulative sum only reaches u",
      "if (c > target) { y = (int32_t)v; break; }", "if (c >= target) { y = (int32_t)v; break; }"),
     ("sampling multiplies by the temperature",

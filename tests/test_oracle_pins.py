@@ -359,3 +359,55 @@ def test_sample_bookkeeping_matches_greedy_rules(orc):
             assert ids[b, lens0[b]:lens[b]].tolist() == list(draft[b, :n]) + [y[b, n]]
         else:
             assert out["status"][b] == orc.ST_CAPACITY and np.array_equal(ids[b], ids0[b])
+
+
+# ----------------------------------------------------------------------------
+# averaged hidden states (App. B.2)
+# ----------------------------------------------------------------------------
+@pytest.mark.parametrize("m", [1, 2, 3, 5])
+def test_rank_hidden_avg_matches_numpy_window_means(orc, m):
+    rng = np.random.default_rng(300 + m)
+    B, T, d, C = 4, 24, 16, 8
+    H = rng.normal(size=(B, T, d)).astype(np.float32)
+    lens = np.array([T, 13, 3, 2], np.int32)
+    cand = np.zeros((B, C), np.int32)
+    cnt = np.zeros(B, np.int32)
+    for b in range(B):
+        js = np.unique(rng.integers(0, max(lens[b] - 1, 1), size=6))
+        js = js[js < max(lens[b] - 1, 1)]
+        cnt[b] = js.size
+        cand[b, :js.size] = js
+    s, best, bs = orc.rank_hidden_avg(H, lens, cand, cnt, m)
+    for b in range(B):
+        t = lens[b] - 1
+        def mean(p):
+            return H[b, max(0, p - m + 1):p + 1].astype(np.float64).mean(axis=0)
+        want = []
+        for i in range(cnt[b]):
+            j = cand[b, i]
+            want.append(1.0 - scipy_cosine(mean(j - 1), mean(t - 1)) if 1 <= j < t else -np.inf)
+        assert np.allclose(s[b, :cnt[b]], want, atol=1e-12, rtol=0)
+        ok = [(w, -cand[b, i]) for i, w in enumerate(want) if np.isfinite(w)]
+        assert best[b] == (-max(ok)[1] if ok else -1)
+
+
+def test_rank_hidden_avg_m1_is_eq3_exactly(orc):
+    rng = np.random.default_rng(17)
+    B, T, d, C = 3, 40, 32, 10
+    H = rng.normal(size=(B, T, d)).astype(np.float32)
+    lens = np.array([40, 22, 5], np.int32)
+    cand = np.tile(np.arange(0, 2 * C, 2, dtype=np.int32), (B, 1))
+    cnt = np.array([10, 10, 3], np.int32)
+    a = orc.rank_hidden_avg(H, lens, cand, cnt, 1, threshold=0.05)
+    e = orc.rank_hidden(H, lens, cand, cnt, threshold=0.05)
+    assert np.array_equal(a[0], e[0], equal_nan=True) and np.array_equal(a[1], e[1])
+
+
+def test_rank_hidden_avg_tie_goes_to_smaller_position(orc):
+    # candidates 9 and 17 have identical windows (rows 6..8 copied to 14..16): equal scores
+    rng = np.random.default_rng(23)
+    H = rng.normal(size=(1, 30, 8)).astype(np.float32)
+    H[0, 14:17] = H[0, 6:9]
+    cand = np.array([[17, 9, 25]], np.int32)
+    s, best, _ = orc.rank_hidden_avg(H, np.array([30], np.int32), cand, np.array([2], np.int32), 3)
+    assert s[0, 0] == s[0, 1] and best[0] == 9
