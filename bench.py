@@ -418,6 +418,7 @@ def run_ours(args, ws_, rank, local):
     }
     if not args.no_sample:
         out["sampling_verify"] = time_sampling_verify(pk, loop, w, flush_l2, peak)
+        out["rank_hidden_avg"] = time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak)
     if not args.no_e2e:
         out["e2e"] = run_e2e(pk, loop, path, K_steps, W_steps, ws_)
     if rank == 0 and ws_ == 1 and not args.no_cpu_baseline:
@@ -456,6 +457,40 @@ def time_sampling_verify(pk, loop, w, flush_l2, peak, calls=64, warm=4, temperat
             "frac": round(by / (us * 1e-6) / 1e9 / peak, 4), "algorithmic_bytes": by,
             "launches_per_call": 2,
             "timing": "CUDA events around each pldp_verify_sample call, L2 flushed before each"}
+
+
+def time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak, m=4, calls=64, warm=4):
+    """Ranking by averaged hidden states (App. B.2, window m) against plain Eq. 3 on the
+    loop's own candidate lists at the same shape, each call timed with CUDA events, L2
+    flushed before each.  Algorithmic bytes: per sequence the window rows of the query
+    and of every listed candidate, (|P| + 1) * m * d * 2."""
+    dev = loop.device
+    B = w.B
+    best = torch.zeros(B, dtype=torch.int32, device=dev)
+    s = torch.cuda.current_stream()
+    res = {}
+    n = float(path.cnt.clamp(min=0, max=w.C_cap).sum().item())
+    for name, mm in (("eq3", 1), (f"avg_m{m}", m)):
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(calls)]
+        for i in range(warm + calls):
+            flush_l2(i)
+            if i >= warm:
+                ev[i - warm][0].record(s)
+            if mm == 1:
+                pk.pldp_rank_hidden(loop.H, loop.seq_len, path.cand, path.cnt, best)
+            else:
+                pk.pldp_rank_hidden_avg(loop.H, loop.seq_len, path.cand, path.cnt, best, mm)
+            if i >= warm:
+                ev[i - warm][1].record(s)
+        torch.cuda.synchronize()
+        us = float(np.mean([a.elapsed_time(b) for a, b in ev])) * 1e3
+        by = (n + B) * mm * w.d * 2.0
+        res[name] = {"us_per_call": round(us, 2), "algorithmic_bytes": by,
+                     "achieved_gbs": round(by / (us * 1e-6) / 1e9, 1)}
+    res.update({"m": m, "candidates_listed": int(n), "peak_gbs": peak,
+                "bound": "latency (a few MB gathered per call)",
+                "timing": "CUDA events around each call, L2 flushed before each"})
+    return res
 
 
 def path_draft(loop, w):

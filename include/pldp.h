@@ -138,6 +138,24 @@ PLDP_API pldp_status pldp_rank_hidden(const void* H, pldp_dtype dtype, int64_t d
                                       uint32_t* status, void* stream);
 
 /*
+ * Ranking by averaged hidden states -- the variant of Eq. 3 studied in App. B.2
+ * (the paper reports it does not help; it is here for completeness):
+ *   Hbar_p  = mean(H_{max(0, p-m+1)}, ..., H_p)     (the m rows ending at p)
+ *   score_j = cos(Hbar_{j-1}, Hbar_{t-1}),  j* = argmax_{j in P} score_j.
+ * The printed formula averages H_1..H_m for every position; it is read as the
+ * window of the m positions ending at the one averaged, cut at position 0.
+ * m = 1 is Eq. 3.  Arguments, outputs and conventions as pldp_rank_hidden, plus
+ *  m   window length, >= 1.
+ * Limit: d * 4 <= 196608 (the query's window sum is held in fp32 in shared memory).
+ */
+PLDP_API pldp_status pldp_rank_hidden_avg(const void* H, pldp_dtype dtype, int64_t d,
+                                          int64_t seq_stride, int m, const int32_t* seq_len, int B,
+                                          int64_t T_cap, const int32_t* cand_pos,
+                                          const int32_t* cand_count, int C_cap, float threshold,
+                                          float* scores, int32_t* best_pos, float* best_score,
+                                          uint32_t* status, void* stream);
+
+/*
  * Ranking by attentions -- Eq. 2 (Sec. 4.2.1):
  *   score_j = max over the selected (layer, head) rows of A^{(l,g)}_{t-1}[j],
  *   j* = argmax_{j in P} score_j;  agg = PLDP_AGG_SUM sums the rows instead

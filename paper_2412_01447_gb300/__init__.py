@@ -102,6 +102,9 @@ def _load():
             lib.pldp_find_candidates.argtypes = [P, i64, P, i32, i64, i32, i32, P, i32, P, P, P, P]
             lib.pldp_rank_hidden.argtypes = [P, i32, i64, i64, P, i32, i64, P, P, i32, f32, P, P, P,
                                              P, P]
+            lib.pldp_rank_hidden_avg.argtypes = [P, i32, i64, i64, i32, P, i32, i64, P, P, i32, f32, P, P,
+                                                 P, P, P]
+            lib.pldp_rank_hidden_avg.restype = ctypes.c_int
             lib.pldp_rank_attention.argtypes = [P, i32, i32, i64, i64, P, i32, i32, P, i32, i64, P,
                                                 P, i32, P, P, P, P, P]
             lib.pldp_extract_draft.argtypes = [P, i64, P, i64, P, i32, i32, P, P, P]
@@ -210,6 +213,23 @@ def pldp_rank_hidden(H, seq_len, cand_pos, cand_count, best_pos, scores=None, be
     C_cap = cand_pos.shape[1]
     _check("pldp_rank_hidden", _load().pldp_rank_hidden(
         _dev(H, "H"), _code(H.dtype), d, H.stride(0), _dense(seq_len, "seq_len", torch.int32), B,
+        T_cap, _dense(cand_pos, "cand_pos", torch.int32), _dense(cand_count, "cand_count", torch.int32),
+        C_cap, float(threshold), _dense(scores, "scores", torch.float32, allow_none=True),
+        _dense(best_pos, "best_pos", torch.int32),
+        _dense(best_score, "best_score", torch.float32, allow_none=True),
+        _dense(status, "status", None, allow_none=True), _stream(stream)))
+
+
+def pldp_rank_hidden_avg(H, seq_len, cand_pos, cand_count, best_pos, m, scores=None, best_score=None,
+                         threshold=float("-inf"), status=None, stream=None):
+    """App. B.2: Eq. 3 on the means of the m rows ending at each position.  Same
+    arguments as pldp_rank_hidden plus the window length m >= 1."""
+    if H.dim() != 3 or H.stride(2) != 1 or H.stride(1) != H.shape[2]:
+        raise ValueError("H must be [B, T_cap, d] with contiguous rows")
+    B, T_cap, d = H.shape
+    C_cap = cand_pos.shape[1]
+    _check("pldp_rank_hidden_avg", _load().pldp_rank_hidden_avg(
+        _dev(H, "H"), _code(H.dtype), d, H.stride(0), int(m), _dense(seq_len, "seq_len", torch.int32), B,
         T_cap, _dense(cand_pos, "cand_pos", torch.int32), _dense(cand_count, "cand_count", torch.int32),
         C_cap, float(threshold), _dense(scores, "scores", torch.float32, allow_none=True),
         _dense(best_pos, "best_pos", torch.int32),

@@ -7,6 +7,8 @@
 // query row H_{t-1} in shared memory with one bulk asynchronous copy (when rows
 // are 16-byte aligned), issued before the warps stream their candidate rows, so
 // the two DRAM round trips overlap.
+#include <type_traits>
+
 #include "pldp_rank.cuh"
 
 namespace pldp {
@@ -143,6 +145,153 @@ rank_hidden_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride,
     store_best<CLUSTER>(sh, mine, b, best_pos, best_score, status, PLDP_ST_TIMEOUT);
 }
 
+// ---------------------------------------------------------------------------
+// Averaged hidden states, the variant of Eq. 3 studied in App. B.2: every vector
+// is replaced by the mean of the m rows ending at its position (cut at position
+// 0), and candidate j scores cos(Hbar_{j-1}, Hbar_{t-1}).  Window sums are used
+// in place of means (the cosine ignores the positive factor).  The query's
+// window sum is built once in shared memory in fp32; each candidate's is formed
+// on the fly by the whole CTA -- thread i takes chunks i, i + 256, ... -- and the
+// partial sums meet in warp order.  One candidate at a time per CTA.
+// ---------------------------------------------------------------------------
+constexpr size_t kMaxAvgQueryBytes = 196608;   // d * 4: the fp32 window sum of the query
+
+template <typename T, bool VEC>
+struct Chunk {
+    static constexpr int E = VEC ? 16 / static_cast<int>(sizeof(T)) : 1;
+    using Raw = typename std::conditional<VEC, uint4, T>::type;
+    static __device__ __forceinline__ Raw load(const T* p) {
+        if constexpr (VEC) return ld_stream16(p);
+        else return *p;
+    }
+    // Adds the E elements of x to acc.
+    static __device__ __forceinline__ void add(const Raw& x, float (&acc)[E]) {
+        if constexpr (VEC) {
+            const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+            if constexpr (sizeof(T) == 2) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    acc[2 * k] += __uint_as_float(w[k] << 16);
+                    acc[2 * k + 1] += __uint_as_float(w[k] & 0xFFFF0000u);
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) acc[k] += __uint_as_float(w[k]);
+            }
+        } else {
+            acc[0] += to_f32(x);
+        }
+    }
+    // acc = sum of the chunks at p + r * d for rows r in [lo, hi], four loads in flight.
+    static __device__ __forceinline__ void window(const T* p, int64_t d, int64_t lo, int64_t hi, float (&acc)[E]) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) acc[e] = 0.f;
+        for (int64_t r0 = lo; r0 <= hi; r0 += 4) {
+            Raw x[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (r0 + u <= hi) x[u] = load(p + (r0 + u) * d);
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (r0 + u <= hi) add(x[u], acc);
+        }
+    }
+};
+
+template <typename T, bool VEC, bool CLUSTER>
+__global__ void __launch_bounds__(kThreads)
+rank_hidden_avg_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride, int m,
+                       const int32_t* __restrict__ seq_len, int64_t T_cap,
+                       const int32_t* __restrict__ cand_pos, const int32_t* __restrict__ cand_count,
+                       int C_cap, float threshold, float* __restrict__ scores,
+                       int32_t* __restrict__ best_pos, float* __restrict__ best_score,
+                       uint32_t* __restrict__ status, int S) {
+    using C = Chunk<T, VEC>;
+    constexpr int E = C::E;
+    extern __shared__ __align__(128) unsigned char dyn_smem[];
+    float* qs = reinterpret_cast<float*>(dyn_smem);       // window sum ending at H_{t-1}
+    __shared__ RankShared sh;
+    __shared__ CtaBest mine;
+
+    pdl_enter();
+    const int b = blockIdx.x / S;
+    const int rank = blockIdx.x - b * S;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t L = seq_len[b];
+    int n = cand_count[b];
+    if (L < 0 || L > T_cap) {       // the same for every CTA of the sequence
+        if (rank == 0 && tid == 0) {
+            best_pos[b] = -1;
+            if (best_score) best_score[b] = -INFINITY;
+            if (status) atomicOr(status + b, PLDP_ST_SEQ_LEN);
+        }
+        return;
+    }
+    const int64_t t = L - 1;
+    n = n < 0 ? 0 : (n > C_cap ? C_cap : n);
+    const T* hb = H + static_cast<int64_t>(b) * seq_stride;
+    const int64_t nch = d / E;
+    rank_shared_init(sh);
+    if (n > rank && t >= 2) {
+        const int64_t lo = t - m > 0 ? t - m : 0;                 // rows lo .. t-1
+        for (int64_t c = tid; c < nch; c += kThreads) {
+            float acc[E];
+            C::window(hb + c * E, d, lo, t - 1, acc);
+#pragma unroll
+            for (int e = 0; e < E; ++e) qs[c * E + e] = acc[e];
+        }
+    }
+    __syncthreads();
+    const int32_t* cands = cand_pos + static_cast<int64_t>(b) * C_cap;
+    for (int i = rank; i < n; i += S) {                           // CTA-uniform
+        const int64_t j = __ldg(cands + i);
+        const bool ok = j >= 1 && j < t;
+        float dot = 0.f, na = 0.f, nq = 0.f;
+        if (ok) {
+            const int64_t lo = j - m > 0 ? j - m : 0;             // rows lo .. j-1
+            for (int64_t c = tid; c < nch; c += kThreads) {
+                float a[E];
+                C::window(hb + c * E, d, lo, j - 1, a);
+#pragma unroll
+                for (int e = 0; e < E; ++e) {
+                    const float q = qs[c * E + e];
+                    dot = fmaf(a[e], q, dot);
+                    na = fmaf(a[e], a[e], na);
+                    nq = fmaf(q, q, nq);
+                }
+            }
+        }
+        dot = warp_sum(dot);
+        na = warp_sum(na);
+        nq = warp_sum(nq);
+        if (lane == 0) {
+            sh.part[warp][0] = dot;
+            sh.part[warp][1] = na;
+            sh.part[warp][2] = nq;
+        }
+        __syncthreads();
+        if (tid == 0) {
+            float s = -INFINITY;
+            if (ok) {
+                float D = 0.f, N = 0.f, Q = 0.f;
+                for (int w = 0; w < kRankWarps; ++w) {            // fixed order
+                    D += sh.part[w][0];
+                    N += sh.part[w][1];
+                    Q += sh.part[w][2];
+                }
+                s = finish_cosine(D, N, Q);
+            }
+            if (scores) scores[static_cast<int64_t>(b) * C_cap + i] = s;
+            if (ok && s > threshold) {
+                const unsigned long long key = pack_key(s, static_cast<uint32_t>(j));
+                if (key > sh.slot_key[0]) sh.slot_key[0] = key;
+            }
+        }
+        __syncthreads();
+    }
+    store_best<CLUSTER>(sh, mine, b, best_pos, best_score, status, PLDP_ST_TIMEOUT);
+}
+
 template <bool CLUSTER>
 __global__ void __launch_bounds__(kThreads)
 rank_attention_kernel(const void* __restrict__ A, bool a_bf16, int R, int64_t row_stride,
@@ -246,10 +395,68 @@ cudaError_t launch_attention(int B, int S, size_t smem, void* stream, const void
                        scores, best_pos, best_score, status);
 }
 
+template <typename T, bool VEC>
+cudaError_t launch_hidden_avg(int B, int S, size_t smem, void* stream, const T* h, int64_t d, int64_t seq_stride,
+                              int m, const int32_t* seq_len, int64_t T_cap, const int32_t* cand_pos,
+                              const int32_t* cand_count, int C_cap, float threshold, float* scores,
+                              int32_t* best_pos, float* best_score, uint32_t* status) {
+    if (S > 1)
+        return launch_rank(rank_hidden_avg_kernel<T, VEC, true>, B, S, smem, stream, h, d, seq_stride, m, seq_len,
+                           T_cap, cand_pos, cand_count, C_cap, threshold, scores, best_pos, best_score, status);
+    return launch_rank(rank_hidden_avg_kernel<T, VEC, false>, B, S, smem, stream, h, d, seq_stride, m, seq_len,
+                       T_cap, cand_pos, cand_count, C_cap, threshold, scores, best_pos, best_score, status);
+}
+
 }  // namespace
 }  // namespace pldp
 
 using namespace pldp;
+
+extern "C" PLDP_API pldp_status pldp_rank_hidden_avg(const void* H, pldp_dtype dtype, int64_t d,
+                                                     int64_t seq_stride, int m, const int32_t* seq_len,
+                                                     int B, int64_t T_cap, const int32_t* cand_pos,
+                                                     const int32_t* cand_count, int C_cap, float threshold,
+                                                     float* scores, int32_t* best_pos, float* best_score,
+                                                     uint32_t* status, void* stream) {
+    if (B < 0) return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: B < 0");
+    if (dtype != PLDP_F32 && dtype != PLDP_BF16)
+        return fail(PLDP_ERR_UNSUPPORTED, "rank_hidden_avg: unsupported dtype %d", (int)dtype);
+    const size_t es = dtype == PLDP_F32 ? 4 : 2;
+    if (d < 1) return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: d < 1");
+    if (m < 1) return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: m < 1");
+    if (static_cast<size_t>(d) * sizeof(float) > kMaxAvgQueryBytes)
+        return fail(PLDP_ERR_UNSUPPORTED, "rank_hidden_avg: d * 4 > %zu", kMaxAvgQueryBytes);
+    if (T_cap < 0 || T_cap > INT32_MAX) return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: bad T_cap");
+    if (seq_stride < T_cap * d) return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: seq_stride < T_cap*d");
+    if (C_cap < 0) return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: C_cap < 0");
+    if (threshold != threshold) return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: threshold is NaN");
+    if (B == 0) return PLDP_OK;
+    if (!H || !seq_len || !cand_count || !best_pos || (C_cap > 0 && !cand_pos))
+        return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: null pointer");
+
+    const bool vec = aligned16(H) && (d * es) % 16 == 0 && (seq_stride * es) % 16 == 0;
+    const int S = pick_split(B, C_cap);
+    const size_t smem = (static_cast<size_t>(d) * sizeof(float) + 127) / 128 * 128;
+    cudaError_t e;
+    if (dtype == PLDP_BF16) {
+        const __nv_bfloat16* h = static_cast<const __nv_bfloat16*>(H);
+        e = vec ? launch_hidden_avg<__nv_bfloat16, true>(B, S, smem, stream, h, d, seq_stride, m, seq_len, T_cap,
+                                                         cand_pos, cand_count, C_cap, threshold, scores, best_pos,
+                                                         best_score, status)
+                : launch_hidden_avg<__nv_bfloat16, false>(B, S, smem, stream, h, d, seq_stride, m, seq_len, T_cap,
+                                                          cand_pos, cand_count, C_cap, threshold, scores, best_pos,
+                                                          best_score, status);
+    } else {
+        const float* h = static_cast<const float*>(H);
+        e = vec ? launch_hidden_avg<float, true>(B, S, smem, stream, h, d, seq_stride, m, seq_len, T_cap, cand_pos,
+                                                 cand_count, C_cap, threshold, scores, best_pos, best_score, status)
+                : launch_hidden_avg<float, false>(B, S, smem, stream, h, d, seq_stride, m, seq_len, T_cap, cand_pos,
+                                                  cand_count, C_cap, threshold, scores, best_pos, best_score,
+                                                  status);
+    }
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "rank_hidden_avg: launch failed: %s", cudaGetErrorString(e));
+    return PLDP_OK;
+}
 
 extern "C" PLDP_API pldp_status pldp_rank_hidden(const void* H, pldp_dtype dtype, int64_t d,
                                                  int64_t seq_stride, const int32_t* seq_len, int B,

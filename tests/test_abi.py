@@ -68,6 +68,12 @@ def test_host_argument_checks(so):
     assert lib.pldp_rank_hidden(*bad) == 2
     bad = list(args); bad[10] = float("nan")
     assert lib.pldp_rank_hidden(*bad) == 1
+    # rank_hidden_avg: m < 1, d too large for the fp32 query sum
+    av = [null, 1, 64, 64 * 8, 2, null, 1, 8, null, null, 4, float("-inf"), null, null, null, null, null]
+    bad = list(av); bad[4] = 0
+    assert lib.pldp_rank_hidden_avg(*bad) == 1 and "m < 1" in pk.pldp_last_error()
+    bad = list(av); bad[2] = 49153; bad[3] = 49153 * 8
+    assert lib.pldp_rank_hidden_avg(*bad) == 2
     # rank_attention: bad aggregation, n_sel out of range
     a = [null, 1, 4, 8, 32, null, 4, 0, null, 1, 8, null, null, 4, null, null, null, null, null]
     bad = list(a); bad[7] = 5
