@@ -72,12 +72,14 @@ def _configure(lib):
                                          P, P, P, P]
     lib.pldpo_extract_draft.argtypes = [P, i64, P, i64, P, i32, i32, P, P]
     lib.pldpo_verify_greedy.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64, P, i64, P, P]
+    lib.pldpo_identify_heads.argtypes = [P, i64, P, i32, i64, i32, P, i32, i32, i64, i64, P, P, P]
     lib.pldpo_rank_hidden_avg.argtypes = [P, i32, i64, i64, i32, P, i32, i64, P, P, i32, ctypes.c_double, P, P,
                                           P, P]
     lib.pldpo_verify_sample.argtypes = [P, i32, i32, i32, i32, ctypes.c_double, P, P, P, P, P, P, P, i64,
                                         P, i64, P, P]
     for f in ("pldpo_find_candidates", "pldpo_rank_hidden", "pldpo_rank_attention",
-              "pldpo_extract_draft", "pldpo_verify_greedy", "pldpo_verify_sample", "pldpo_rank_hidden_avg"):
+              "pldpo_extract_draft", "pldpo_verify_greedy", "pldpo_verify_sample", "pldpo_rank_hidden_avg",
+              "pldpo_identify_heads"):
         getattr(lib, f).restype = ctypes.c_int
 
 
@@ -176,6 +178,25 @@ def rank_hidden_avg(H, seq_len, cand_pos, cand_count, m, threshold=-np.inf, stat
                                          _ptr(cand_pos), _ptr(cand_count), C_cap, float(threshold),
                                          _ptr(scores), _ptr(best), _ptr(bs), _ptr(status)), "rank_hidden_avg")
     return scores, best, bs
+
+
+def identify_heads(ids, pos, A, max_suffix=64, counts=None):
+    """Sec. 4.2.1 head identification.  ids int32 [B, T_cap]; pos int32 [B] (the
+    generated token's position p); A [B, R, T_cap] float32 or bf16 bits, the rows of
+    query p-1.  Returns (counts uint32 [R] (added to ``counts`` when given), r_star
+    int32 [B], status uint32 [B])."""
+    ids = _i32(ids)
+    B, T_cap = ids.shape
+    A, dt = _elem(A)
+    R = A.shape[1]
+    pos = _i32(pos)
+    c = np.zeros(R, np.uint32) if counts is None else counts
+    assert c.dtype == np.uint32 and c.flags.c_contiguous and c.size == R
+    rs = np.zeros(B, np.int32)
+    st = np.zeros(B, np.uint32)
+    _check(_load().pldpo_identify_heads(_ptr(ids), T_cap, _ptr(pos), B, T_cap, int(max_suffix), _ptr(A), dt, R,
+                                        A.shape[2], R * A.shape[2], _ptr(c), _ptr(rs), _ptr(st)), "identify_heads")
+    return c, rs, st
 
 
 def rank_attention(A, seq_len, cand_pos, cand_count, row_idx=None, agg=AGG_MAX, status=None):

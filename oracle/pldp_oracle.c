@@ -332,6 +332,63 @@ int pldpo_extract_draft(const int32_t* ids, int64_t ids_stride, const int32_t* s
     return 0;
 }
 
+/* --------------------------------------------------------------------------
+ * Induction-head identification (Sec. 4.2.1): for generated tokens that also
+ * occur earlier, find the position r* they were most likely copied from, and
+ * count, for every (layer, head) row, how often that row puts its maximum
+ * attention on r*.  The rows with the highest counts are the G* / L* of Eq. 2.
+ *
+ * Observation b: the generated token is x_p with p = pos[b]; ids[b, 0..p] is
+ * the context; A holds, per observation, the R attention rows of query p-1 over
+ * keys 0..p-1: element (r, key) at A[b*seq_stride + r*row_stride + key].
+ *   P      = {j < p : x_j = x_p}
+ *   ov(j)  = the largest k <= max_suffix with x_{j-i} = x_{p-i} for i < k
+ *            (the overlapping suffix of the context before j and the output)
+ *   r*     = argmax_{j in P} ov(j)
+ *   row r counts when argmax_{key < p} A[r, key] = r*.
+ * READING: ties in ov(j) go to the smallest j (the library's tie rule); ties in
+ * a row's maximum go to the smallest key; "the token position x_{r*} has the
+ * maximum attention" is read per row (r* is the argmax of that head's row).
+ * r_star[b] = r*, or -1 when P is empty (then nothing is counted); counts[r]
+ * are ADDED to (uint32, caller-initialised) so that batches accumulate.
+ * pos[b] outside [1, T_cap - 1] sets SEQ_LEN and counts nothing.
+ * ------------------------------------------------------------------------ */
+int pldpo_identify_heads(const int32_t* ids, int64_t ids_stride, const int32_t* pos, int B,
+                         int64_t T_cap, int max_suffix, const void* A, int dtype, int R,
+                         int64_t row_stride, int64_t seq_stride, uint32_t* counts,
+                         int32_t* r_star, uint32_t* status) {
+    if (B < 0 || R < 1 || max_suffix < 1 || (dtype != ORC_F32 && dtype != ORC_BF16)) return 1;
+    for (int b = 0; b < B; ++b) {
+        int64_t p = pos[b];
+        if (r_star) r_star[b] = -1;
+        if (p < 1 || p >= T_cap) {
+            if (status) status[b] |= ORC_ST_SEQ_LEN;
+            continue;
+        }
+        const int32_t* x = ids + (int64_t)b * ids_stride;
+        int64_t rs = -1, best_ov = 0;
+        for (int64_t j = 0; j < p; ++j) {
+            if (x[j] != x[p]) continue;
+            int64_t k = 0;
+            while (k < max_suffix && j - k >= 0 && x[j - k] == x[p - k]) ++k;
+            if (k > best_ov) { best_ov = k; rs = j; }     /* strict: the smallest j keeps a tie */
+        }
+        if (r_star) r_star[b] = (int32_t)rs;
+        if (rs < 0) continue;
+        for (int r = 0; r < R; ++r) {
+            int64_t row = (int64_t)b * seq_stride + (int64_t)r * row_stride;
+            double mx = orc_load(A, dtype, row);
+            int64_t arg = 0;
+            for (int64_t key = 1; key < p; ++key) {
+                double v = orc_load(A, dtype, row + key);
+                if (v > mx) { mx = v; arg = key; }
+            }
+            if (arg == rs) counts[r] += 1u;
+        }
+    }
+    return 0;
+}
+
 /* Acceptance and bookkeeping shared by both verifications, for sequence b
  * whose K+1 target tokens (argmax or sampled) are tok[0..K]:
  * n = first i < d with draft_i != tok_i (else d), bonus = tok_n, then the

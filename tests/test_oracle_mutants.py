@@ -69,6 +69,15 @@ MUTANTS = [
      "int64_t lo = p - m + 1;\n    if (lo < 0) lo = 0;", "int64_t lo = p - m;\n    if (lo < 0) lo = 0;"),
     ("averaging window misses the row averaged",
      "for (int64_t r = lo; r <= p; ++r)", "for (int64_t r = lo; r < p; ++r)"),
+    ("identification overlap ignores the copied token itself",
+     "while (k < max_suffix && j - k >= 0 && x[j - k] == x[p - k]) ++k;",
+     "while (k < max_suffix && j - k - 1 >= 0 && x[j - k - 1] == x[p - k - 1]) ++k;"),
+    ("identification tie goes to the larger position",
+     "if (k > best_ov) { best_ov = k; rs = j; }", "if (k >= best_ov) { best_ov = k; rs = j; }"),
+    ("identification row argmax keeps the last maximum",
+     "if (v > mx) { mx = v; arg = key; }", "if (v >= mx) { mx = v; arg = key; }"),
+    ("identification looks at the generated position's own key",
+     "for (int64_t key = 1; key < p; ++key) {", "for (int64_t key = 1; key <= p; ++key) {"),
     ("sampling draws where the cumulative sum only reaches u",
      "if (c > target) { y = (int32_t)v; break; }", "if (c >= target) { y = (int32_t)v; break; }"),
     ("sampling multiplies by the temperature",

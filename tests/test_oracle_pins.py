@@ -411,3 +411,96 @@ def test_rank_hidden_avg_tie_goes_to_smaller_position(orc):
     cand = np.array([[17, 9, 25]], np.int32)
     s, best, _ = orc.rank_hidden_avg(H, np.array([30], np.int32), cand, np.array([2], np.int32), 3)
     assert s[0, 0] == s[0, 1] and best[0] == 9
+
+
+# ----------------------------------------------------------------------------
+# induction-head identification (Sec. 4.2.1)
+# ----------------------------------------------------------------------------
+def _identify_brute(ids, pos, A, max_suffix):
+    """Direct restatement with Python loops: P, overlap, r* (smallest j on ties),
+    and per row numpy's first argmax over keys < p."""
+    B, R, _ = A.shape
+    counts = np.zeros(R, np.uint32)
+    rs = np.full(B, -1, np.int32)
+    for b in range(B):
+        p = int(pos[b])
+        x = ids[b]
+        best = (0, 0)
+        for j in range(p):
+            if x[j] != x[p]:
+                continue
+            k = 0
+            while k < max_suffix and j - k >= 0 and x[j - k] == x[p - k]:
+                k += 1
+            if (k, -j) > best:
+                best = (k, -j)
+        if best[0] == 0:
+            continue
+        rs[b] = -best[1]
+        for r in range(R):
+            if int(np.argmax(A[b, r, :p])) == rs[b]:
+                counts[r] += 1
+    return counts, rs
+
+
+@pytest.mark.parametrize("V,max_suffix", [(2, 64), (3, 2), (5, 1), (50, 64)])
+def test_identify_heads_matches_brute_force(orc, V, max_suffix):
+    rng = np.random.default_rng(V * 10 + max_suffix)
+    B, T, R = 40, 30, 6
+    ids = rng.integers(0, V, size=(B, T)).astype(np.int32)
+    pos = rng.integers(1, T, size=B).astype(np.int32)
+    A = rng.integers(0, 4, size=(B, R, T)).astype(np.float32)       # many equal maxima
+    for b in range(0, B, 3):                                       # some rows point at a repeat
+        p = pos[b]
+        occ = [j for j in range(p) if ids[b, j] == ids[b, p]]
+        if occ:
+            A[b, rng.integers(0, R), occ[-1]] = 9.0
+    c, rs, st = orc.identify_heads(ids, pos, A, max_suffix)
+    wc, wrs = _identify_brute(ids, pos, A, max_suffix)
+    assert np.array_equal(rs, wrs) and np.array_equal(c, wc) and (st == 0).all()
+
+
+def test_identify_heads_recovers_planted_heads(orc):
+    """Copied spans; rows of 3 planted heads per layer put extra attention on the
+    true copy source of the generated token: they are exactly the top heads."""
+    import workloads as wl
+    w = wl.CONFIGS["c4"].replace(B=24, prompt_len=600, out_len=400, V=5000, layers=2, heads=8,
+                                 planted_heads=3)
+    tok, src = wl.token_streams(w, w.T, 77)
+    rng = np.random.default_rng(78)
+    obs_b, obs_p = [], []
+    for b in range(w.B):                                           # positions deep inside copied spans
+        inside = [p for p in range(w.prompt_len + 2, w.T)
+                  if src[b, p] >= 2 and src[b, p - 1] == src[b, p] - 1 and src[b, p - 2] == src[b, p] - 2]
+        for p in rng.choice(inside, size=min(4, len(inside)), replace=False):
+            obs_b.append(b)
+            obs_p.append(p)
+    n = len(obs_b)
+    ids = tok[obs_b].astype(np.int32)
+    pos = np.array(obs_p, np.int32)
+    R, T = w.layers * w.heads, w.T
+    planted = set(wl.induction_rows(w).tolist())
+    logits = rng.normal(size=(n, R, T))
+    for i in range(n):
+        for r in planted:
+            logits[i, r, src[obs_b[i], obs_p[i]]] += 8.0
+        logits[i, :, obs_p[i]:] = -np.inf
+    A = np.exp(logits - logits.max(-1, keepdims=True))
+    A = (A / A.sum(-1, keepdims=True)).astype(np.float32)
+    c, rs, _ = orc.identify_heads(ids, pos, A)
+    assert np.array_equal(rs, [src[b, p] for b, p in zip(obs_b, obs_p)])
+    top = set(np.argsort(-c.astype(np.int64), kind="stable")[:len(planted)].tolist())
+    assert top == planted and c[sorted(planted)].min() == n
+
+
+def test_identify_heads_edges_and_accumulation(orc):
+    ids = np.array([[1, 2, 3, 4, 5, 6], [7, 8, 7, 8, 7, 8]], np.int32)
+    A = np.zeros((2, 2, 6), np.float32)
+    A[1, 0, 3] = 1.0                      # row 0 points at key 3 (x_3 = 8, overlap 4)
+    A[1, 1, 1] = 1.0                      # row 1 at key 1 (overlap 2)
+    c, rs, st = orc.identify_heads(ids, np.array([5, 5], np.int32), A)
+    assert rs.tolist() == [-1, 3] and c.tolist() == [1, 0] and st.tolist() == [0, 0]
+    c2, _, _ = orc.identify_heads(ids, np.array([5, 5], np.int32), A, counts=c)
+    assert c2.tolist() == [2, 0]
+    _, rs, st = orc.identify_heads(ids, np.array([0, 6], np.int32), A)
+    assert rs.tolist() == [-1, -1] and st.tolist() == [orc.ST_SEQ_LEN, orc.ST_SEQ_LEN]
