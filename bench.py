@@ -419,6 +419,7 @@ def run_ours(args, ws_, rank, local):
     if not args.no_sample:
         out["sampling_verify"] = time_sampling_verify(pk, loop, w, flush_l2, peak)
         out["rank_hidden_avg"] = time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak)
+        out["identify_heads"] = time_identify_heads(pk, loop, w, flush_l2, peak)
     if not args.no_e2e:
         out["e2e"] = run_e2e(pk, loop, path, K_steps, W_steps, ws_)
     if rank == 0 and ws_ == 1 and not args.no_cpu_baseline:
@@ -491,6 +492,41 @@ def time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak, m=4, calls=64, warm=
                 "bound": "latency (a few MB gathered per call)",
                 "timing": "CUDA events around each call, L2 flushed before each"})
     return res
+
+
+def time_identify_heads(pk, loop, w, flush_l2, peak, calls=16, warm=2):
+    """Induction-head identification (Sec. 4.2.1) over the loop's current state: each
+    sequence's last token x_t is an observation, with the attention rows of query
+    t-1 that the workload plants on the copy source in its chosen heads.  Timed per
+    call (pldp_identify_heads then pldp_top_heads) with CUDA events, L2 flushed
+    before each; algorithmic bytes: every row over keys < t plus the ids scanned."""
+    dev = loop.device
+    loop.step_inputs(0)                                   # attention rows for the current lengths
+    pos = (loop.seq_len - 1).to(torch.int32)
+    R = w.R
+    counts = torch.zeros(R, dtype=torch.int32, device=dev)
+    k = int(wl.induction_rows(w).size)
+    top = torch.zeros(k, dtype=torch.int32, device=dev)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(calls)]
+    s = torch.cuda.current_stream()
+    for i in range(warm + calls):
+        flush_l2(i)
+        counts.zero_()
+        if i >= warm:
+            ev[i - warm][0].record(s)
+        pk.pldp_identify_heads(loop.ids, pos, loop.A, counts)
+        pk.pldp_top_heads(counts, k, top)
+        if i >= warm:
+            ev[i - warm][1].record(s)
+    torch.cuda.synchronize()
+    us = float(np.mean([a.elapsed_time(b) for a, b in ev])) * 1e3
+    keys = float(pos.double().sum().item())
+    by = keys * R * 2.0 + keys * 4.0
+    recovered = sorted(top.cpu().tolist()) == sorted(wl.induction_rows(w).tolist())
+    return {"observations": w.B, "rows": R, "us_per_call": round(us, 2), "algorithmic_bytes": by,
+            "achieved_gbs": round(by / (us * 1e-6) / 1e9, 1), "peak_gbs": peak,
+            "frac": round(by / (us * 1e-6) / 1e9 / peak, 4), "top_rows_are_the_planted_heads": recovered,
+            "timing": "CUDA events around pldp_identify_heads + pldp_top_heads, L2 flushed before each"}
 
 
 def path_draft(loop, w):

@@ -399,6 +399,45 @@ PLDP_API pldp_status pldp_verify_greedy_noalloc(const void* logits, pldp_dtype d
 /* Bytes of workspace pldp_verify_greedy needs for these sizes (0 if invalid). */
 PLDP_API size_t pldp_verify_workspace_size(int B, int K, int V);
 
+/*
+ * Induction-head identification -- Sec. 4.2.1, the offline step that picks the
+ * (layer, head) rows Eq. 2 aggregates.  Each observation b is a generated token
+ * x_p (p = pos[b]) with its context ids[b, 0..p] and the attention rows of query
+ * p-1 over keys 0..p-1 for R candidate (layer, head) rows:
+ *   P      = {j < p : x_j = x_p}
+ *   ov(j)  = the largest k <= max_suffix with x_{j-i} = x_{p-i} for all i < k
+ *   r*     = argmax_{j in P} ov(j)              (the smaller j on ties)
+ *   counts[r] += 1 when row r's largest attention is at key r*
+ *                                               (the smaller key on ties)
+ * The paper's rule is read per row: a head counts when r* is where its own
+ * attention peaks.  Run it over many observations, then keep the rows with the
+ * most counts (pldp_top_heads).
+ *
+ *  ids, ids_stride, T_cap   int32 contexts [B, ids_stride], T_cap <= ids_stride.
+ *  pos        int32 [B]; outside [1, T_cap - 1]: SEQ_LEN, nothing counted.
+ *  max_suffix >= 1: cap on ov(j).
+ *  A          dtype [B, seq_stride]: row r of observation b at
+ *             A + b*seq_stride + r*row_stride, keys 0..p-1 (row_stride >= T_cap,
+ *             seq_stride >= R*row_stride).
+ *  counts     uint32 [R], ADDED to (initialise once, accumulate over calls).
+ *  r_star     int32 [B] out or NULL: r*, -1 when x_p does not occur before p.
+ *  status     uint32 [B] or NULL.
+ * Atomic adds on counts: concurrent calls on one counts array accumulate
+ * correctly.  Offline utility: not part of the decode step.
+ */
+PLDP_API pldp_status pldp_identify_heads(const int32_t* ids, int64_t ids_stride, const int32_t* pos,
+                                         int B, int64_t T_cap, int max_suffix, const void* A,
+                                         pldp_dtype dtype, int R, int64_t row_stride,
+                                         int64_t seq_stride, uint32_t* counts, int32_t* r_star,
+                                         uint32_t* status, void* stream);
+
+/*
+ * The k rows with the most counts (ties to the smaller row index), written in
+ * that order to row_idx int32 [k] -- the row_idx argument of pldp_rank_attention.
+ * 1 <= k <= R <= 8192.  counts: uint32 [R] (device).
+ */
+PLDP_API pldp_status pldp_top_heads(const uint32_t* counts, int R, int k, int32_t* row_idx, void* stream);
+
 /* Message describing the last failed call on this host thread ("" if none). */
 PLDP_API const char* pldp_last_error(void);
 

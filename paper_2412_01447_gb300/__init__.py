@@ -102,6 +102,10 @@ def _load():
             lib.pldp_find_candidates.argtypes = [P, i64, P, i32, i64, i32, i32, P, i32, P, P, P, P]
             lib.pldp_rank_hidden.argtypes = [P, i32, i64, i64, P, i32, i64, P, P, i32, f32, P, P, P,
                                              P, P]
+            lib.pldp_identify_heads.argtypes = [P, i64, P, i32, i64, i32, P, i32, i32, i64, i64, P, P, P, P]
+            lib.pldp_identify_heads.restype = ctypes.c_int
+            lib.pldp_top_heads.argtypes = [P, i32, i32, P, P]
+            lib.pldp_top_heads.restype = ctypes.c_int
             lib.pldp_rank_hidden_avg.argtypes = [P, i32, i64, i64, i32, P, i32, i64, P, P, i32, f32, P, P,
                                                  P, P, P]
             lib.pldp_rank_hidden_avg.restype = ctypes.c_int
@@ -235,6 +239,28 @@ def pldp_rank_hidden_avg(H, seq_len, cand_pos, cand_count, best_pos, m, scores=N
         _dense(best_pos, "best_pos", torch.int32),
         _dense(best_score, "best_score", torch.float32, allow_none=True),
         _dense(status, "status", None, allow_none=True), _stream(stream)))
+
+
+def pldp_identify_heads(ids, pos, A, counts, max_suffix=64, r_star=None, status=None, stream=None):
+    """Sec. 4.2.1 head identification.  ids int32 [B, T_cap]; pos int32 [B] (the
+    generated token's position p); A [B, R, T_cap] float32/bfloat16, the attention
+    rows of query p-1 (unit inner stride); counts int32/uint32 [R] CUDA tensor,
+    added to.  r_star int32 [B] out (optional)."""
+    p_ids, stride, T_cap = _rows(ids, "ids")
+    if A.dim() != 3 or A.stride(2) != 1:
+        raise ValueError("A must be [B, R, T_cap] with unit inner stride")
+    B, R = A.shape[0], A.shape[1]
+    _check("pldp_identify_heads", _load().pldp_identify_heads(
+        p_ids, stride, _dense(pos, "pos", torch.int32), B, T_cap, int(max_suffix), _dev(A, "A"), _code(A.dtype),
+        R, A.stride(1), A.stride(0), _dense(counts, "counts", None), _dense(r_star, "r_star", torch.int32,
+                                                                             allow_none=True),
+        _dense(status, "status", None, allow_none=True), _stream(stream)))
+
+
+def pldp_top_heads(counts, k, row_idx, stream=None):
+    """The k rows with the most counts (ties to the smaller index) into row_idx int32 [k]."""
+    _check("pldp_top_heads", _load().pldp_top_heads(_dense(counts, "counts", None), counts.numel(), int(k),
+                                                    _dense(row_idx, "row_idx", torch.int32), _stream(stream)))
 
 
 def pldp_rank_attention(A, seq_len, cand_pos, cand_count, best_pos, row_idx=None, agg=PLDP_AGG_MAX,

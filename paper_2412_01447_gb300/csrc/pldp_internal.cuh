@@ -65,6 +65,36 @@ __device__ __forceinline__ float warp_sum(float v) {
     return v;
 }
 
+// Max and first index of the max of one 16-byte vector (8 bf16 or 4 fp32): a
+// packed max first, the index search only when the caller needs it.
+__device__ __forceinline__ float vmax(const uint4& x, __nv_bfloat16) {
+    const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&x.x);
+    const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&x.y);
+    const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&x.z);
+    const __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&x.w);
+    const __nv_bfloat162 m = __hmax2(__hmax2(a, b), __hmax2(c, d));
+    return fmaxf(__low2float(m), __high2float(m));
+}
+__device__ __forceinline__ int vfirst(const uint4& x, float m, __nv_bfloat16) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        if (__uint_as_float(w[k] << 16) == m) return 2 * k;
+        if (__uint_as_float(w[k] & 0xFFFF0000u) == m) return 2 * k + 1;
+    }
+    return 0;
+}
+__device__ __forceinline__ float vmax(const uint4& x, float) {
+    return fmaxf(fmaxf(__uint_as_float(x.x), __uint_as_float(x.y)),
+                 fmaxf(__uint_as_float(x.z), __uint_as_float(x.w)));
+}
+__device__ __forceinline__ int vfirst(const uint4& x, float m, float) {
+    if (__uint_as_float(x.x) == m) return 0;
+    if (__uint_as_float(x.y) == m) return 1;
+    if (__uint_as_float(x.z) == m) return 2;
+    return 3;
+}
+
 // Streaming 16-byte global load (read-once data: no L1 allocation).
 __device__ __forceinline__ uint4 ld_stream16(const void* p) {
     uint4 r;

@@ -51,35 +51,6 @@ __global__ void extract_draft_kernel(const int32_t* __restrict__ ids, int64_t id
     if (i == 0) draft_len[b] = static_cast<int32_t>(d);
 }
 
-// ---- per-vector max and first index of the max ---------------------------------
-__device__ __forceinline__ float vmax(const uint4& x, __nv_bfloat16) {
-    const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&x.x);
-    const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&x.y);
-    const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162*>(&x.z);
-    const __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162*>(&x.w);
-    const __nv_bfloat162 m = __hmax2(__hmax2(a, b), __hmax2(c, d));
-    return fmaxf(__low2float(m), __high2float(m));
-}
-__device__ __forceinline__ int vfirst(const uint4& x, float m, __nv_bfloat16) {
-    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-        if (__uint_as_float(w[k] << 16) == m) return 2 * k;
-        if (__uint_as_float(w[k] & 0xFFFF0000u) == m) return 2 * k + 1;
-    }
-    return 0;
-}
-__device__ __forceinline__ float vmax(const uint4& x, float) {
-    return fmaxf(fmaxf(__uint_as_float(x.x), __uint_as_float(x.y)),
-                 fmaxf(__uint_as_float(x.z), __uint_as_float(x.w)));
-}
-__device__ __forceinline__ int vfirst(const uint4& x, float m, float) {
-    if (__uint_as_float(x.x) == m) return 0;
-    if (__uint_as_float(x.y) == m) return 1;
-    if (__uint_as_float(x.z) == m) return 2;
-    return 3;
-}
-
 // Running (max, first index) of one lane over elements [c0, c1) of a row.
 template <typename T, bool VEC>
 __device__ __forceinline__ void lane_argmax(const T* __restrict__ row, int64_t c0, int64_t c1,

@@ -74,6 +74,14 @@ def test_host_argument_checks(so):
     assert lib.pldp_rank_hidden_avg(*bad) == 1 and "m < 1" in pk.pldp_last_error()
     bad = list(av); bad[2] = 49153; bad[3] = 49153 * 8
     assert lib.pldp_rank_hidden_avg(*bad) == 2
+    # identify_heads: max_suffix < 1, row_stride < T_cap; top_heads: k > R
+    ih = [null, 16, null, 2, 16, 8, null, 1, 4, 16, 64, null, null, null, null]
+    bad = list(ih); bad[5] = 0
+    assert lib.pldp_identify_heads(*bad) == 1 and "max_suffix" in pk.pldp_last_error()
+    bad = list(ih); bad[9] = 8
+    assert lib.pldp_identify_heads(*bad) == 1 and "row_stride" in pk.pldp_last_error()
+    assert lib.pldp_top_heads(ctypes.c_void_p(256), 4, 5, ctypes.c_void_p(256), null) == 1
+    assert lib.pldp_top_heads(ctypes.c_void_p(256), 9000, 5, ctypes.c_void_p(256), null) == 1
     # rank_attention: bad aggregation, n_sel out of range
     a = [null, 1, 4, 8, 32, null, 4, 0, null, 1, 8, null, null, 4, null, null, null, null, null]
     bad = list(a); bad[7] = 5
