@@ -189,12 +189,20 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def profiled_traffic(kernel_src, profile_name):
+def source_sha256(paths):
+    """sha256 over the concatenated source files a kernel is built from."""
+    h = hashlib.sha256()
+    for p in paths:
+        h.update(open(p, "rb").read())
+    return h.hexdigest()
+
+
+def profiled_traffic(kernel_srcs, profile_name):
     """Per-launch DRAM bytes from the committed ncu summary, valid only while the
-    kernel source is the one that was profiled (its sha256 is recorded there)."""
+    kernel sources are the ones that were profiled (their sha256 is recorded there)."""
     try:
         txt = open(os.path.join(ROOT, "profiles", profile_name)).read()
-        sha = hashlib.sha256(open(kernel_src, "rb").read()).hexdigest()
+        sha = source_sha256(kernel_srcs)
         rec = dict(ln.split(":", 1) for ln in txt.splitlines() if ln.startswith(("traffic_bytes_per_launch",
                                                                                "source_sha256")))
         if rec.get("source_sha256", "").strip() != sha:
@@ -361,7 +369,8 @@ def run_ours(args, ws_, rank, local):
     ver_s = per_k[nk - 1] / K_steps / 1e3
     ver_bytes = by["verify_greedy"]
     achieved = ver_bytes / ver_s / 1e9
-    traffic = profiled_traffic(os.path.join(ROOT, "paper_2412_01447_gb300", "csrc", "verify.cu"),
+    csrc = os.path.join(ROOT, "paper_2412_01447_gb300", "csrc")
+    traffic = profiled_traffic([os.path.join(csrc, "verify.cu"), os.path.join(csrc, "pldp_internal.cuh")],
                                "verify_greedy_c5.md")
     step_bytes_total = sum(by[k] for k in ("find_candidates", "rank_hidden", "rank_attention",
                                             "extract_draft", "verify_greedy"))
