@@ -53,12 +53,18 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="c5")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--slack-us", type=float, default=300.0,
+                    help="GPU spin after each flush, outside the timed region, so that a step's launches "
+                         "are all queued before its first event (the intervals then hold no host time)")
     ap.add_argument("--flush", choices=["write-read", "write"], default="write-read",
                     help="L2 flush before each step: write 256 MB then read 256 MB (cold, clean L2), "
                          "or the write alone (cold L2 full of dirty lines)")
     ap.add_argument("--events", choices=["kernel", "step"], default="kernel",
                     help="CUDA events around every kernel (per-kernel times, the roofline) or only "
                          "around each step (kernels chained by programmatic dependent launch)")
+    ap.add_argument("--scan", action="store_true",
+                    help="draft by scanning the contexts instead of with the incremental token index (which "
+                         "is built before the timed loop and kept up to date inside every timed step)")
     ap.add_argument("--separate", action="store_true",
                     help="draft with the four separate calls instead of the fused launch")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -215,7 +221,7 @@ def profiled_traffic(kernel_srcs, profile_name):
 class Path:
     """Device buffers and the five C-ABI calls of one step."""
 
-    def __init__(self, pk, loop: wl.DecodeLoop, fused=True):
+    def __init__(self, pk, loop: wl.DecodeLoop, fused=True, index=False):
         self.pk, self.loop = pk, loop
         w, dev = loop.w, loop.device
         B, K, C = w.B, w.K, w.C_cap
@@ -229,10 +235,17 @@ class Path:
         self.ws = torch.zeros(pk.pldp_verify_workspace_size(B, K, w.V), dtype=torch.uint8, device=dev)
         self.dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=dev)
         self.row_idx = None   # all R rows of the chosen layers
+        self.index = (torch.empty(pk.pldp_index_size(B, w.V), dtype=torch.uint8, device=dev)
+                      if index and fused else None)
         self.fused = fused
         self.launches_per_step = 3 if fused else 6     # pldp_verify_greedy launches two kernels
         self.kernels = (["draft_step"] if fused else
                         ["find_candidates", "rank_hidden", "rank_attention", "extract_draft"]) + ["verify_greedy"]
+
+    def build_index(self):
+        """(Re)builds the token index for the loop's current contexts (not timed)."""
+        if self.index is not None:
+            self.pk.pldp_index_build(self.loop.ids, self.loop.seq_len, self.loop.w.V, self.index)
 
     def run(self, ev=None, stream=None, step_only=False):
         """One step: the drafting half (one fused launch, or the four separate calls)
@@ -255,7 +268,7 @@ class Path:
             pk.pldp_draft_step(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt, self.ml,
                                w.K, self.draft, self.dlen, self.dws, H=lp.H, best_h=self.best_h, A=lp.A,
                                best_a=self.best_a, row_idx=self.row_idx, draft_from="hidden",
-                               status=self.status, stream=s)
+                               status=self.status, index=self.index, V=w.V, stream=s)
             rec()
         else:
             pk.pldp_find_candidates(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt,
@@ -309,15 +322,21 @@ def run_ours(args, ws_, rank, local):
     K_steps, W_steps = args.steps, args.warmup
     t0 = time.perf_counter()
     loop = wl.DecodeLoop(w, steps=W_steps + K_steps, device=dev)
-    path = Path(pk, loop, fused=not args.separate)
+    path = Path(pk, loop, fused=not args.separate, index=not args.scan)
+    path.build_index()
     nk = len(path.kernels)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)     # 2x the 129 MB L2
     flush_sink = torch.empty((), dtype=torch.int64, device=dev)
+
+    sm_hz = torch.cuda.get_device_properties(dev).clock_rate * 1e3 if hasattr(
+        torch.cuda.get_device_properties(dev), "clock_rate") else 2.07e9
 
     def flush_l2(s):
         flush.fill_(s & 0xFF)
         if args.flush == "write-read":
             torch.sum(flush.view(torch.int64), dim=0, out=flush_sink)   # evicts the dirty lines
+        if args.slack_us > 0:
+            torch.cuda._sleep(int(args.slack_us * 1e-6 * sm_hz))         # the host queues the step meanwhile
     torch.cuda.synchronize()
     setup_s = time.perf_counter() - t0
 
@@ -349,13 +368,16 @@ def run_ours(args, ws_, rank, local):
     clk = clocks.stop()
 
     per_k = np.zeros(nk)
+    per_step = np.zeros((K_steps, nk))
     if args.events == "step":                                 # no per-kernel split in this mode
         step_ms_total = float(sum(e[0].elapsed_time(e[1]) for e in evs))
         per_k[:] = np.nan
+        per_step[:] = np.nan
     else:
-        for e in evs:
+        for i, e in enumerate(evs):
             for k in range(nk):
-                per_k[k] += e[k].elapsed_time(e[k + 1])
+                per_step[i, k] = e[k].elapsed_time(e[k + 1])
+        per_k = per_step.sum(axis=0)
         step_ms_total = float(per_k.sum())                    # device ms over K steps
     step_ms_total = max_over_ranks(step_ms_total, ws_)
     ms_per_step = step_ms_total / K_steps
@@ -404,7 +426,9 @@ def run_ours(args, ws_, rank, local):
                           if args.flush == "write-read" else
                           "flushed before every step: 256 MB write (cold L2 holding dirty lines)")
                          + "; per-step logits 427 MB and attention rows 1.18 GB regenerated between steps",
-                   "path": ("pldp_draft_step (fused scan + both rankings + draft) + pldp_verify_greedy"
+                   "path": (("pldp_draft_step (incremental token index + both rankings + draft)"
+                             if path.index is not None else
+                             "pldp_draft_step (fused scan + both rankings + draft)") + " + pldp_verify_greedy"
                             if path.fused else "five separate C-ABI calls"),
                    "timing": "CUDA events around every kernel of each step on the launch stream; "
                              "artifact generation between steps is not timed",
@@ -412,6 +436,9 @@ def run_ours(args, ws_, rank, local):
         "achieved_step_gbs": round(step_bytes_total / (ms_per_step / 1e3) / 1e9, 1),
         "frac_step_of_nominal_8tbs": round(step_bytes_total / (ms_per_step / 1e3) / 1e9 / NOMINAL_HBM_GBS, 4),
         "kernel_us": {k: round(per_k[i] / K_steps * 1e3, 2) for i, k in enumerate(path.kernels)},
+        "kernel_us_p50_p90": {k: [round(float(np.percentile(per_step[:, i], 50)) * 1e3, 2),
+                                  round(float(np.percentile(per_step[:, i], 90)) * 1e3, 2)]
+                              for i, k in enumerate(path.kernels)},
         "kernel_gbs": {k: round(by[k] / (per_k[i] / K_steps / 1e3) / 1e9, 1)
                        for i, k in enumerate(path.kernels)},
         "roofline": {"kernel": "verify_greedy", "bound": "hbm", "achieved": round(achieved, 1),
@@ -425,6 +452,8 @@ def run_ours(args, ws_, rank, local):
                   "lossless_vs_ground_truth": lossless, "setup_s": round(setup_s, 1),
                   "timed_loop_wall_s": round(wall, 3)},
     }
+    if path.index is not None:
+        out["draft_scan_variant"] = time_scan_variant(pk, loop, w, flush_l2)
     if not args.no_sample:
         out["sampling_verify"] = time_sampling_verify(pk, loop, w, flush_l2, peak)
         out["rank_hidden_avg"] = time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak)
@@ -434,6 +463,24 @@ def run_ours(args, ws_, rank, local):
     if rank == 0 and ws_ == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline_from_loop(loop, path, w)
     return out
+
+
+def time_scan_variant(pk, loop, w, flush_l2, steps=64, warm=3):
+    """The same loop drafted by scanning the contexts (no token index), for comparison:
+    per-call CUDA events as in the timed loop, from the loop's initial state."""
+    loop.reset()
+    path = Path(pk, loop, fused=True, index=False)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for s in range(warm + steps):
+        loop.step_inputs(s)
+        flush_l2(s)
+        path.run(evs[s - warm] if s >= warm else None)
+    torch.cuda.synchronize()
+    d = [e[0].elapsed_time(e[1]) for e in evs]
+    v = [e[1].elapsed_time(e[2]) for e in evs]
+    return {"steps": steps, "us_per_step": round((sum(d) + sum(v)) / steps * 1e3, 2),
+            "draft_us": round(sum(d) / steps * 1e3, 2), "verify_us": round(sum(v) / steps * 1e3, 2),
+            "path": "pldp_draft_step scanning the contexts + pldp_verify_greedy"}
 
 
 def time_sampling_verify(pk, loop, w, flush_l2, peak, calls=64, warm=4, temperature=1.0):
@@ -550,6 +597,7 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     pass produced) from pinned host memory and reads back its results."""
     w, dev = loop.w, loop.device
     loop.reset()
+    path.build_index()                  # the contexts were cut back: index them again
     B, K1 = w.B, w.K + 1
     h_logits = torch.empty(loop.logits.shape, dtype=loop.logits.dtype, pin_memory=True)
     h_A = torch.empty(loop.A.shape, dtype=loop.A.dtype, pin_memory=True)
@@ -629,6 +677,7 @@ def cpu_baseline_from_loop(loop, path, w, budget_s=20.0, nseq=64, max_steps=192)
     import oracle
     oracle.build()
     loop.reset()
+    path.build_index()                  # the contexts were cut back: index them again
     nseq = min(nseq, w.B)
     max_steps = min(max_steps, loop.steps)
     Hs = np.zeros((nseq, loop.T_cap, w.d), np.uint16)       # zero pages until written

@@ -232,7 +232,20 @@ PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
  *  workspace             device scratch of pldp_draft_workspace_size(B) bytes,
  *                        16-byte aligned, ZEROED by the caller before its first
  *                        use; every call leaves it zeroed again.  Calls that may
- *                        run concurrently need separate workspaces.
+ *                        run concurrently need separate workspaces.  May be NULL
+ *                        when an index is given.
+ *  index, index_bytes, V optional incremental token index (NULL: scan the
+ *                        contexts): device memory of pldp_index_size(B, V)
+ *                        bytes, built by pldp_index_build, for token ids in
+ *                        [0, V).  With it, a step looks up the occurrences of
+ *                        x_t instead of scanning the context, and appends the
+ *                        positions added since the last step; results are the
+ *                        same as without it (a token with more than 8 earlier
+ *                        occurrences, or a sequence whose index is unusable,
+ *                        is scanned).  The index must only ever see the
+ *                        contexts grow by appending: a sequence whose length
+ *                        fell below what was indexed is marked unusable (and
+ *                        scanned) until the index is rebuilt.
  * Layouts the fused path does not take return PLDP_ERR_UNSUPPORTED; the
  * separate calls accept them.
  */
@@ -274,6 +287,9 @@ typedef struct pldp_draft_step_args {
     uint32_t* status;
     void* workspace;
     size_t workspace_bytes;
+    void* index;
+    size_t index_bytes;
+    int V;
 } pldp_draft_step_args;
 
 /* `args` is a HOST pointer to the argument block, read before the call returns. */
@@ -281,6 +297,21 @@ PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* args, void* str
 
 /* Bytes of workspace pldp_draft_step needs for B sequences (0 if B < 0). */
 PLDP_API size_t pldp_draft_workspace_size(int B);
+
+/*
+ * The incremental token index of pldp_draft_step (no counterpart in the paper:
+ * it is a way to find the occurrences of Eq. 1 without rescanning the context).
+ * Per sequence and token it holds the number of occurrences among the indexed
+ * positions and up to 8 of them; per sequence the number of positions indexed.
+ * pldp_index_build clears `index` and indexes positions 0 .. seq_len[b]-2 of
+ * every sequence (all but the last token, which the next draft step looks up).
+ * Token ids outside [0, V) mark that sequence's index unusable (TOKEN_RANGE);
+ * seq_len outside [0, T_cap] too (SEQ_LEN).  Memory: about B * V * 36 bytes.
+ */
+PLDP_API size_t pldp_index_size(int B, int V);
+PLDP_API pldp_status pldp_index_build(const int32_t* ids, int64_t ids_stride, const int32_t* seq_len,
+                                      int B, int64_t T_cap, int V, void* index,
+                                      size_t index_bytes, uint32_t* status, void* stream);
 
 /*
  * Greedy verification -- Sec. 4.4 at temperature 0, with the K+1 next-token

@@ -75,6 +75,7 @@ class pldp_draft_step_args(ctypes.Structure):
         ("draft_from", ctypes.c_int), ("K", ctypes.c_int), ("draft", ctypes.c_void_p),
         ("draft_len", ctypes.c_void_p), ("status", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
+        ("index", ctypes.c_void_p), ("index_bytes", ctypes.c_size_t), ("V", ctypes.c_int),
     ]
 
 
@@ -121,6 +122,10 @@ def _load():
             lib.pldp_draft_step.restype = ctypes.c_int
             lib.pldp_draft_workspace_size.argtypes = [i32]
             lib.pldp_draft_workspace_size.restype = sz
+            lib.pldp_index_size.argtypes = [i32, i32]
+            lib.pldp_index_size.restype = sz
+            lib.pldp_index_build.argtypes = [P, i64, P, i32, i64, i32, P, sz, P, P]
+            lib.pldp_index_build.restype = ctypes.c_int
             lib.pldp_verify_greedy_noalloc.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64,
                                                        P, i64, P, P, P]
             lib.pldp_verify_greedy_noalloc.restype = ctypes.c_int
@@ -301,10 +306,13 @@ def pldp_draft_step(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, ma
                     draft_len, workspace, H=None, best_h=None, h_scores=None, best_h_score=None,
                     threshold=float("-inf"), A=None, best_a=None, row_idx=None, agg=PLDP_AGG_MAX,
                     a_scores=None, best_a_score=None, draft_from="hidden", status=None, T_cap=None,
-                    stream=None):
+                    index=None, V=None, stream=None):
     """Candidate search, ranking (hidden and/or attention) and draft in one call; the
     arguments mean what they mean in the separate calls.  workspace: a uint8 CUDA
-    tensor of pldp_draft_workspace_size(B) bytes, zeroed once before first use."""
+    tensor of pldp_draft_workspace_size(B) bytes, zeroed once before first use (may be
+    None with an index).  index: a uint8 CUDA tensor of pldp_index_size(B, V) bytes
+    built by pldp_index_build (token ids in [0, V)); the step then looks occurrences
+    up instead of scanning, with the same results."""
     p_ids, stride, T = _rows(ids, "ids")
     B = ids.shape[0]
     a = pldp_draft_step_args()
@@ -339,9 +347,32 @@ def pldp_draft_step(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, ma
     a.draft = _dense(draft, "draft", torch.int32)
     a.draft_len = _dense(draft_len, "draft_len", torch.int32)
     a.status = _dense(status, "status", None, allow_none=True)
-    a.workspace = _dense(workspace, "workspace")
-    a.workspace_bytes = workspace.numel() * workspace.element_size()
+    if workspace is not None:
+        a.workspace = _dense(workspace, "workspace")
+        a.workspace_bytes = workspace.numel() * workspace.element_size()
+    if index is not None:
+        if V is None:
+            raise ValueError("an index needs V")
+        a.index = _dense(index, "index")
+        a.index_bytes = index.numel() * index.element_size()
+        a.V = int(V)
     _check("pldp_draft_step", _load().pldp_draft_step(ctypes.byref(a), _stream(stream)))
+
+
+def pldp_index_size(B, V) -> int:
+    return int(_load().pldp_index_size(B, V))
+
+
+def pldp_index_build(ids, seq_len, V, index, status=None, T_cap=None, stream=None):
+    """Builds the incremental token index of pldp_draft_step over positions
+    0 .. seq_len[b]-2 of every sequence.  index: uint8 CUDA tensor of
+    pldp_index_size(B, V) bytes (cleared by the call)."""
+    p_ids, stride, T = _rows(ids, "ids")
+    B = ids.shape[0]
+    _check("pldp_index_build", _load().pldp_index_build(
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32), B, T if T_cap is None else T_cap, int(V),
+        _dense(index, "index"), index.numel() * index.element_size(),
+        _dense(status, "status", None, allow_none=True), _stream(stream)))
 
 
 def pldp_verify_workspace_size(B, K, V) -> int:

@@ -41,7 +41,8 @@ constexpr int64_t kChunk = int64_t(kThreads) * kScanVec * 4;   // positions per 
 constexpr int kHitCap = 256;                                   // occurrences kept per sequence
 constexpr size_t kSeqWs = 16 + kHitCap * 16;                   // header + 16-byte entries
 constexpr int kScoreUnroll = 2;                                // 16-byte row loads in flight
-constexpr int kScoreBatch = 2;                                 // occurrences scored per pass
+constexpr int kScoreBatch = 2;                                 // occurrences scored per pass (scan kernel)
+constexpr int kMaxScoreBatch = 4;                              // ... and at most (the indexed kernel)
 constexpr size_t kMaxQueryBytes = 196608;
 constexpr int kMaxSelRows = 8192;
 constexpr int64_t kMaxPositions = int64_t(1) << 27;            // (j << 4) | m fits 31 bits
@@ -110,9 +111,14 @@ struct Hit {
     int32_t j, m;
 };
 
+template <int NB>
+__device__ __forceinline__ float (&part_buf(float (&part)[kMaxScoreBatch][kWarps][4]))[NB][kWarps][4] {
+    return *reinterpret_cast<float(*)[NB][kWarps][4]>(&part[0]);
+}
+
 struct StepShared {
     Hit hit[kHitCap];                        // occurrences this CTA found (the first kHitCap)
-    float part[2][kScoreBatch][kWarps][4];   // per-warp partial sums: dot, |a|^2, |q|^2, attention
+    float part[2][kMaxScoreBatch][kWarps][4];   // per-warp partial sums: dot, |a|^2, |q|^2, attention
     int32_t jl[kHitCap];                     // finish: positions of the candidates (else INT_MAX)
     unsigned long long wkey[2][kWarps];      // finish: per-warp best keys (hidden, attention)
     int wmax[kWarps];
@@ -129,12 +135,10 @@ struct StepShared {
 // depend on which pass or slot computes it.  Scores are returned in thread 0:
 // the cosine (-inf when j = 0 has no H_{j-1}) and the attention max / sum.
 // CTA-uniform call with one barrier; callers alternate `part` buffers.
-template <typename TH>
-__device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int64_t (&j)[kScoreBatch], int nb,
-                                          int64_t t, float (&part)[kScoreBatch][kWarps][4],
-                                          float (&s_h)[kScoreBatch], float (&s_a)[kScoreBatch]) {
+template <typename TH, int NB>
+__device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int64_t (&j)[NB], int nb, int64_t t,
+                                          float (&part)[NB][kWarps][4], float (&s_h)[NB], float (&s_a)[NB]) {
     constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
-    constexpr int NB = kScoreBatch;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const bool is_max = p.agg == PLDP_AGG_MAX;
     bool h_ok[NB], a_ok[NB];
@@ -278,7 +282,8 @@ __device__ __noinline__ void finish_overflow(const DraftParams& p, int b, int64_
 #pragma unroll
         for (int h = 0; h < kScoreBatch; ++h) j[h] = h < nb ? __ldcg(cand_row + i0 + h) : -1;
         float s_h[kScoreBatch], s_a[kScoreBatch];
-        cta_score<TH>(p, b, j, nb, t, sh.part[(i0 / kScoreBatch) & 1], s_h, s_a);
+        cta_score<TH, kScoreBatch>(p, b, j, nb, t, part_buf<kScoreBatch>(sh.part[(i0 / kScoreBatch) & 1]), s_h,
+                                   s_a);
         if (tid == 0)
             for (int h = 0; h < nb; ++h) {
                 const int i = i0 + h;
@@ -396,7 +401,8 @@ __global__ void __launch_bounds__(kThreads, 4) draft_step_kernel(const DraftPara
 #pragma unroll
                 for (int h = 0; h < kScoreBatch; ++h) j[h] = h < nb ? sh.hit[k + h].j : -1;
                 float s_h[kScoreBatch], s_a[kScoreBatch];
-                cta_score<TH>(p, b, j, nb, t, sh.part[(k / kScoreBatch) & 1], s_h, s_a);
+                cta_score<TH, kScoreBatch>(p, b, j, nb, t, part_buf<kScoreBatch>(sh.part[(k / kScoreBatch) & 1]), s_h,
+                                           s_a);
                 if (tid == 0)
                     for (int h = 0; h < nb; ++h) {
                         const Hit e = sh.hit[k + h];
@@ -533,6 +539,332 @@ __global__ void __launch_bounds__(kThreads, 4) draft_step_kernel(const DraftPara
     }
 }
 
+// ---------------------------------------------------------------------------
+// The incremental token index: drafting without rescanning the context.
+//
+// Per sequence b and token v the index holds how often v occurs among the
+// indexed positions (counts) and up to kIndexSlots of those positions (slots,
+// in no particular order); ilen[b] is the number of positions indexed (0 ..
+// ilen-1), -1 when the index of b is unusable.  A step with t = seq_len - 1:
+//  * reads x_t's count and slots in one round trip; when the count is at most
+//    kIndexSlots the slots are every occurrence before ilen, and the positions
+//    appended since (ilen .. t-1, read anyway) supply the rest;
+//  * otherwise (a frequent token, a stale or unusable index) falls back to the
+//    ordered rescan of the context, so results are those of the scan either way;
+//  * then appends positions ilen .. t-1 to the index and sets ilen = t.
+// Only the candidates (match length n*) are scored.  One CTA per sequence.
+// ---------------------------------------------------------------------------
+constexpr int kIndexSlots = 8;
+constexpr int kNewCap = kThreads;                  // appended positions taken in one step
+constexpr int kOccCap = kIndexSlots + kNewCap;
+
+struct IndexView {
+    int32_t* ilen;     // [B]
+    int32_t* flags;    // [B], build scratch
+    int32_t* counts;   // [B][V]
+    int32_t* slots;    // [B][V][kIndexSlots]
+    int V;
+};
+
+struct IndexShared {
+    int32_t occ[kOccCap];          // occurrences of x_t, ascending
+    int32_t occ_m[kOccCap];        // their suffix-match lengths
+    int32_t cand[kOccCap];         // the candidates (match length >= n*), ascending
+    int32_t newtok[kNewCap];       // ids of positions il .. t-1
+    int32_t suf[PLDP_MAX_NGRAM];   // x_t, x_{t-1}, ...
+    int32_t slot[kIndexSlots];
+    int count_old, nocc, ncand, nstar, bad_token, wmax[kWarps];
+};
+
+// Appends position q (token tok) to sequence b's index.
+__device__ __forceinline__ bool index_insert(const IndexView& ix, int b, int64_t q, int32_t tok) {
+    if (tok < 0 || tok >= ix.V) return false;
+    const int64_t e = static_cast<int64_t>(b) * ix.V + tok;
+    const int c = atomicAdd(ix.counts + e, 1);
+    if (c < kIndexSlots) ix.slots[e * kIndexSlots + c] = static_cast<int32_t>(q);
+    return true;
+}
+
+template <typename TH, bool IVEC>
+__global__ void __launch_bounds__(kThreads) draft_index_kernel(const DraftParams p, const IndexView ix) {
+    constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
+    __shared__ StepShared sh;
+    __shared__ IndexShared is;
+    pdl_enter();
+    const int b = blockIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int64_t L = p.seq_len[b];
+    const int64_t il = ix.ilen[b];
+    const bool valid = L >= 0 && L <= p.T_cap;
+    const int64_t t = L - 1;
+    const int32_t* row = p.ids + static_cast<int64_t>(b) * p.ids_stride;
+    const bool has_a = p.A != nullptr;
+    const size_t h_es = p.h_bf16 ? 2 : 4;
+    bool bad = false;                                             // a selected row outside [0, R)
+    if (has_a && valid && p.row_idx)
+        for (int k = tid; k < p.n_sel; k += kThreads) {
+            const int r = __ldg(p.row_idx + k);
+            bad |= r < 0 || r >= p.R;
+        }
+    if (tid <= PLDP_MAX_NGRAM) sh.ss.cnt[tid] = 0;
+    if (tid == 0) is.bad_token = 0;
+    bad = __syncthreads_or(bad) != 0;
+    if (!valid) {
+        for (int i = tid; i < p.K; i += kThreads) p.draft[static_cast<int64_t>(b) * p.K + i] = -1;
+        if (tid == 0) {
+            p.cand_count[b] = 0;
+            p.match_len[b] = 0;
+            if (HAS_H) {
+                p.best_h[b] = -1;
+                if (p.best_h_score) p.best_h_score[b] = -INFINITY;
+            }
+            if (has_a) {
+                p.best_a[b] = -1;
+                if (p.best_a_score) p.best_a_score[b] = -INFINITY;
+            }
+            p.draft_len[b] = 0;
+            if (p.status) atomicOr(p.status + b, PLDP_ST_SEQ_LEN);
+        }
+        return;
+    }
+    // usable: the index covers a prefix of the context; small: what was appended fits the CTA
+    const bool usable = il >= 0 && il <= t;
+    const int64_t nnew = usable ? t - il : 0;
+    const bool small = usable && nnew <= kNewCap;
+    if (tid == 0 && HAS_H && t >= 2)                              // H_{t-1}: every candidate's score reads it
+        prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (t - 1) * p.d) * h_es,
+                         static_cast<uint32_t>(p.d * h_es));
+    if (small && tid < nnew) is.newtok[tid] = __ldg(row + il + tid);
+    if (tid < PLDP_MAX_NGRAM) is.suf[tid] = (tid < p.ngram_max && t - tid >= 0) ? __ldg(row + t - tid) : 0;
+    __syncthreads();
+    const int32_t xt = is.suf[0];
+    bool indexed = small && t >= 1 && xt >= 0 && xt < ix.V;
+    if (indexed) {
+        const int64_t e = static_cast<int64_t>(b) * ix.V + xt;
+        if (tid == 0) is.count_old = __ldcg(ix.counts + e);
+        if (tid < kIndexSlots) is.slot[tid] = __ldcg(ix.slots + e * kIndexSlots + tid);
+    }
+    __syncthreads();
+    // append positions il .. t-1 (after x_t's entry was read; the answers are not waited for)
+    if (usable) {
+        bool badtok = false;
+        if (small) {
+            if (tid < nnew) badtok = !index_insert(ix, b, il + tid, is.newtok[tid]);
+        } else {
+            for (int64_t q = il + tid; q < t; q += kThreads) badtok |= !index_insert(ix, b, q, __ldg(row + q));
+        }
+        if (badtok) atomicOr(&is.bad_token, 1);
+    }
+    if (indexed && is.count_old > kIndexSlots) indexed = false;   // the slots do not hold them all
+
+    int32_t* cand_row = p.cand_pos + static_cast<int64_t>(b) * p.C_cap;
+    float* hsc = (HAS_H && p.h_scores) ? p.h_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
+    float* asc = (has_a && p.a_scores) ? p.a_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
+    unsigned long long hk = 0, ak = 0;
+    int nstar = 0, total = 0;
+    if (indexed) {
+        // the occurrences, ascending: the indexed ones (all before il) ranked, then the appended ones
+        if (warp == 0) {
+            const int nold = is.count_old;
+            if (lane < nold) {
+                const int32_t v = is.slot[lane];
+                int rank = 0;
+                for (int k = 0; k < nold; ++k) rank += is.slot[k] < v ? 1 : 0;
+                is.occ[rank] = v;
+            }
+            int base = nold;
+            for (int c0 = 0; c0 < nnew; c0 += 32) {
+                const bool hit = c0 + lane < nnew && is.newtok[c0 + lane] == xt;
+                const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
+                if (hit) is.occ[base + __popc(bal & ((1u << lane) - 1u))] = static_cast<int32_t>(il + c0 + lane);
+                base += __popc(bal);
+            }
+            if (lane == 0) is.nocc = base;
+        }
+        __syncthreads();
+        const int nocc = is.nocc;
+        // suffix-match lengths; the rows the ranking will read start towards L2
+        int mloc = 0;
+        for (int i = tid; i < nocc; i += kThreads) {
+            const int64_t j = is.occ[i];
+            if (HAS_H && j >= 1)
+                prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (j - 1) * p.d) * h_es,
+                                 static_cast<uint32_t>(p.d * h_es));
+            int m = 1;
+            while (m < p.ngram_max && j - m >= 0) {
+                const int64_t q = j - m;
+                const int32_t v = q >= il ? is.newtok[q - il] : __ldg(row + q);
+                if (v != is.suf[m]) break;
+                ++m;
+            }
+            is.occ_m[i] = m;
+            mloc = m > mloc ? m : mloc;
+        }
+        if (has_a) {                                             // the attention values of every occurrence
+            const size_t es = p.a_bf16 ? 2 : 4;
+            const char* ab = static_cast<const char*>(p.A) + static_cast<int64_t>(b) * p.a_seq_stride * es;
+            for (int i = 0; i < nocc; ++i) {
+                const int64_t j = is.occ[i];
+                for (int k = tid; k < p.n_sel; k += kThreads) {
+                    const int r = p.row_idx ? __ldg(p.row_idx + k) : k;
+                    if (r >= 0 && r < p.R)
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(ab + (static_cast<int64_t>(r) * p.a_row_stride + j) * es));
+                }
+            }
+        }
+        mloc = __reduce_max_sync(0xFFFFFFFFu, mloc);
+        if (lane == 0) is.wmax[warp] = mloc;
+        __syncthreads();
+        if (warp == 0) {
+            int mx = 0;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) mx = is.wmax[w] > mx ? is.wmax[w] : mx;
+            const int ns = mx >= p.ngram_min ? mx : 0;           // m <= ngram_max already
+            int base = 0;
+            if (ns > 0)
+                for (int c0 = 0; c0 < nocc; c0 += 32) {
+                    const bool c = c0 + lane < nocc && is.occ_m[c0 + lane] >= ns;
+                    const unsigned bal = __ballot_sync(0xFFFFFFFFu, c);
+                    if (c) {
+                        const int r = base + __popc(bal & ((1u << lane) - 1u));
+                        is.cand[r] = is.occ[c0 + lane];
+                        if (r < p.C_cap) cand_row[r] = is.occ[c0 + lane];
+                    }
+                    base += __popc(bal);
+                }
+            if (lane == 0) {
+                is.nstar = ns;
+                is.ncand = base;
+            }
+        }
+        __syncthreads();
+        nstar = is.nstar;
+        total = is.ncand;
+        const int n = total < p.C_cap ? total : p.C_cap;
+        constexpr int NB = kMaxScoreBatch;
+        for (int i0 = 0; i0 < n; i0 += NB) {
+            const int nb = n - i0 < NB ? n - i0 : NB;
+            int64_t j[NB];
+#pragma unroll
+            for (int h = 0; h < NB; ++h) j[h] = h < nb ? is.cand[i0 + h] : -1;
+            float s_h[NB], s_a[NB];
+            cta_score<TH, NB>(p, b, j, nb, t, part_buf<NB>(sh.part[(i0 / NB) & 1]), s_h, s_a);
+            if (tid == 0)
+                for (int h = 0; h < nb; ++h) {
+                    const int i = i0 + h;
+                    if (HAS_H) {
+                        if (hsc) hsc[i] = s_h[h];
+                        if (j[h] >= 1 && s_h[h] > p.threshold) {
+                            const unsigned long long key = pack_key(s_h[h], static_cast<uint32_t>(j[h]));
+                            hk = key > hk ? key : hk;
+                        }
+                    }
+                    if (has_a) {
+                        if (asc) asc[i] = s_a[h];
+                        const unsigned long long key = pack_key(s_a[h], static_cast<uint32_t>(j[h]));
+                        ak = key > ak ? key : ak;
+                    }
+                }
+        }
+    } else {
+        finish_overflow<TH, IVEC>(p, b, t, row, cand_row, hsc, asc, sh, hk, ak, nstar, total);
+    }
+
+    // ---- best of each ranking, then the draft (Sec. 4.3) ----------------------------------
+    hk = warp_max_u64(hk);
+    ak = warp_max_u64(ak);
+    if (lane == 0) {
+        sh.wkey[0][warp] = hk;
+        sh.wkey[1][warp] = ak;
+    }
+    __syncthreads();
+    if (warp != 0) return;
+    hk = 0;
+    ak = 0;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+        hk = sh.wkey[0][w] > hk ? sh.wkey[0][w] : hk;
+        ak = sh.wkey[1][w] > ak ? sh.wkey[1][w] : ak;
+    }
+    const int32_t bh = hk == 0 ? -1 : static_cast<int32_t>(key_index(hk));
+    const int32_t ba = ak == 0 ? -1 : static_cast<int32_t>(key_index(ak));
+    const int64_t js = p.draft_from == 0 ? bh : ba;
+    int64_t dl = 0;
+    if (js >= 0 && js < t) dl = (t - js < p.K) ? (t - js) : p.K;
+    for (int i = lane; i < p.K; i += 32)
+        p.draft[static_cast<int64_t>(b) * p.K + i] = (i < dl) ? __ldg(row + js + 1 + i) : -1;
+    if (lane == 0) {
+        p.cand_count[b] = total;
+        p.match_len[b] = nstar;
+        if (HAS_H) {
+            p.best_h[b] = bh;
+            if (p.best_h_score) p.best_h_score[b] = bh >= 0 ? key_value(hk) : -INFINITY;
+        }
+        if (has_a) {
+            p.best_a[b] = ba;
+            if (p.best_a_score) p.best_a_score[b] = ba >= 0 ? key_value(ak) : -INFINITY;
+        }
+        p.draft_len[b] = static_cast<int32_t>(dl);
+        if (p.status && total > p.C_cap) atomicOr(p.status + b, PLDP_ST_CAND_OVERFLOW);
+        if (p.status && bad) atomicOr(p.status + b, PLDP_ST_ROW_INDEX);
+        // the index now covers 0 .. t-1 (or is unusable: a token it cannot hold, or stale)
+        if (usable) ix.ilen[b] = is.bad_token ? -1 : static_cast<int32_t>(t);
+        else if (il > t) ix.ilen[b] = -1;
+    }
+}
+
+// Index build: positions 0 .. seq_len-2 of every sequence.
+__global__ void __launch_bounds__(kThreads) index_build_kernel(const int32_t* __restrict__ ids, int64_t ids_stride,
+                                                               const int32_t* __restrict__ seq_len, int64_t T_cap,
+                                                               IndexView ix) {
+    pdl_enter();
+    const int b = blockIdx.y;
+    const int64_t L = seq_len[b];
+    if (L < 0 || L > T_cap) return;
+    const int64_t t = L - 1;
+    const int32_t* row = ids + static_cast<int64_t>(b) * ids_stride;
+    for (int64_t q = static_cast<int64_t>(blockIdx.x) * kThreads + threadIdx.x; q < t;
+         q += static_cast<int64_t>(gridDim.x) * kThreads)
+        if (!index_insert(ix, b, q, __ldg(row + q))) atomicOr(ix.flags + b, 1);
+}
+
+__global__ void index_finish_kernel(const int32_t* __restrict__ seq_len, int B, int64_t T_cap, IndexView ix,
+                                    uint32_t* __restrict__ status) {
+    pdl_enter();
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= B) return;
+    const int64_t L = seq_len[b];
+    if (L < 0 || L > T_cap) {
+        ix.ilen[b] = -1;
+        if (status) atomicOr(status + b, PLDP_ST_SEQ_LEN);
+        return;
+    }
+    const bool bad_token = ix.flags[b] != 0;
+    ix.ilen[b] = bad_token ? -1 : static_cast<int32_t>(L >= 1 ? L - 1 : 0);
+    if (bad_token && status) atomicOr(status + b, PLDP_ST_TOKEN_RANGE);
+}
+
+// Byte offsets of the index parts (ilen, flags, counts, slots), 256-byte aligned.
+struct IndexLayout {
+    size_t ilen, flags, counts, slots, total;
+};
+inline IndexLayout index_layout(int B, int V) {
+    auto up = [](size_t x) { return (x + 255) / 256 * 256; };
+    IndexLayout l;
+    l.ilen = 0;
+    l.flags = up(static_cast<size_t>(B) * 4);
+    l.counts = l.flags + up(static_cast<size_t>(B) * 4);
+    l.slots = l.counts + up(static_cast<size_t>(B) * V * 4);
+    l.total = l.slots + up(static_cast<size_t>(B) * V * kIndexSlots * 4);
+    return l;
+}
+inline IndexView index_view(void* base, int B, int V) {
+    const IndexLayout l = index_layout(B, V);
+    char* c = static_cast<char*>(base);
+    return IndexView{reinterpret_cast<int32_t*>(c + l.ilen), reinterpret_cast<int32_t*>(c + l.flags),
+                     reinterpret_cast<int32_t*>(c + l.counts), reinterpret_cast<int32_t*>(c + l.slots), V};
+}
+
 template <typename TH, bool IVEC>
 pldp_status launch_t(const DraftParams& p, int B, cudaStream_t s) {
     int64_t chunks = (p.T_cap + kChunk - 1) / kChunk;
@@ -545,8 +877,17 @@ pldp_status launch_t(const DraftParams& p, int B, cudaStream_t s) {
     return PLDP_OK;
 }
 
+template <typename TH, bool IVEC>
+pldp_status launch_index_t(const DraftParams& p, const IndexView& ix, int B, cudaStream_t s) {
+    cudaError_t e = launch_pdl(draft_index_kernel<TH, IVEC>, dim3(static_cast<unsigned>(B)), dim3(kThreads), 0, s, 0,
+                               p, ix);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "draft_step (indexed): launch failed: %s", cudaGetErrorString(e));
+    return PLDP_OK;
+}
+
 template <typename TH>
-pldp_status launch_draft_step(const DraftParams& p, int B, cudaStream_t s, bool ivec) {
+pldp_status launch_draft_step(const DraftParams& p, int B, cudaStream_t s, bool ivec, const IndexView* ix) {
+    if (ix) return ivec ? launch_index_t<TH, true>(p, *ix, B, s) : launch_index_t<TH, false>(p, *ix, B, s);
     return ivec ? launch_t<TH, true>(p, B, s) : launch_t<TH, false>(p, B, s);
 }
 
@@ -608,9 +949,19 @@ extern "C" PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* a, v
     if (!a->ids || !a->seq_len || !a->cand_count || !a->match_len || !a->draft || !a->draft_len ||
         (a->C_cap > 0 && !a->cand_pos) || (a->H && !a->best_h) || (a->A && !a->best_a))
         return fail(PLDP_ERR_INVALID_ARG, "draft_step: null pointer");
-    if (!a->workspace || a->workspace_bytes < pldp_draft_workspace_size(B) || !aligned16(a->workspace))
+    IndexView ixv = {};
+    const IndexView* ix = nullptr;
+    if (a->index) {
+        if (a->V < 1) return fail(PLDP_ERR_INVALID_ARG, "draft_step: V < 1 with an index");
+        const size_t need = index_layout(B, a->V).total;
+        if (a->index_bytes < need || !aligned16(a->index))
+            return fail(PLDP_ERR_INVALID_ARG, "draft_step: index needs %zu bytes, 16-byte aligned", need);
+        ixv = index_view(a->index, B, a->V);
+        ix = &ixv;
+    } else if (!a->workspace || a->workspace_bytes < pldp_draft_workspace_size(B) || !aligned16(a->workspace)) {
         return fail(PLDP_ERR_INVALID_ARG, "draft_step: workspace needs %zu bytes, 16-byte aligned",
                     pldp_draft_workspace_size(B));
+    }
     if (a->H && !(aligned16(a->H) && qbytes % 16 == 0 && (a->h_seq_stride * h_es) % 16 == 0))
         return fail(PLDP_ERR_UNSUPPORTED,
                     "draft_step: hidden rows must be 16-byte aligned (the separate calls accept any layout)");
@@ -653,7 +1004,41 @@ extern "C" PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* a, v
     p.ws = static_cast<unsigned char*>(a->workspace);
     const bool ivec = aligned16(a->ids) && a->ids_stride % 4 == 0 && a->T_cap % 4 == 0;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (!a->H) return launch_draft_step<NoHidden>(p, B, s, ivec);
-    if (a->h_dtype == PLDP_BF16) return launch_draft_step<__nv_bfloat16>(p, B, s, ivec);
-    return launch_draft_step<float>(p, B, s, ivec);
+    if (!a->H) return launch_draft_step<NoHidden>(p, B, s, ivec, ix);
+    if (a->h_dtype == PLDP_BF16) return launch_draft_step<__nv_bfloat16>(p, B, s, ivec, ix);
+    return launch_draft_step<float>(p, B, s, ivec, ix);
+}
+
+extern "C" PLDP_API size_t pldp_index_size(int B, int V) {
+    if (B < 0 || V < 1) return 0;
+    return index_layout(B, V).total;
+}
+
+extern "C" PLDP_API pldp_status pldp_index_build(const int32_t* ids, int64_t ids_stride, const int32_t* seq_len,
+                                                 int B, int64_t T_cap, int V, void* index, size_t index_bytes,
+                                                 uint32_t* status, void* stream) {
+    if (B < 0) return fail(PLDP_ERR_INVALID_ARG, "index_build: B < 0");
+    if (B > 65535) return fail(PLDP_ERR_UNSUPPORTED, "index_build: B > 65535");
+    if (V < 1) return fail(PLDP_ERR_INVALID_ARG, "index_build: V < 1");
+    if (T_cap < 0 || T_cap > kMaxPositions) return fail(PLDP_ERR_INVALID_ARG, "index_build: T_cap outside [0, 2^27]");
+    if (ids_stride < T_cap) return fail(PLDP_ERR_INVALID_ARG, "index_build: ids_stride < T_cap");
+    if (B == 0) return PLDP_OK;
+    if (!ids || !seq_len || !index) return fail(PLDP_ERR_INVALID_ARG, "index_build: null pointer");
+    const size_t need = index_layout(B, V).total;
+    if (index_bytes < need || !aligned16(index))
+        return fail(PLDP_ERR_INVALID_ARG, "index_build: index needs %zu bytes, 16-byte aligned", need);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemsetAsync(index, 0, need, s);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "index_build: clearing the index: %s", cudaGetErrorString(e));
+    const IndexView ix = index_view(index, B, V);
+    int64_t chunks = (T_cap + 8191) / 8192;
+    if (chunks < 1) chunks = 1;
+    if (chunks > 65535) chunks = 65535;
+    e = launch_pdl(index_build_kernel, dim3(static_cast<unsigned>(chunks), static_cast<unsigned>(B)), dim3(kThreads), 0,
+                   s, 0, ids, ids_stride, seq_len, T_cap, ix);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "index_build: launch failed: %s", cudaGetErrorString(e));
+    e = launch_pdl(index_finish_kernel, dim3(static_cast<unsigned>((B + 255) / 256)), dim3(256), 0, s, 0, seq_len, B,
+                   T_cap, ix, status);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "index_build: launch failed: %s", cudaGetErrorString(e));
+    return PLDP_OK;
 }

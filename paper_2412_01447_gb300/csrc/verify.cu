@@ -206,10 +206,14 @@ __device__ __forceinline__ unsigned long long pack_ordered(uint32_t okey, uint32
 // the lane(s) holding it search for the element; a second redux picks the
 // smallest index.  A segment that crosses into row r0 + 1 keeps a running
 // (max, first index) per row and lane.
+struct SegKeys {
+    unsigned long long k0;   // the segment's best in its first row
+    unsigned long long k1;   // ... in the next row when the segment crosses into it, else 0
+};
+
 template <typename T>
-__device__ __forceinline__ void segment_argmax(const uint4* __restrict__ p, uint32_t s0, uint32_t nvec,
-                                               uint32_t r0, uint32_t rem, uint32_t vrow, int lane,
-                                               unsigned long long* __restrict__ keys) {
+__device__ __forceinline__ SegKeys segment_argmax(const uint4* __restrict__ p, uint32_t s0, uint32_t nvec,
+                                                  uint32_t r0, uint32_t rem, uint32_t vrow, int lane) {
     constexpr uint32_t VW = 16 / sizeof(T);
     constexpr uint32_t seg = 32 * kSegLoads;
     uint4 x[kSegLoads];
@@ -232,8 +236,7 @@ __device__ __forceinline__ void segment_argmax(const uint4* __restrict__ p, uint
                     idx = (rem + lane + 32 * u) * VW + vfirst(x[u], m, T());
         }
         idx = __reduce_min_sync(0xFFFFFFFFu, idx);
-        if (lane == 0) atomicMax(keys + r0, pack_ordered(wk, idx));
-        return;
+        return SegKeys{pack_ordered(wk, idx), 0ull};
     }
     const uint32_t bnd = s0 - rem + vrow;                      // first vector of row r0 + 1
     float b0 = -INFINITY, b1 = -INFINITY;
@@ -255,11 +258,9 @@ __device__ __forceinline__ void segment_argmax(const uint4* __restrict__ p, uint
         }
     }
     const unsigned long long k0 = warp_max_u64(pack_key(b0, i0));
-    if (lane == 0) atomicMax(keys + r0, k0);
-    if (s0 + seg > bnd && bnd < nvec) {
-        const unsigned long long k1 = warp_max_u64(pack_key(b1, i1));
-        if (lane == 0) atomicMax(keys + r0 + 1, k1);
-    }
+    unsigned long long k1 = 0ull;
+    if (s0 + seg > bnd && bnd < nvec) k1 = warp_max_u64(pack_key(b1, i1));
+    return SegKeys{k0, k1};
 }
 
 // Any segment: row by row, each row piece with the lane loop above.
@@ -290,6 +291,13 @@ verify_argmax_kernel(const T* __restrict__ logits, int64_t N, int64_t V, int64_t
     const int lane = threadIdx.x & 31;
     const int64_t w = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);
     if constexpr (PATH == 0) {
+        // Per round the CTA's warps hold 8 consecutive segments (16 KB, rarely more
+        // than one row): their keys meet in shared memory and thread 0 issues one
+        // atomicMax per row touched.  Rounds are counted from the CTA's first warp,
+        // so every warp takes part in every round (with no segment past the end).
+        __shared__ unsigned long long sk[2][kWarps][2];
+        __shared__ uint32_t srow[2][kWarps];
+        const int warp = threadIdx.x >> 5;
         constexpr uint32_t VW = 16 / sizeof(T);
         constexpr uint32_t seg = 32 * kSegLoads;
         const uint32_t nvec = static_cast<uint32_t>(N / VW), vrow = static_cast<uint32_t>(V / VW);
@@ -298,8 +306,38 @@ verify_argmax_kernel(const T* __restrict__ logits, int64_t N, int64_t V, int64_t
         const uint32_t dq = stride / vrow, dr = stride - dq * vrow;      // rows and vectors per stride
         uint32_t s0 = static_cast<uint32_t>(w) * seg;
         uint32_t r0 = s0 / vrow, rem = s0 - r0 * vrow;
-        for (; s0 < nvec; s0 += stride) {
-            segment_argmax<T>(p, s0, nvec, r0, rem, vrow, lane, keys);
+        uint32_t first = blockIdx.x * kWarps * seg;                       // the CTA's first segment
+        for (int buf = 0; first < nvec; first += stride, buf ^= 1) {
+            const bool mine = s0 < nvec;
+            SegKeys k = {0ull, 0ull};
+            if (mine) k = segment_argmax<T>(p, s0, nvec, r0, rem, vrow, lane);
+            if (lane == 0) {
+                srow[buf][warp] = mine ? r0 : 0xFFFFFFFFu;
+                sk[buf][warp][0] = k.k0;
+                sk[buf][warp][1] = k.k1;
+            }
+            __syncthreads();
+            if (threadIdx.x == 0) {                                       // rows are nondecreasing here
+                uint32_t cur = 0xFFFFFFFFu;
+                unsigned long long best = 0ull;
+                for (int q = 0; q < kWarps; ++q) {
+                    const uint32_t r = srow[buf][q];
+                    if (r == 0xFFFFFFFFu) continue;
+                    if (r != cur) {
+                        if (cur != 0xFFFFFFFFu) atomicMax(keys + cur, best);
+                        cur = r;
+                        best = 0ull;
+                    }
+                    best = sk[buf][q][0] > best ? sk[buf][q][0] : best;
+                    if (sk[buf][q][1]) {                                  // it crosses into row r + 1
+                        atomicMax(keys + cur, best);
+                        cur = r + 1;
+                        best = sk[buf][q][1];
+                    }
+                }
+                if (cur != 0xFFFFFFFFu) atomicMax(keys + cur, best);
+            }
+            s0 += stride;
             r0 += dq;
             rem += dr;
             if (rem >= vrow) {
