@@ -43,6 +43,7 @@ constexpr size_t kSeqWs = 16 + kHitCap * 16;                   // header + 16-by
 constexpr int kScoreUnroll = 2;                                // 16-byte row loads in flight
 constexpr int kScoreBatch = 2;                                 // occurrences scored per pass (scan kernel)
 constexpr int kMaxScoreBatch = 4;                              // ... and at most (the indexed kernel)
+constexpr int kSpeculate = kMaxScoreBatch;                     // occurrences scored before their suffix match
 constexpr size_t kMaxQueryBytes = 196608;
 constexpr int kMaxSelRows = 8192;
 constexpr int64_t kMaxPositions = int64_t(1) << 27;            // (j << 4) | m fits 31 bits
@@ -101,15 +102,41 @@ __device__ __forceinline__ void prefetch_l2_bulk(const void* ptr, uint32_t bytes
     asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
 }
 
-__device__ __forceinline__ float warp_max_f(float v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
-    return v;
-}
-
 struct Hit {
     int32_t j, m;
 };
+
+// Warp reduce-scatter of N values (N a power of two, <= 32): at each butterfly
+// level a lane keeps half of its values and trades the other half with its
+// partner, so the N totals take N - 1 + 5 - log2(N) shuffles instead of 5 N.
+// Returns the total (sum, or max when use_max) of value lane >> (5 - log2 N).
+// Every total is formed in one fixed order, the same in every lane holding it.
+template <int N>
+__device__ __forceinline__ float warp_reduce_scatter(float (&v)[N], bool use_max) {
+    static_assert(N >= 1 && N <= 32 && (N & (N - 1)) == 0, "N: a power of two up to 32");
+    constexpr int LOG2N = N >= 32 ? 5 : N >= 16 ? 4 : N >= 8 ? 3 : N >= 4 ? 2 : N >= 2 ? 1 : 0;
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int s = 0; s < LOG2N; ++s) {
+        const int n = N >> s, o = 16 >> s;
+        const bool upper = (lane & o) != 0;
+#pragma unroll
+        for (int i = 0; i < N / 2; ++i) {
+            if (i >= n / 2) continue;
+            const float keep = upper ? v[i + n / 2] : v[i];
+            const float send = upper ? v[i] : v[i + n / 2];
+            const float got = __shfl_xor_sync(0xFFFFFFFFu, send, o);
+            v[i] = use_max ? fmaxf(keep, got) : keep + got;
+        }
+    }
+    float r = v[0];
+#pragma unroll
+    for (int o = 16 >> LOG2N; o > 0; o >>= 1) {
+        const float got = __shfl_xor_sync(0xFFFFFFFFu, r, o);
+        r = use_max ? fmaxf(r, got) : r + got;
+    }
+    return r;
+}
 
 template <int NB>
 __device__ __forceinline__ float (&part_buf(float (&part)[kMaxScoreBatch][kWarps][4]))[NB][kWarps][4] {
@@ -118,7 +145,7 @@ __device__ __forceinline__ float (&part_buf(float (&part)[kMaxScoreBatch][kWarps
 
 struct StepShared {
     Hit hit[kHitCap];                        // occurrences this CTA found (the first kHitCap)
-    float part[2][kMaxScoreBatch][kWarps][4];   // per-warp partial sums: dot, |a|^2, |q|^2, attention
+    alignas(16) float part[2][kMaxScoreBatch][kWarps][4];   // per-warp partials: dot, |a|^2, |q|^2, attention
     int32_t jl[kHitCap];                     // finish: positions of the candidates (else INT_MAX)
     unsigned long long wkey[2][kWarps];      // finish: per-warp best keys (hidden, attention)
     int wmax[kWarps];
@@ -127,14 +154,16 @@ struct StepShared {
     ScanShared ss;                           // finish: the ordered rescan of an overflowed list
 };
 
-// Eq. 3 and Eq. 2 for candidates j[0 .. nb) of sequence b (nb <= kScoreBatch),
-// by all threads of the CTA: thread i takes 16-byte chunks i, i + 256, ... of
-// H_{j-1} and H_{t-1} and selected rows i, i + 256, ...; partial sums meet in
-// `part` and thread 0 combines them in warp order.  The candidates of one pass
-// share the loads of H_{t-1} and are otherwise independent: a score does not
-// depend on which pass or slot computes it.  Scores are returned in thread 0:
-// the cosine (-inf when j = 0 has no H_{j-1}) and the attention max / sum.
-// CTA-uniform call with one barrier; callers alternate `part` buffers.
+// Eq. 3 and Eq. 2 for candidates j[0 .. nb) of sequence b (nb <= NB), by all
+// threads of the CTA: thread i takes 16-byte chunks i, i + 256, ... of H_{j-1}
+// and H_{t-1} and selected rows i, i + 256, ...; partial sums meet in `part`
+// and are combined in warp order.  The candidates of one pass share the loads of
+// H_{t-1} and are otherwise independent: a score does not depend on which pass
+// or slot computes it.  The attention values of each thread's first selected row
+// are loaded before the hidden rows are used, so both arrive in one round trip.
+// Scores are returned in thread 0: the cosine (-inf when j = 0 has no H_{j-1})
+// and the attention max / sum.  CTA-uniform call with one barrier; callers
+// alternate `part` buffers.
 template <typename TH, int NB>
 __device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int64_t (&j)[NB], int nb, int64_t t,
                                           float (&part)[NB][kWarps][4], float (&s_h)[NB], float (&s_a)[NB]) {
@@ -155,6 +184,16 @@ __device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int
         dot[h] = 0.f;
         na[h] = 0.f;
         acc[h] = is_max ? -INFINITY : 0.0f;
+    }
+    const size_t a_es = p.a_bf16 ? 2 : 4;
+    const void* ab = p.A ? static_cast<const char*>(p.A) + static_cast<int64_t>(b) * p.a_seq_stride * a_es : nullptr;
+    float av[NB];                                                 // selected row `tid`, in flight with H
+    {
+        const int r = (p.A != nullptr && tid < p.n_sel) ? (p.row_idx ? __ldg(p.row_idx + tid) : tid) : -1;
+        const bool rv = r >= 0 && r < p.R;
+#pragma unroll
+        for (int h = 0; h < NB; ++h)
+            av[h] = (rv && a_ok[h]) ? load_attn(ab, static_cast<int64_t>(r) * p.a_row_stride + j[h], p.a_bf16) : NAN;
     }
     if constexpr (HAS_H) {
         if (any_h) {
@@ -192,9 +231,10 @@ __device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int
         }
     }
     if (p.A != nullptr) {
-        const size_t es = p.a_bf16 ? 2 : 4;
-        const void* ab = static_cast<const char*>(p.A) + static_cast<int64_t>(b) * p.a_seq_stride * es;
-        for (int k = tid; k < p.n_sel; k += kThreads) {
+#pragma unroll
+        for (int h = 0; h < NB; ++h)
+            if (av[h] == av[h]) acc[h] = is_max ? fmaxf(acc[h], av[h]) : acc[h] + av[h];
+        for (int k = tid + kThreads; k < p.n_sel; k += kThreads) {
             const int r = p.row_idx ? __ldg(p.row_idx + k) : k;
             const bool rv = r >= 0 && r < p.R;
             float v[NB];
@@ -206,44 +246,68 @@ __device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int
                 if (v[h] == v[h]) acc[h] = is_max ? fmaxf(acc[h], v[h]) : acc[h] + v[h];
         }
     }
-    if constexpr (HAS_H) nq = warp_sum(nq);
-#pragma unroll
-    for (int h = 0; h < NB; ++h) {
-        if constexpr (HAS_H) {
-            dot[h] = warp_sum(dot[h]);
-            na[h] = warp_sum(na[h]);
-        }
-        acc[h] = is_max ? warp_max_f(acc[h]) : warp_sum(acc[h]);
-        if (lane == 0) {
-            part[h][warp][0] = dot[h];
-            part[h][warp][1] = na[h];
-            part[h][warp][2] = nq;
-            part[h][warp][3] = acc[h];
-        }
-    }
-    __syncthreads();
-    if (tid == 0) {
+    // warp totals by reduce-scatter: lane l ends with one of them
+    if constexpr (HAS_H) {
+        float w[2 * NB];                                          // dot products, then |H_{j-1}|^2
 #pragma unroll
         for (int h = 0; h < NB; ++h) {
-            float D = 0.f, N = 0.f, Q = 0.f, S = part[h][0][3];
+            w[h] = dot[h];
+            w[NB + h] = na[h];
+        }
+        const float tw = warp_reduce_scatter<2 * NB>(w, false);
+        constexpr int SW = 32 / (2 * NB);                         // lanes holding each total
+        const int iw = lane / SW;
+        if (lane % SW == 0) part[iw % NB][warp][iw < NB ? 0 : 1] = tw;
+        nq = warp_sum(nq);
+        if (lane < NB) part[lane][warp][2] = nq;
+    } else {
+        if (lane < NB) part[lane][warp][0] = part[lane][warp][1] = part[lane][warp][2] = 0.f;
+    }
+    {
+        const float ta = warp_reduce_scatter<NB>(acc, is_max);
+        constexpr int SA = 32 / NB;
+        if (lane % SA == 0) part[lane / SA][warp][3] = ta;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        // lane (h, w) = (lane / kWarps, lane % kWarps) takes warp w's partials of
+        // candidate h; the kWarps lanes of a candidate combine them in a fixed tree
+        static_assert(NB * kWarps <= 32, "a lane per (candidate, warp)");
+        const int h = lane / kWarps, w = lane % kWarps;
+        float4 v = make_float4(0.f, 0.f, 0.f, is_max ? -INFINITY : 0.f);
+        if (h < NB) v = *reinterpret_cast<const float4*>(&part[h][w][0]);
 #pragma unroll
-            for (int w = 0; w < kWarps; ++w) {
-                D += part[h][w][0];
-                N += part[h][w][1];
-                Q += part[h][w][2];
-                if (w > 0) S = is_max ? fmaxf(S, part[h][w][3]) : S + part[h][w][3];
+        for (int o = kWarps / 2; o > 0; o >>= 1) {
+            v.x += __shfl_xor_sync(0xFFFFFFFFu, v.x, o);
+            v.y += __shfl_xor_sync(0xFFFFFFFFu, v.y, o);
+            v.z += __shfl_xor_sync(0xFFFFFFFFu, v.z, o);
+            const float x = __shfl_xor_sync(0xFFFFFFFFu, v.w, o);
+            v.w = is_max ? fmaxf(v.w, x) : v.w + x;
+        }
+        bool hv = false, avl = false;
+#pragma unroll
+        for (int k = 0; k < NB; ++k)
+            if (k == h) {
+                hv = h_ok[k];
+                avl = a_ok[k];
             }
-            s_h[h] = h_ok[h] ? finish_cosine(D, N, Q) : -INFINITY;
-            s_a[h] = a_ok[h] ? S : -INFINITY;
+        const float sh_ = hv ? finish_cosine(v.x, v.y, v.z) : -INFINITY;
+        const float sa_ = avl ? v.w : -INFINITY;
+#pragma unroll
+        for (int k = 0; k < NB; ++k) {
+            s_h[k] = __shfl_sync(0xFFFFFFFFu, sh_, k * kWarps);
+            s_a[k] = __shfl_sync(0xFFFFFFFFu, sa_, k * kWarps);
         }
     }
 }
 
-// The finish of a sequence whose list overflowed (more than kHitCap occurrences):
-// an ordered rescan of the context writes the candidate list, then each
-// candidate is scored by cta_score.  Kept out of line: its registers do not
-// weigh on the common path.  CTA-uniform call; keys are left in thread 0.
-template <typename TH, bool IVEC>
+// The finish of a sequence whose occurrences were not gathered (an overflowed
+// list, or a token the index cannot answer for): an ordered rescan of the
+// context writes the candidate list, the candidates' hidden rows start towards
+// L2, then the candidates are scored by cta_score, NB per pass.  Kept out of
+// line: its registers do not weigh on the common path.  CTA-uniform call; keys
+// are left in thread 0.
+template <typename TH, bool IVEC, int NB>
 __device__ __noinline__ void finish_overflow(const DraftParams& p, int b, int64_t t, const int32_t* row,
                                              int32_t* cand_row, float* hsc, float* asc, StepShared& sh,
                                              unsigned long long& hk, unsigned long long& ak, int& nstar,
@@ -276,14 +340,22 @@ __device__ __noinline__ void finish_overflow(const DraftParams& p, int b, int64_
     scan_write<IVEC>(GlobalIds{row}, row, 0, t, t, p.ngram_max, sh.ss, cand_row, p.C_cap);
     __syncthreads();
     const int n = total < p.C_cap ? total : p.C_cap;
-    for (int i0 = 0; i0 < n; i0 += kScoreBatch) {
-        const int nb = n - i0 < kScoreBatch ? n - i0 : kScoreBatch;
-        int64_t j[kScoreBatch];
+    if (HAS_H && n > NB) {
+        const size_t h_es = p.h_bf16 ? 2 : 4;
+        for (int i = tid; i < n; i += kThreads) {
+            const int64_t j = __ldcg(cand_row + i);
+            if (j >= 1 && j < t)
+                prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (j - 1) * p.d) * h_es,
+                                 static_cast<uint32_t>(p.d * h_es));
+        }
+    }
+    for (int i0 = 0; i0 < n; i0 += NB) {
+        const int nb = n - i0 < NB ? n - i0 : NB;
+        int64_t j[NB];
 #pragma unroll
-        for (int h = 0; h < kScoreBatch; ++h) j[h] = h < nb ? __ldcg(cand_row + i0 + h) : -1;
-        float s_h[kScoreBatch], s_a[kScoreBatch];
-        cta_score<TH, kScoreBatch>(p, b, j, nb, t, part_buf<kScoreBatch>(sh.part[(i0 / kScoreBatch) & 1]), s_h,
-                                   s_a);
+        for (int h = 0; h < NB; ++h) j[h] = h < nb ? __ldcg(cand_row + i0 + h) : -1;
+        float s_h[NB], s_a[NB];
+        cta_score<TH, NB>(p, b, j, nb, t, part_buf<NB>(sh.part[(i0 / NB) & 1]), s_h, s_a);
         if (tid == 0)
             for (int h = 0; h < nb; ++h) {
                 const int i = i0 + h;
@@ -494,7 +566,7 @@ __global__ void __launch_bounds__(kThreads, 4) draft_step_kernel(const DraftPara
             }
         }
     } else {
-        finish_overflow<TH, IVEC>(p, b, t, row, cand_row, hsc, asc, sh, hk, ak, nstar, total);
+        finish_overflow<TH, IVEC, kScoreBatch>(p, b, t, row, cand_row, hsc, asc, sh, hk, ak, nstar, total);
     }
 
     // ---- best of each ranking, then the draft (Sec. 4.3) ----------------------------------
@@ -542,51 +614,77 @@ __global__ void __launch_bounds__(kThreads, 4) draft_step_kernel(const DraftPara
 // ---------------------------------------------------------------------------
 // The incremental token index: drafting without rescanning the context.
 //
-// Per sequence b and token v the index holds how often v occurs among the
-// indexed positions (counts) and up to kIndexSlots of those positions (slots,
-// in no particular order); ilen[b] is the number of positions indexed (0 ..
+// Per sequence b and token v the index holds one 32-byte entry: how often v
+// occurs among the indexed positions, then up to kIndexSlots of those positions
+// (in no particular order); ilen[b] is the number of positions indexed (0 ..
 // ilen-1), -1 when the index of b is unusable.  A step with t = seq_len - 1:
-//  * reads x_t's count and slots in one round trip; when the count is at most
-//    kIndexSlots the slots are every occurrence before ilen, and the positions
-//    appended since (ilen .. t-1, read anyway) supply the rest;
+//  * reads x_t's entry in one sector; when the count is at most kIndexSlots the
+//    slots are every occurrence before ilen, and the positions appended since
+//    (ilen .. t-1, read anyway) supply the rest;
 //  * otherwise (a frequent token, a stale or unusable index) falls back to the
 //    ordered rescan of the context, so results are those of the scan either way;
-//  * then appends positions ilen .. t-1 to the index and sets ilen = t.
-// Only the candidates (match length n*) are scored.  One CTA per sequence.
+//  * appends positions ilen .. t-1 to the index and sets ilen = t.  Each
+//    appended position takes its slot with an atomic on its token's count; the
+//    answer is used (the slot written) only at the end of the CTA, and tokens
+//    equal to x_t take theirs only after x_t's entry has been read.
+// With at most kSpeculate occurrences (most steps) every occurrence is scored
+// while its suffix-match length is found, in one round trip to memory: its
+// preceding tokens, the K tokens after it, H_{j-1} and the attention values at
+// j are loaded together, and n* then picks the candidates among the scored
+// occurrences.  With more, scoring all of them would cost more than it saves
+// (each needs a d-element row and R scattered attention values): the suffix
+// matches come first, then only the candidates are scored, with the tokens
+// after them read in the same round trip.  One CTA per sequence.
 // ---------------------------------------------------------------------------
-constexpr int kIndexSlots = 8;
+constexpr int kIndexSlots = 15;
+constexpr int kEntryWords = 1 + kIndexSlots;       // count, then the slots: 64 bytes, half a line
 constexpr int kNewCap = kThreads;                  // appended positions taken in one step
 constexpr int kOccCap = kIndexSlots + kNewCap;
+constexpr int kDraftWin = 32;                      // draft tokens staged per occurrence (a lane each)
+
+static_assert(kEntryWords * 4 == 64 && kEntryWords <= 32, "an entry is 64 bytes, a word per lane");
 
 struct IndexView {
-    int32_t* ilen;     // [B]
-    int32_t* flags;    // [B], build scratch
-    int32_t* counts;   // [B][V]
-    int32_t* slots;    // [B][V][kIndexSlots]
+    int32_t* ilen;      // [B]
+    int32_t* flags;     // [B], build scratch
+    int32_t* entries;   // [B][V][kEntryWords]
     int V;
 };
 
 struct IndexShared {
-    int32_t occ[kOccCap];          // occurrences of x_t, ascending
-    int32_t occ_m[kOccCap];        // their suffix-match lengths
-    int32_t cand[kOccCap];         // the candidates (match length >= n*), ascending
-    int32_t newtok[kNewCap];       // ids of positions il .. t-1
-    int32_t suf[PLDP_MAX_NGRAM];   // x_t, x_{t-1}, ...
-    int32_t slot[kIndexSlots];
-    int count_old, nocc, ncand, nstar, bad_token, wmax[kWarps];
+    int32_t occ[kOccCap];              // occurrences of x_t, ascending
+    int32_t occ_m[kOccCap];            // their suffix-match lengths
+    int32_t cand[kOccCap];             // the candidates (match length >= n*), ascending
+    int32_t newtok[kNewCap];           // ids of positions il .. t-1
+    int32_t occ_new[kNewCap];          // the appended occurrences, ascending
+    int32_t suf[PLDP_MAX_NGRAM];       // x_t, x_{t-1}, ...
+    int nocc, ncand, nstar, bad_token, indexed, wmax[kWarps];
 };
 
-// Appends position q (token tok) to sequence b's index.
+__device__ __forceinline__ int32_t* index_entry(const IndexView& ix, int b, int32_t tok) {
+    return ix.entries + (static_cast<int64_t>(b) * ix.V + tok) * kEntryWords;
+}
+
+// Counts one more occurrence of token tok in sequence b's index: returns the slot
+// it takes (the old count; >= kIndexSlots: none), or -1 for a token outside [0, V).
+__device__ __forceinline__ int index_take(const IndexView& ix, int b, int32_t tok) {
+    if (tok < 0 || tok >= ix.V) return -1;
+    return atomicAdd(index_entry(ix, b, tok), 1);
+}
+
+// Writes position q into the slot taken by index_take.
+__device__ __forceinline__ void index_put(const IndexView& ix, int b, int32_t tok, int slot, int64_t q) {
+    if (slot >= 0 && slot < kIndexSlots) index_entry(ix, b, tok)[1 + slot] = static_cast<int32_t>(q);
+}
+
 __device__ __forceinline__ bool index_insert(const IndexView& ix, int b, int64_t q, int32_t tok) {
-    if (tok < 0 || tok >= ix.V) return false;
-    const int64_t e = static_cast<int64_t>(b) * ix.V + tok;
-    const int c = atomicAdd(ix.counts + e, 1);
-    if (c < kIndexSlots) ix.slots[e * kIndexSlots + c] = static_cast<int32_t>(q);
-    return true;
+    const int slot = index_take(ix, b, tok);
+    index_put(ix, b, tok, slot, q);
+    return slot >= 0;
 }
 
 template <typename TH, bool IVEC>
-__global__ void __launch_bounds__(kThreads) draft_index_kernel(const DraftParams p, const IndexView ix) {
+__global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftParams p, const IndexView ix) {
     constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
     __shared__ StepShared sh;
     __shared__ IndexShared is;
@@ -638,79 +736,111 @@ __global__ void __launch_bounds__(kThreads) draft_index_kernel(const DraftParams
     if (tid < PLDP_MAX_NGRAM) is.suf[tid] = (tid < p.ngram_max && t - tid >= 0) ? __ldg(row + t - tid) : 0;
     __syncthreads();
     const int32_t xt = is.suf[0];
-    bool indexed = small && t >= 1 && xt >= 0 && xt < ix.V;
-    if (indexed) {
-        const int64_t e = static_cast<int64_t>(b) * ix.V + xt;
-        if (tid == 0) is.count_old = __ldcg(ix.counts + e);
-        if (tid < kIndexSlots) is.slot[tid] = __ldcg(ix.slots + e * kIndexSlots + tid);
-    }
-    __syncthreads();
-    // append positions il .. t-1 (after x_t's entry was read; the answers are not waited for)
-    if (usable) {
-        bool badtok = false;
-        if (small) {
-            if (tid < nnew) badtok = !index_insert(ix, b, il + tid, is.newtok[tid]);
-        } else {
-            for (int64_t q = il + tid; q < t; q += kThreads) badtok |= !index_insert(ix, b, q, __ldg(row + q));
+    const bool lookup = small && t >= 1 && xt >= 0 && xt < ix.V;
+    int32_t ev = 0;                                               // x_t's entry, word `lane` (warp 0)
+    if (lookup && tid < kEntryWords) ev = __ldcg(index_entry(ix, b, xt) + tid);
+    // this thread's appended position (small): its token and the slot it takes
+    const bool mine = small && tid < nnew;
+    const int32_t mytok = mine ? is.newtok[tid] : 0;
+    int myslot = -1;
+    if (mine && mytok != xt) myslot = index_take(ix, b, mytok);  // other entries: no wait for x_t's
+    if (mine && (mytok < 0 || mytok >= ix.V)) atomicOr(&is.bad_token, 1);
+    if (warp == 0 && lookup) {
+        // the appended occurrences (ascending) while the entry is on its way
+        int nn = 0;
+        for (int c0 = 0; c0 < nnew; c0 += 32) {
+            const bool hit = c0 + lane < nnew && is.newtok[c0 + lane] == xt;
+            const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
+            if (hit) is.occ_new[nn + __popc(bal & ((1u << lane) - 1u))] = static_cast<int32_t>(il + c0 + lane);
+            nn += __popc(bal);
         }
+        const int nold = __shfl_sync(0xFFFFFFFFu, ev, 0);
+        const bool ok = nold >= 0 && nold <= kIndexSlots;         // else the slots do not hold them all
+        if (ok) {
+            if (lane >= 1 && lane <= nold) {                      // the indexed ones (all before il), ranked
+                int rank = 0;
+                for (int k = 1; k <= nold; ++k) rank += __shfl_sync((1u << (nold + 1)) - 2u, ev, k) < ev ? 1 : 0;
+                is.occ[rank] = ev;
+            }
+            __syncwarp();
+            for (int k = lane; k < nn; k += 32) is.occ[nold + k] = is.occ_new[k];
+        }
+        if (lane == 0) {
+            is.indexed = ok;
+            is.nocc = ok ? nold + nn : 0;
+        }
+    }
+    __syncthreads();                                              // x_t's entry has been read
+    const bool indexed = lookup && is.indexed;
+    if (mine && mytok == xt) myslot = index_take(ix, b, mytok);
+    if (usable && !small) {                                       // a long append: inserted in turn
+        bool badtok = false;
+        for (int64_t q = il + tid; q < t; q += kThreads) badtok |= !index_insert(ix, b, q, __ldg(row + q));
         if (badtok) atomicOr(&is.bad_token, 1);
     }
-    if (indexed && is.count_old > kIndexSlots) indexed = false;   // the slots do not hold them all
 
     int32_t* cand_row = p.cand_pos + static_cast<int64_t>(b) * p.C_cap;
     float* hsc = (HAS_H && p.h_scores) ? p.h_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
     float* asc = (has_a && p.a_scores) ? p.a_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
+    const int nocc = indexed ? is.nocc : 0;
+
+    // Warp 0: the choices of both rankings (best keys hk, ak), the draft (Sec. 4.3)
+    // with draft_tok(i, j*) giving token j* + 1 + i, and the per-sequence outputs.
+    auto outputs = [&](unsigned long long hk, unsigned long long ak, int nstar, int total, auto draft_tok) {
+        const int32_t bh = hk == 0 ? -1 : static_cast<int32_t>(key_index(hk));
+        const int32_t ba = ak == 0 ? -1 : static_cast<int32_t>(key_index(ak));
+        const int64_t js = p.draft_from == 0 ? bh : ba;
+        int64_t dl = 0;
+        if (js >= 0 && js < t) dl = (t - js < p.K) ? (t - js) : p.K;
+        for (int i = lane; i < p.K; i += 32)
+            p.draft[static_cast<int64_t>(b) * p.K + i] = (i < dl) ? draft_tok(i, js) : -1;
+        if (lane == 0) {
+            p.cand_count[b] = total;
+            p.match_len[b] = nstar;
+            if (HAS_H) {
+                p.best_h[b] = bh;
+                if (p.best_h_score) p.best_h_score[b] = bh >= 0 ? key_value(hk) : -INFINITY;
+            }
+            if (has_a) {
+                p.best_a[b] = ba;
+                if (p.best_a_score) p.best_a_score[b] = ba >= 0 ? key_value(ak) : -INFINITY;
+            }
+            p.draft_len[b] = static_cast<int32_t>(dl);
+            if (p.status && total > p.C_cap) atomicOr(p.status + b, PLDP_ST_CAND_OVERFLOW);
+            if (p.status && bad) atomicOr(p.status + b, PLDP_ST_ROW_INDEX);
+            // the index now covers 0 .. t-1 (or is unusable: a token it cannot hold, or stale)
+            if (usable) ix.ilen[b] = is.bad_token ? -1 : static_cast<int32_t>(t);
+            else if (il > t) ix.ilen[b] = -1;
+        }
+    };
+
+    // ---- the list scored: every occurrence, or the candidates --------------------------
+    // spec: at most kSpeculate occurrences, all scored at once; their suffix matches
+    // are read in the same round trip and n* then picks the candidates among them.
+    // Otherwise the suffix matches come first (each scored occurrence costs a
+    // d-element row and R scattered attention values) and only the candidates
+    // (the first C_cap) are scored.  Either way one loop with one call of the
+    // scorer, kSpeculate positions a pass: every case runs the same code.
+    constexpr int NB = kSpeculate;
     unsigned long long hk = 0, ak = 0;
     int nstar = 0, total = 0;
-    if (indexed) {
-        // the occurrences, ascending: the indexed ones (all before il) ranked, then the appended ones
-        if (warp == 0) {
-            const int nold = is.count_old;
-            if (lane < nold) {
-                const int32_t v = is.slot[lane];
-                int rank = 0;
-                for (int k = 0; k < nold; ++k) rank += is.slot[k] < v ? 1 : 0;
-                is.occ[rank] = v;
-            }
-            int base = nold;
-            for (int c0 = 0; c0 < nnew; c0 += 32) {
-                const bool hit = c0 + lane < nnew && is.newtok[c0 + lane] == xt;
-                const unsigned bal = __ballot_sync(0xFFFFFFFFu, hit);
-                if (hit) is.occ[base + __popc(bal & ((1u << lane) - 1u))] = static_cast<int32_t>(il + c0 + lane);
-                base += __popc(bal);
-            }
-            if (lane == 0) is.nocc = base;
-        }
-        __syncthreads();
-        const int nocc = is.nocc;
-        // suffix-match lengths; the rows the ranking will read start towards L2
+    const bool spec = indexed && nocc <= kSpeculate;
+    if (indexed && !spec) {
         int mloc = 0;
         for (int i = tid; i < nocc; i += kThreads) {
             const int64_t j = is.occ[i];
-            if (HAS_H && j >= 1)
-                prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (j - 1) * p.d) * h_es,
-                                 static_cast<uint32_t>(p.d * h_es));
-            int m = 1;
-            while (m < p.ngram_max && j - m >= 0) {
+            int32_t pv[PLDP_MAX_NGRAM - 1];                       // x_{j-1}, x_{j-2}, ... all requested at once
+#pragma unroll
+            for (int m = 1; m < PLDP_MAX_NGRAM; ++m) {
                 const int64_t q = j - m;
-                const int32_t v = q >= il ? is.newtok[q - il] : __ldg(row + q);
-                if (v != is.suf[m]) break;
-                ++m;
+                pv[m - 1] = (m < p.ngram_max && q >= 0) ? (q >= il ? is.newtok[q - il] : __ldg(row + q)) : 0;
             }
+            int m = 1;
+#pragma unroll
+            for (int k = 1; k < PLDP_MAX_NGRAM; ++k)
+                if (m == k && k < p.ngram_max && j - k >= 0 && pv[k - 1] == is.suf[k]) m = k + 1;
             is.occ_m[i] = m;
             mloc = m > mloc ? m : mloc;
-        }
-        if (has_a) {                                             // the attention values of every occurrence
-            const size_t es = p.a_bf16 ? 2 : 4;
-            const char* ab = static_cast<const char*>(p.A) + static_cast<int64_t>(b) * p.a_seq_stride * es;
-            for (int i = 0; i < nocc; ++i) {
-                const int64_t j = is.occ[i];
-                for (int k = tid; k < p.n_sel; k += kThreads) {
-                    const int r = p.row_idx ? __ldg(p.row_idx + k) : k;
-                    if (r >= 0 && r < p.R)
-                        asm volatile("prefetch.global.L2 [%0];" ::"l"(ab + (static_cast<int64_t>(r) * p.a_row_stride + j) * es));
-                }
-            }
         }
         mloc = __reduce_max_sync(0xFFFFFFFFu, mloc);
         if (lane == 0) is.wmax[warp] = mloc;
@@ -740,43 +870,122 @@ __global__ void __launch_bounds__(kThreads) draft_index_kernel(const DraftParams
         __syncthreads();
         nstar = is.nstar;
         total = is.ncand;
-        const int n = total < p.C_cap ? total : p.C_cap;
-        constexpr int NB = kMaxScoreBatch;
-        for (int i0 = 0; i0 < n; i0 += NB) {
+    } else if (!indexed) {
+        finish_overflow<TH, IVEC, kMaxScoreBatch>(p, b, t, row, cand_row, hsc, asc, sh, hk, ak, nstar, total);
+    }
+
+    if (indexed) {
+        const int32_t* list = spec ? is.occ : is.cand;
+        const int n = spec ? nocc : (total < p.C_cap ? total : p.C_cap);
+        int32_t pre[PLDP_MAX_NGRAM - 1];                          // spec, thread h < n: x_{j-1}, x_{j-2}, ...
+        const int64_t jm = (spec && tid < n) ? list[tid] : -1;
+#pragma unroll
+        for (int m = 1; m < PLDP_MAX_NGRAM; ++m) {
+            const int64_t q = jm - m;
+            pre[m - 1] = (jm >= 0 && m < p.ngram_max && q >= 0) ? (q >= il ? is.newtok[q - il] : __ldg(row + q)) : 0;
+        }
+        const bool staged = p.K <= kDraftWin;                     // warp 0, lane i: token i after list[h], h < NB
+        int32_t dv[NB];
+        int64_t j0[NB];
+#pragma unroll
+        for (int h = 0; h < NB; ++h) {
+            j0[h] = h < n ? list[h] : -1;
+            const int64_t q = j0[h] + 1 + lane;
+            dv[h] = (staged && warp == 0 && h < n && lane < p.K && q <= t) ? __ldg(row + q) : -1;
+        }
+        float s_h[NB], s_a[NB];
+        for (int i0 = 0; i0 < n; i0 += NB) {                      // one pass but for many candidates
             const int nb = n - i0 < NB ? n - i0 : NB;
             int64_t j[NB];
 #pragma unroll
-            for (int h = 0; h < NB; ++h) j[h] = h < nb ? is.cand[i0 + h] : -1;
-            float s_h[NB], s_a[NB];
+            for (int h = 0; h < NB; ++h) j[h] = h < nb ? list[i0 + h] : -1;
             cta_score<TH, NB>(p, b, j, nb, t, part_buf<NB>(sh.part[(i0 / NB) & 1]), s_h, s_a);
-            if (tid == 0)
-                for (int h = 0; h < nb; ++h) {
-                    const int i = i0 + h;
+            if (!spec && warp == 0)                               // candidates: keys now
+#pragma unroll
+                for (int h = 0; h < NB; ++h) {
+                    if (h >= nb) continue;
+                    const int r = i0 + h;
                     if (HAS_H) {
-                        if (hsc) hsc[i] = s_h[h];
+                        if (hsc && lane == 0) hsc[r] = s_h[h];
                         if (j[h] >= 1 && s_h[h] > p.threshold) {
                             const unsigned long long key = pack_key(s_h[h], static_cast<uint32_t>(j[h]));
                             hk = key > hk ? key : hk;
                         }
                     }
                     if (has_a) {
-                        if (asc) asc[i] = s_a[h];
+                        if (asc && lane == 0) asc[r] = s_a[h];
                         const unsigned long long key = pack_key(s_a[h], static_cast<uint32_t>(j[h]));
                         ak = key > ak ? key : ak;
                     }
                 }
         }
-    } else {
-        finish_overflow<TH, IVEC>(p, b, t, row, cand_row, hsc, asc, sh, hk, ak, nstar, total);
+        if (mine) index_put(ix, b, mytok, myslot, il + tid);      // the slot taken above
+        if (warp != 0) return;
+        if (spec) {
+            // n* among the scored occurrences (n <= NB: one pass), then their keys
+            int m = 0;
+            if (lane < n) {
+                m = 1;
+#pragma unroll
+                for (int k = 1; k < PLDP_MAX_NGRAM; ++k)
+                    if (m == k && k < p.ngram_max && jm - k >= 0 && pre[k - 1] == is.suf[k]) m = k + 1;
+            }
+            int mh[NB], mx = 0;
+#pragma unroll
+            for (int h = 0; h < NB; ++h) {
+                mh[h] = __shfl_sync(0xFFFFFFFFu, m, h);
+                mx = mh[h] > mx ? mh[h] : mx;
+            }
+            nstar = mx >= p.ngram_min ? mx : 0;                   // m <= ngram_max already
+            int r = 0;                                            // candidates: ascending, as the occurrences
+            if (nstar > 0)
+#pragma unroll
+                for (int h = 0; h < NB; ++h) {
+                    if (h >= n || mh[h] < nstar) continue;
+                    if (r < p.C_cap) {
+                        if (lane == 0) cand_row[r] = static_cast<int32_t>(j0[h]);
+                        if (HAS_H) {
+                            if (hsc && lane == 0) hsc[r] = s_h[h];
+                            if (j0[h] >= 1 && s_h[h] > p.threshold) {
+                                const unsigned long long key = pack_key(s_h[h], static_cast<uint32_t>(j0[h]));
+                                hk = key > hk ? key : hk;
+                            }
+                        }
+                        if (has_a) {
+                            if (asc && lane == 0) asc[r] = s_a[h];
+                            const unsigned long long key = pack_key(s_a[h], static_cast<uint32_t>(j0[h]));
+                            ak = key > ak ? key : ak;
+                        }
+                    }
+                    ++r;
+                }
+            total = r;
+        }
+        outputs(hk, ak, nstar, total, [&](int i, int64_t js) -> int32_t {
+            if (staged && i == lane) {
+                int32_t v = -1;
+                bool found = false;
+#pragma unroll
+                for (int h = 0; h < NB; ++h)
+                    if (h < n && j0[h] == js) {
+                        v = dv[h];
+                        found = true;
+                    }
+                if (found) return v;
+            }
+            return __ldg(row + js + 1 + i);
+        });
+        return;
     }
 
-    // ---- best of each ranking, then the draft (Sec. 4.3) ----------------------------------
+    // ---- the rescan's keys, combined over the CTA, then the outputs ---------------------
     hk = warp_max_u64(hk);
     ak = warp_max_u64(ak);
     if (lane == 0) {
         sh.wkey[0][warp] = hk;
         sh.wkey[1][warp] = ak;
     }
+    if (mine) index_put(ix, b, mytok, myslot, il + tid);          // the slot taken above
     __syncthreads();
     if (warp != 0) return;
     hk = 0;
@@ -786,31 +995,7 @@ __global__ void __launch_bounds__(kThreads) draft_index_kernel(const DraftParams
         hk = sh.wkey[0][w] > hk ? sh.wkey[0][w] : hk;
         ak = sh.wkey[1][w] > ak ? sh.wkey[1][w] : ak;
     }
-    const int32_t bh = hk == 0 ? -1 : static_cast<int32_t>(key_index(hk));
-    const int32_t ba = ak == 0 ? -1 : static_cast<int32_t>(key_index(ak));
-    const int64_t js = p.draft_from == 0 ? bh : ba;
-    int64_t dl = 0;
-    if (js >= 0 && js < t) dl = (t - js < p.K) ? (t - js) : p.K;
-    for (int i = lane; i < p.K; i += 32)
-        p.draft[static_cast<int64_t>(b) * p.K + i] = (i < dl) ? __ldg(row + js + 1 + i) : -1;
-    if (lane == 0) {
-        p.cand_count[b] = total;
-        p.match_len[b] = nstar;
-        if (HAS_H) {
-            p.best_h[b] = bh;
-            if (p.best_h_score) p.best_h_score[b] = bh >= 0 ? key_value(hk) : -INFINITY;
-        }
-        if (has_a) {
-            p.best_a[b] = ba;
-            if (p.best_a_score) p.best_a_score[b] = ba >= 0 ? key_value(ak) : -INFINITY;
-        }
-        p.draft_len[b] = static_cast<int32_t>(dl);
-        if (p.status && total > p.C_cap) atomicOr(p.status + b, PLDP_ST_CAND_OVERFLOW);
-        if (p.status && bad) atomicOr(p.status + b, PLDP_ST_ROW_INDEX);
-        // the index now covers 0 .. t-1 (or is unusable: a token it cannot hold, or stale)
-        if (usable) ix.ilen[b] = is.bad_token ? -1 : static_cast<int32_t>(t);
-        else if (il > t) ix.ilen[b] = -1;
-    }
+    outputs(hk, ak, nstar, total, [&](int i, int64_t js) -> int32_t { return __ldg(row + js + 1 + i); });
 }
 
 // Index build: positions 0 .. seq_len-2 of every sequence.
@@ -844,25 +1029,24 @@ __global__ void index_finish_kernel(const int32_t* __restrict__ seq_len, int B, 
     if (bad_token && status) atomicOr(status + b, PLDP_ST_TOKEN_RANGE);
 }
 
-// Byte offsets of the index parts (ilen, flags, counts, slots), 256-byte aligned.
+// Byte offsets of the index parts (ilen, flags, entries), 256-byte aligned.
 struct IndexLayout {
-    size_t ilen, flags, counts, slots, total;
+    size_t ilen, flags, entries, total;
 };
 inline IndexLayout index_layout(int B, int V) {
     auto up = [](size_t x) { return (x + 255) / 256 * 256; };
     IndexLayout l;
     l.ilen = 0;
     l.flags = up(static_cast<size_t>(B) * 4);
-    l.counts = l.flags + up(static_cast<size_t>(B) * 4);
-    l.slots = l.counts + up(static_cast<size_t>(B) * V * 4);
-    l.total = l.slots + up(static_cast<size_t>(B) * V * kIndexSlots * 4);
+    l.entries = l.flags + up(static_cast<size_t>(B) * 4);
+    l.total = l.entries + up(static_cast<size_t>(B) * V * kEntryWords * 4);
     return l;
 }
 inline IndexView index_view(void* base, int B, int V) {
     const IndexLayout l = index_layout(B, V);
     char* c = static_cast<char*>(base);
     return IndexView{reinterpret_cast<int32_t*>(c + l.ilen), reinterpret_cast<int32_t*>(c + l.flags),
-                     reinterpret_cast<int32_t*>(c + l.counts), reinterpret_cast<int32_t*>(c + l.slots), V};
+                     reinterpret_cast<int32_t*>(c + l.entries), V};
 }
 
 template <typename TH, bool IVEC>

@@ -42,12 +42,26 @@ def _ilen(index, B):
     return host(index[:4 * B].view(torch.int32))
 
 
-@pytest.mark.parametrize("T,V,B", [(300, 4, 12), (4096, 50, 8), (8000, 3000, 16), (2048, 2, 20)])
+# V sets how many occurrences x_t has: hundreds (scanned), 9..15 (suffix matches first,
+# then the candidates scored), up to 8 (all scored in one pass)
+@pytest.mark.parametrize("T,V,B", [(300, 4, 12), (4096, 50, 8), (4096, 300, 8), (8000, 3000, 16), (2048, 2, 20)])
 @pytest.mark.parametrize("mode", ["both", "hidden", "attention"])
 def test_indexed_step_equals_scan(lib, T, V, B, mode):
+    _indexed_case(T, V, B, mode, C=64, K=10, ngram=(1, 3))
+
+
+@pytest.mark.parametrize("T,V,B", [(4096, 50, 8), (4096, 300, 8), (8000, 3000, 16), (30000, 20000, 6)])
+@pytest.mark.parametrize("C,K,ngram", [(2, 70, (1, 3)), (1, 5, (2, 4)), (3, 64, (1, 8))])
+def test_indexed_step_small_caps(lib, T, V, B, C, K, ngram):
+    """Candidate lists shorter than the occurrences scored in one pass, drafts longer
+    than the staged window, and other n-gram ranges."""
+    _indexed_case(T, V, B, "both", C=C, K=K, ngram=ngram)
+
+
+def _indexed_case(T, V, B, mode, C, K, ngram):
     rng = np.random.default_rng(T + V)
     gen = torch.Generator(device=DEV).manual_seed(T + 1)
-    C, K, d, R = 64, 10, 128, 12
+    d, R = 128, 12
     T_cap = T + 2000
     ids = rng.integers(0, V, size=(B, T_cap)).astype(np.int32)
     lens = rng.integers(0, T + 1, size=B)
@@ -63,11 +77,11 @@ def test_indexed_step_equals_scan(lib, T, V, B, mode):
     assert host(st)[3] == pk.PLDP_ST_SEQ_LEN and (np.delete(host(st), 3) == 0).all()
     a, b_ = Buffers(B, K, 8, C, DEV), Buffers(B, K, 8, C, DEV)
     for step in range(5):
-        g_scan = _draft(a, ids_g, L_g, K, H, A, draft_from=draft_from)
-        g_idx = _draft(b_, ids_g, L_g, K, H, A, index=index, V=V, draft_from=draft_from)
+        g_scan = _draft(a, ids_g, L_g, K, H, A, ngram=ngram, draft_from=draft_from)
+        g_idx = _draft(b_, ids_g, L_g, K, H, A, index=index, V=V, ngram=ngram, draft_from=draft_from)
         _same(g_scan, g_idx)
         if step == 0:
-            _compare(g_idx, ids, lens, H, A, None, 0, (1, 3), C, K, draft_from)
+            _compare(g_idx, ids, lens, H, A, None, 0, ngram, C, K, draft_from)
         # the contexts grow: 1..13 tokens, one long append, one sequence cut back
         L = host(L_g).astype(np.int64)
         for s in range(B):
