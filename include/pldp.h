@@ -356,6 +356,51 @@ PLDP_API pldp_status pldp_verify_greedy(const void* logits, pldp_dtype dtype, in
                                         size_t workspace_bytes, void* stream);
 
 /*
+ * Greedy verification of the current step followed by the drafting of the next
+ * one, in one call -- pldp_verify_greedy then pldp_draft_step (with the token
+ * index) on the context it has just extended, with the same results and status
+ * bits as those two calls in turn.  The paper has no counterpart: in a decode
+ * loop the next draft depends only on this step's verification (the accepted
+ * tokens, the bonus token) and on the hidden states and attention rows of the
+ * forward pass that produced this step's logits, so nothing runs between the
+ * two.  The argmax pass is followed, one CTA per sequence, by the accept/bonus/
+ * append of verification and then the candidate search, ranking and draft of
+ * the next step.
+ *
+ *  logits, dtype, V   this step's logits [B, K+1, V], as pldp_verify_greedy.
+ *  draft, draft_len   this step's draft [B, K] and lengths [B]; they may be the
+ *                     same buffers as next.draft and next.draft_len (each
+ *                     sequence's draft is read before it is replaced).
+ *  argmax, accept_len, next_token, kv_keep_len, workspace, workspace_bytes
+ *                     as pldp_verify_greedy (workspace zeroed before first use;
+ *                     every call leaves it zero).
+ *  next               the next step's pldp_draft_step arguments.  next.index is
+ *                     required (built by pldp_index_build, with next.V == V).
+ *                     next.B and next.K are the verification's B and K;
+ *                     next.ids, next.ids_stride, next.seq_len and next.T_cap are
+ *                     the context verification appends to (read and WRITTEN by
+ *                     this call); next.status receives both calls' bits.
+ *                     next.workspace is not used.
+ */
+typedef struct pldp_verify_draft_args {
+    const void* logits;
+    pldp_dtype dtype;
+    int V;
+    const int32_t* draft;
+    const int32_t* draft_len;
+    int32_t* argmax;
+    int32_t* accept_len;
+    int32_t* next_token;
+    int32_t* kv_keep_len;
+    void* workspace;
+    size_t workspace_bytes;
+    pldp_draft_step_args next;
+} pldp_verify_draft_args;
+
+/* `args` is a HOST pointer to the argument block, read before the call returns. */
+PLDP_API pldp_status pldp_verify_greedy_draft(const pldp_verify_draft_args* args, void* stream);
+
+/*
  * Sampling verification -- Sec. 4.4 at temperature T > 0 (the paper's sampled
  * runs use T = 1, Table 2).  Position i of sequence b draws
  *   y_i = the smallest v with sum_{v' <= v} p_v' > u[b, i],

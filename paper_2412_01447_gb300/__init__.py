@@ -44,6 +44,12 @@ PLDP_ST_DRAFT_LEN = 16
 PLDP_ST_ROW_INDEX = 32
 PLDP_ST_TIMEOUT = 64
 
+PLDP_OK = 0
+PLDP_ERR_INVALID_ARG = 1
+PLDP_ERR_UNSUPPORTED = 2
+PLDP_ERR_CUDA = 3
+PLDP_ERR_TIMEOUT = 4
+
 _STATUS_NAMES = {1: "PLDP_ERR_INVALID_ARG", 2: "PLDP_ERR_UNSUPPORTED", 3: "PLDP_ERR_CUDA",
                  4: "PLDP_ERR_TIMEOUT"}
 
@@ -76,6 +82,16 @@ class pldp_draft_step_args(ctypes.Structure):
         ("draft_len", ctypes.c_void_p), ("status", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
         ("index", ctypes.c_void_p), ("index_bytes", ctypes.c_size_t), ("V", ctypes.c_int),
+    ]
+
+
+class pldp_verify_draft_args(ctypes.Structure):
+    """Mirror of the C argument block of pldp_verify_greedy_draft (include/pldp.h)."""
+    _fields_ = [
+        ("logits", ctypes.c_void_p), ("dtype", ctypes.c_int), ("V", ctypes.c_int),
+        ("draft", ctypes.c_void_p), ("draft_len", ctypes.c_void_p), ("argmax", ctypes.c_void_p),
+        ("accept_len", ctypes.c_void_p), ("next_token", ctypes.c_void_p), ("kv_keep_len", ctypes.c_void_p),
+        ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t), ("next", pldp_draft_step_args),
     ]
 
 
@@ -120,6 +136,8 @@ def _load():
                 getattr(lib, f).restype = ctypes.c_int
             lib.pldp_draft_step.argtypes = [ctypes.POINTER(pldp_draft_step_args), P]
             lib.pldp_draft_step.restype = ctypes.c_int
+            lib.pldp_verify_greedy_draft.argtypes = [ctypes.POINTER(pldp_verify_draft_args), P]
+            lib.pldp_verify_greedy_draft.restype = ctypes.c_int
             lib.pldp_draft_workspace_size.argtypes = [i32]
             lib.pldp_draft_workspace_size.restype = sz
             lib.pldp_index_size.argtypes = [i32, i32]
@@ -302,17 +320,12 @@ def pldp_draft_workspace_size(B) -> int:
     return int(_load().pldp_draft_workspace_size(B))
 
 
-def pldp_draft_step(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, draft,
-                    draft_len, workspace, H=None, best_h=None, h_scores=None, best_h_score=None,
-                    threshold=float("-inf"), A=None, best_a=None, row_idx=None, agg=PLDP_AGG_MAX,
-                    a_scores=None, best_a_score=None, draft_from="hidden", status=None, T_cap=None,
-                    index=None, V=None, stream=None):
-    """Candidate search, ranking (hidden and/or attention) and draft in one call; the
-    arguments mean what they mean in the separate calls.  workspace: a uint8 CUDA
-    tensor of pldp_draft_workspace_size(B) bytes, zeroed once before first use (may be
-    None with an index).  index: a uint8 CUDA tensor of pldp_index_size(B, V) bytes
-    built by pldp_index_build (token ids in [0, V)); the step then looks occurrences
-    up instead of scanning, with the same results."""
+def _draft_args(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, draft,
+                draft_len, workspace, H=None, best_h=None, h_scores=None, best_h_score=None,
+                threshold=float("-inf"), A=None, best_a=None, row_idx=None, agg=PLDP_AGG_MAX,
+                a_scores=None, best_a_score=None, draft_from="hidden", status=None, T_cap=None,
+                index=None, V=None):
+    """The argument block of pldp_draft_step (marshalling only)."""
     p_ids, stride, T = _rows(ids, "ids")
     B = ids.shape[0]
     a = pldp_draft_step_args()
@@ -356,7 +369,49 @@ def pldp_draft_step(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, ma
         a.index = _dense(index, "index")
         a.index_bytes = index.numel() * index.element_size()
         a.V = int(V)
+    return a
+
+
+def pldp_draft_step(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, draft,
+                    draft_len, workspace, stream=None, **kw):
+    """Candidate search, ranking (hidden and/or attention) and draft in one call; the
+    arguments mean what they mean in the separate calls.  workspace: a uint8 CUDA
+    tensor of pldp_draft_workspace_size(B) bytes, zeroed once before first use (may be
+    None with an index).  index: a uint8 CUDA tensor of pldp_index_size(B, V) bytes
+    built by pldp_index_build (token ids in [0, V)); the step then looks occurrences
+    up instead of scanning, with the same results.  Keyword arguments: H, best_h,
+    h_scores, best_h_score, threshold, A, best_a, row_idx, agg, a_scores,
+    best_a_score, draft_from, status, T_cap, index, V."""
+    a = _draft_args(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, draft,
+                    draft_len, workspace, **kw)
     _check("pldp_draft_step", _load().pldp_draft_step(ctypes.byref(a), _stream(stream)))
+
+
+def pldp_verify_greedy_draft(logits, draft, draft_len, accept_len, next_token, workspace, ids, seq_len,
+                             ngram_min, ngram_max, cand_pos, cand_count, match_len, next_draft,
+                             next_draft_len, index, argmax=None, kv_keep_len=None, stream=None, **kw):
+    """Greedy verification of this step (as pldp_verify_greedy, appending to ids and
+    seq_len) followed by the next step's drafting with the token index (as
+    pldp_draft_step on the extended context), in one call.  next_draft /
+    next_draft_len receive the next draft (they may be draft / draft_len).  Keyword
+    arguments are pldp_draft_step's (H, best_h, A, best_a, status, ...)."""
+    B, K1, V = logits.shape
+    K = K1 - 1
+    if draft.shape != (B, K) or next_draft.shape != (B, K):
+        raise ValueError("draft and next_draft must be [B, K] with K = logits.shape[1] - 1")
+    a = pldp_verify_draft_args()
+    a.next = _draft_args(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, next_draft,
+                         next_draft_len, None, index=index, V=V, **kw)
+    a.logits, a.dtype, a.V = _dense(logits, "logits"), _code(logits.dtype), V
+    a.draft = _dense(draft, "draft", torch.int32)
+    a.draft_len = _dense(draft_len, "draft_len", torch.int32)
+    a.argmax = _dense(argmax, "argmax", torch.int32, allow_none=True)
+    a.accept_len = _dense(accept_len, "accept_len", torch.int32)
+    a.next_token = _dense(next_token, "next_token", torch.int32)
+    a.kv_keep_len = _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True)
+    a.workspace = _dense(workspace, "workspace")
+    a.workspace_bytes = workspace.numel() * workspace.element_size()
+    _check("pldp_verify_greedy_draft", _load().pldp_verify_greedy_draft(ctypes.byref(a), _stream(stream)))
 
 
 def pldp_index_size(B, V) -> int:

@@ -30,6 +30,7 @@
 
 #include "pldp_rank.cuh"
 #include "pldp_scan.cuh"
+#include "pldp_verify.cuh"
 
 namespace pldp {
 namespace {
@@ -307,7 +308,7 @@ __device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int
 // L2, then the candidates are scored by cta_score, NB per pass.  Kept out of
 // line: its registers do not weigh on the common path.  CTA-uniform call; keys
 // are left in thread 0.
-template <typename TH, bool IVEC, int NB>
+template <typename TH, bool IVEC, int NB, typename RD = ReadOnlyIds>
 __device__ __noinline__ void finish_overflow(const DraftParams& p, int b, int64_t t, const int32_t* row,
                                              int32_t* cand_row, float* hsc, float* asc, StepShared& sh,
                                              unsigned long long& hk, unsigned long long& ak, int& nstar,
@@ -318,7 +319,7 @@ __device__ __noinline__ void finish_overflow(const DraftParams& p, int b, int64_
     int c[PLDP_MAX_NGRAM];
 #pragma unroll
     for (int k = 0; k < PLDP_MAX_NGRAM; ++k) c[k] = 0;
-    scan_count<IVEC>(GlobalIds{row}, row, 0, t, t, p.ngram_max, c);
+    scan_count<IVEC, GlobalIdsT<RD>, RD>(GlobalIdsT<RD>{row}, row, 0, t, t, p.ngram_max, c);
     scan_reduce_counts(c, p.ngram_max, sh.ss);
     __syncthreads();
     if (tid == 0) {
@@ -337,7 +338,8 @@ __device__ __noinline__ void finish_overflow(const DraftParams& p, int b, int64_
     __syncthreads();
     nstar = sh.ss.nstar;
     total = sh.ss.total;
-    scan_write<IVEC>(GlobalIds{row}, row, 0, t, t, p.ngram_max, sh.ss, cand_row, p.C_cap);
+    scan_write<IVEC, GlobalIdsT<RD>, NoHook, RD>(GlobalIdsT<RD>{row}, row, 0, t, t, p.ngram_max, sh.ss, cand_row,
+                                                 p.C_cap);
     __syncthreads();
     const int n = total < p.C_cap ? total : p.C_cap;
     if (HAS_H && n > NB) {
@@ -683,15 +685,14 @@ __device__ __forceinline__ bool index_insert(const IndexView& ix, int b, int64_t
     return slot >= 0;
 }
 
-template <typename TH, bool IVEC>
-__global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftParams p, const IndexView ix) {
+// The indexed drafting of sequence b by the whole CTA, for context length L.
+// RD: how ids are read -- CoherentIds when this kernel has just appended to the
+// context (verification fused in front), else through the read-only cache.
+template <typename TH, bool IVEC, typename RD>
+__device__ __forceinline__ void index_draft(const DraftParams& p, const IndexView& ix, int b, int64_t L,
+                                            StepShared& sh, IndexShared& is) {
     constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
-    __shared__ StepShared sh;
-    __shared__ IndexShared is;
-    pdl_enter();
-    const int b = blockIdx.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int64_t L = p.seq_len[b];
     const int64_t il = ix.ilen[b];
     const bool valid = L >= 0 && L <= p.T_cap;
     const int64_t t = L - 1;
@@ -732,8 +733,8 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
     if (tid == 0 && HAS_H && t >= 2)                              // H_{t-1}: every candidate's score reads it
         prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (t - 1) * p.d) * h_es,
                          static_cast<uint32_t>(p.d * h_es));
-    if (small && tid < nnew) is.newtok[tid] = __ldg(row + il + tid);
-    if (tid < PLDP_MAX_NGRAM) is.suf[tid] = (tid < p.ngram_max && t - tid >= 0) ? __ldg(row + t - tid) : 0;
+    if (small && tid < nnew) is.newtok[tid] = RD::one(row + il + tid);
+    if (tid < PLDP_MAX_NGRAM) is.suf[tid] = (tid < p.ngram_max && t - tid >= 0) ? RD::one(row + t - tid) : 0;
     __syncthreads();
     const int32_t xt = is.suf[0];
     const bool lookup = small && t >= 1 && xt >= 0 && xt < ix.V;
@@ -775,7 +776,7 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
     if (mine && mytok == xt) myslot = index_take(ix, b, mytok);
     if (usable && !small) {                                       // a long append: inserted in turn
         bool badtok = false;
-        for (int64_t q = il + tid; q < t; q += kThreads) badtok |= !index_insert(ix, b, q, __ldg(row + q));
+        for (int64_t q = il + tid; q < t; q += kThreads) badtok |= !index_insert(ix, b, q, RD::one(row + q));
         if (badtok) atomicOr(&is.bad_token, 1);
     }
 
@@ -833,7 +834,7 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
 #pragma unroll
             for (int m = 1; m < PLDP_MAX_NGRAM; ++m) {
                 const int64_t q = j - m;
-                pv[m - 1] = (m < p.ngram_max && q >= 0) ? (q >= il ? is.newtok[q - il] : __ldg(row + q)) : 0;
+                pv[m - 1] = (m < p.ngram_max && q >= 0) ? (q >= il ? is.newtok[q - il] : RD::one(row + q)) : 0;
             }
             int m = 1;
 #pragma unroll
@@ -871,7 +872,7 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
         nstar = is.nstar;
         total = is.ncand;
     } else if (!indexed) {
-        finish_overflow<TH, IVEC, kMaxScoreBatch>(p, b, t, row, cand_row, hsc, asc, sh, hk, ak, nstar, total);
+        finish_overflow<TH, IVEC, kMaxScoreBatch, RD>(p, b, t, row, cand_row, hsc, asc, sh, hk, ak, nstar, total);
     }
 
     if (indexed) {
@@ -882,7 +883,7 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
 #pragma unroll
         for (int m = 1; m < PLDP_MAX_NGRAM; ++m) {
             const int64_t q = jm - m;
-            pre[m - 1] = (jm >= 0 && m < p.ngram_max && q >= 0) ? (q >= il ? is.newtok[q - il] : __ldg(row + q)) : 0;
+            pre[m - 1] = (jm >= 0 && m < p.ngram_max && q >= 0) ? (q >= il ? is.newtok[q - il] : RD::one(row + q)) : 0;
         }
         const bool staged = p.K <= kDraftWin;                     // warp 0, lane i: token i after list[h], h < NB
         int32_t dv[NB];
@@ -891,7 +892,7 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
         for (int h = 0; h < NB; ++h) {
             j0[h] = h < n ? list[h] : -1;
             const int64_t q = j0[h] + 1 + lane;
-            dv[h] = (staged && warp == 0 && h < n && lane < p.K && q <= t) ? __ldg(row + q) : -1;
+            dv[h] = (staged && warp == 0 && h < n && lane < p.K && q <= t) ? RD::one(row + q) : -1;
         }
         float s_h[NB], s_a[NB];
         for (int i0 = 0; i0 < n; i0 += NB) {                      // one pass but for many candidates
@@ -973,7 +974,7 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
                     }
                 if (found) return v;
             }
-            return __ldg(row + js + 1 + i);
+            return RD::one(row + js + 1 + i);
         });
         return;
     }
@@ -995,7 +996,39 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
         hk = sh.wkey[0][w] > hk ? sh.wkey[0][w] : hk;
         ak = sh.wkey[1][w] > ak ? sh.wkey[1][w] : ak;
     }
-    outputs(hk, ak, nstar, total, [&](int i, int64_t js) -> int32_t { return __ldg(row + js + 1 + i); });
+    outputs(hk, ak, nstar, total, [&](int i, int64_t js) -> int32_t { return RD::one(row + js + 1 + i); });
+}
+
+template <typename TH, bool IVEC>
+__global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftParams p, const IndexView ix) {
+    __shared__ StepShared sh;
+    __shared__ IndexShared is;
+    pdl_enter();
+    index_draft<TH, IVEC, ReadOnlyIds>(p, ix, blockIdx.x, p.seq_len[blockIdx.x], sh, is);
+}
+
+// Verification of the current step -- the finish of greedy verification: the
+// accepted length, the bonus token and the append (Sec. 4.4) -- and then, in the
+// same CTA, the next step's drafting with the token index.  One CTA per
+// sequence, launched behind the verification's argmax pass.  The draft step
+// starts from the context the finish has just written: its length is known
+// without a read, and the appended ids are read through L2.
+template <typename TH, bool IVEC>
+__global__ void __launch_bounds__(kThreads, 1) verify_draft_kernel(const VerifyArgs va, const DraftParams p,
+                                                                    const IndexView ix) {
+    __shared__ StepShared sh;
+    __shared__ IndexShared is;
+    __shared__ long long L_after;
+    pdl_enter();                                                  // the pass's row keys are final
+    const int b = blockIdx.x;
+    if (threadIdx.x < 32) {
+        const int64_t L1 = finish_sequence(va, b, static_cast<int>(threadIdx.x),
+                                           KeyTokens{va.row_keys + static_cast<int64_t>(b) * (va.K + 1)});
+        if (threadIdx.x == 0) L_after = L1;
+    }
+    __syncthreads();                                              // the append is visible to the whole CTA
+    const int64_t L = L_after >= 0 ? static_cast<int64_t>(L_after) : static_cast<int64_t>(__ldcg(p.seq_len + b));
+    index_draft<TH, IVEC, CoherentIds>(p, ix, b, L, sh, is);
 }
 
 // Index build: positions 0 .. seq_len-2 of every sequence.
@@ -1075,82 +1108,74 @@ pldp_status launch_draft_step(const DraftParams& p, int B, cudaStream_t s, bool 
     return ivec ? launch_t<TH, true>(p, B, s) : launch_t<TH, false>(p, B, s);
 }
 
-}  // namespace
-}  // namespace pldp
-
-using namespace pldp;
-
-extern "C" PLDP_API size_t pldp_draft_workspace_size(int B) {
-    return B < 0 ? 0 : static_cast<size_t>(B) * kSeqWs;
-}
-
-extern "C" PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* a, void* stream) {
-    if (!a) return fail(PLDP_ERR_INVALID_ARG, "draft_step: null argument block");
+// The checks and argument block of pldp_draft_step (`what` names the call in
+// messages).  empty: B == 0, nothing to launch.
+pldp_status prepare_draft(const pldp_draft_step_args* a, const char* what, DraftParams& p, IndexView& ixv,
+                          bool& has_ix, bool& ivec, bool& empty) {
     const int B = a->B;
-    if (B < 0) return fail(PLDP_ERR_INVALID_ARG, "draft_step: B < 0");
-    if (B > 65535) return fail(PLDP_ERR_UNSUPPORTED, "draft_step: B > 65535");
+    if (B < 0) return fail(PLDP_ERR_INVALID_ARG, "%s: B < 0", what);
+    if (B > 65535) return fail(PLDP_ERR_UNSUPPORTED, "%s: B > 65535", what);
     if (a->T_cap < 0 || a->T_cap > kMaxPositions)
-        return fail(PLDP_ERR_INVALID_ARG, "draft_step: T_cap outside [0, 2^27]");
-    if (a->ids_stride < a->T_cap) return fail(PLDP_ERR_INVALID_ARG, "draft_step: ids_stride < T_cap");
+        return fail(PLDP_ERR_INVALID_ARG, "%s: T_cap outside [0, 2^27]", what);
+    if (a->ids_stride < a->T_cap) return fail(PLDP_ERR_INVALID_ARG, "%s: ids_stride < T_cap", what);
     if (a->ngram_min < 1 || a->ngram_max < a->ngram_min || a->ngram_max > PLDP_MAX_NGRAM)
-        return fail(PLDP_ERR_INVALID_ARG, "draft_step: need 1 <= ngram_min <= ngram_max <= %d",
+        return fail(PLDP_ERR_INVALID_ARG, "%s: need 1 <= ngram_min <= ngram_max <= %d", what,
                     PLDP_MAX_NGRAM);
-    if (a->C_cap < 0) return fail(PLDP_ERR_INVALID_ARG, "draft_step: C_cap < 0");
-    if (a->K < 1) return fail(PLDP_ERR_INVALID_ARG, "draft_step: K < 1");
-    if (!a->H && !a->A) return fail(PLDP_ERR_INVALID_ARG, "draft_step: neither H nor A given");
+    if (a->C_cap < 0) return fail(PLDP_ERR_INVALID_ARG, "%s: C_cap < 0", what);
+    if (a->K < 1) return fail(PLDP_ERR_INVALID_ARG, "%s: K < 1", what);
+    if (!a->H && !a->A) return fail(PLDP_ERR_INVALID_ARG, "%s: neither H nor A given", what);
     if (a->draft_from != 0 && a->draft_from != 1)
-        return fail(PLDP_ERR_INVALID_ARG, "draft_step: draft_from must be 0 (hidden) or 1 (attention)");
+        return fail(PLDP_ERR_INVALID_ARG, "%s: draft_from must be 0 (hidden) or 1 (attention)", what);
     if ((a->draft_from == 0 && !a->H) || (a->draft_from == 1 && !a->A))
-        return fail(PLDP_ERR_INVALID_ARG, "draft_step: draft_from names a ranking that is not given");
+        return fail(PLDP_ERR_INVALID_ARG, "%s: draft_from names a ranking that is not given", what);
     size_t qbytes = 0, h_es = 0;
     if (a->H) {
         if (a->h_dtype != PLDP_F32 && a->h_dtype != PLDP_BF16)
-            return fail(PLDP_ERR_UNSUPPORTED, "draft_step: unsupported hidden dtype %d", (int)a->h_dtype);
+            return fail(PLDP_ERR_UNSUPPORTED, "%s: unsupported hidden dtype %d", what, (int)a->h_dtype);
         h_es = a->h_dtype == PLDP_F32 ? 4 : 2;
-        if (a->d < 1) return fail(PLDP_ERR_INVALID_ARG, "draft_step: d < 1");
+        if (a->d < 1) return fail(PLDP_ERR_INVALID_ARG, "%s: d < 1", what);
         qbytes = static_cast<size_t>(a->d) * h_es;
         if (qbytes > kMaxQueryBytes)
-            return fail(PLDP_ERR_UNSUPPORTED, "draft_step: d * sizeof(dtype) > %zu", kMaxQueryBytes);
+            return fail(PLDP_ERR_UNSUPPORTED, "%s: d * sizeof(dtype) > %zu", what, kMaxQueryBytes);
         if (a->h_seq_stride < a->T_cap * a->d)
-            return fail(PLDP_ERR_INVALID_ARG, "draft_step: h_seq_stride < T_cap*d");
-        if (a->threshold != a->threshold) return fail(PLDP_ERR_INVALID_ARG, "draft_step: threshold is NaN");
+            return fail(PLDP_ERR_INVALID_ARG, "%s: h_seq_stride < T_cap*d", what);
+        if (a->threshold != a->threshold) return fail(PLDP_ERR_INVALID_ARG, "%s: threshold is NaN", what);
     }
     int sel = 0;
     if (a->A) {
         if (a->a_dtype != PLDP_F32 && a->a_dtype != PLDP_BF16)
-            return fail(PLDP_ERR_UNSUPPORTED, "draft_step: unsupported attention dtype %d", (int)a->a_dtype);
+            return fail(PLDP_ERR_UNSUPPORTED, "%s: unsupported attention dtype %d", what, (int)a->a_dtype);
         if (a->agg != PLDP_AGG_MAX && a->agg != PLDP_AGG_SUM)
-            return fail(PLDP_ERR_INVALID_ARG, "draft_step: unknown aggregation %d", (int)a->agg);
-        if (a->R < 1) return fail(PLDP_ERR_INVALID_ARG, "draft_step: R < 1");
-        if (a->a_row_stride < a->T_cap) return fail(PLDP_ERR_INVALID_ARG, "draft_step: a_row_stride < T_cap");
+            return fail(PLDP_ERR_INVALID_ARG, "%s: unknown aggregation %d", what, (int)a->agg);
+        if (a->R < 1) return fail(PLDP_ERR_INVALID_ARG, "%s: R < 1", what);
+        if (a->a_row_stride < a->T_cap) return fail(PLDP_ERR_INVALID_ARG, "%s: a_row_stride < T_cap", what);
         if (a->a_seq_stride < static_cast<int64_t>(a->R) * a->a_row_stride)
-            return fail(PLDP_ERR_INVALID_ARG, "draft_step: a_seq_stride < R*a_row_stride");
+            return fail(PLDP_ERR_INVALID_ARG, "%s: a_seq_stride < R*a_row_stride", what);
         sel = a->row_idx ? a->n_sel : a->R;
         if (sel < 1 || sel > kMaxSelRows)
-            return fail(PLDP_ERR_INVALID_ARG, "draft_step: need 1 <= n_sel <= %d", kMaxSelRows);
+            return fail(PLDP_ERR_INVALID_ARG, "%s: need 1 <= n_sel <= %d", what, kMaxSelRows);
     }
-    if (B == 0) return PLDP_OK;
+    empty = B == 0;
+    if (empty) return PLDP_OK;
     if (!a->ids || !a->seq_len || !a->cand_count || !a->match_len || !a->draft || !a->draft_len ||
         (a->C_cap > 0 && !a->cand_pos) || (a->H && !a->best_h) || (a->A && !a->best_a))
-        return fail(PLDP_ERR_INVALID_ARG, "draft_step: null pointer");
-    IndexView ixv = {};
-    const IndexView* ix = nullptr;
+        return fail(PLDP_ERR_INVALID_ARG, "%s: null pointer", what);
+    has_ix = a->index != nullptr;
     if (a->index) {
-        if (a->V < 1) return fail(PLDP_ERR_INVALID_ARG, "draft_step: V < 1 with an index");
+        if (a->V < 1) return fail(PLDP_ERR_INVALID_ARG, "%s: V < 1 with an index", what);
         const size_t need = index_layout(B, a->V).total;
         if (a->index_bytes < need || !aligned16(a->index))
-            return fail(PLDP_ERR_INVALID_ARG, "draft_step: index needs %zu bytes, 16-byte aligned", need);
+            return fail(PLDP_ERR_INVALID_ARG, "%s: index needs %zu bytes, 16-byte aligned", what, need);
         ixv = index_view(a->index, B, a->V);
-        ix = &ixv;
-    } else if (!a->workspace || a->workspace_bytes < pldp_draft_workspace_size(B) || !aligned16(a->workspace)) {
-        return fail(PLDP_ERR_INVALID_ARG, "draft_step: workspace needs %zu bytes, 16-byte aligned",
-                    pldp_draft_workspace_size(B));
+    } else if (!a->workspace || a->workspace_bytes < static_cast<size_t>(B) * kSeqWs || !aligned16(a->workspace)) {
+        return fail(PLDP_ERR_INVALID_ARG, "%s: workspace needs %zu bytes, 16-byte aligned", what,
+                    static_cast<size_t>(B) * kSeqWs);
     }
     if (a->H && !(aligned16(a->H) && qbytes % 16 == 0 && (a->h_seq_stride * h_es) % 16 == 0))
         return fail(PLDP_ERR_UNSUPPORTED,
                     "draft_step: hidden rows must be 16-byte aligned (the separate calls accept any layout)");
 
-    DraftParams p = {};
+    p = DraftParams{};
     p.ids = a->ids;
     p.ids_stride = a->ids_stride;
     p.seq_len = a->seq_len;
@@ -1186,11 +1211,79 @@ extern "C" PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* a, v
     p.draft_len = a->draft_len;
     p.status = a->status;
     p.ws = static_cast<unsigned char*>(a->workspace);
-    const bool ivec = aligned16(a->ids) && a->ids_stride % 4 == 0 && a->T_cap % 4 == 0;
+    ivec = aligned16(a->ids) && a->ids_stride % 4 == 0 && a->T_cap % 4 == 0;
+    return PLDP_OK;
+}
+
+template <typename TH, bool IVEC>
+pldp_status launch_verify_draft_t(const VerifyArgs& va, const DraftParams& p, const IndexView& ix, int B,
+                                  cudaStream_t s) {
+    const cudaError_t e = launch_pdl(verify_draft_kernel<TH, IVEC>, dim3(static_cast<unsigned>(B)), dim3(kThreads), 0,
+                                     s, 0, va, p, ix);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "verify_greedy_draft: launch failed: %s", cudaGetErrorString(e));
+    return PLDP_OK;
+}
+
+template <typename TH>
+pldp_status launch_verify_draft(const VerifyArgs& va, const DraftParams& p, const IndexView& ix, int B, bool ivec,
+                                cudaStream_t s) {
+    return ivec ? launch_verify_draft_t<TH, true>(va, p, ix, B, s) : launch_verify_draft_t<TH, false>(va, p, ix, B, s);
+}
+
+}  // namespace
+}  // namespace pldp
+
+using namespace pldp;
+
+extern "C" PLDP_API size_t pldp_draft_workspace_size(int B) {
+    return B < 0 ? 0 : static_cast<size_t>(B) * kSeqWs;
+}
+
+extern "C" PLDP_API pldp_status pldp_draft_step(const pldp_draft_step_args* a, void* stream) {
+    if (!a) return fail(PLDP_ERR_INVALID_ARG, "draft_step: null argument block");
+    DraftParams p;
+    IndexView ixv = {};
+    bool has_ix = false, ivec = false, empty = false;
+    const pldp_status st = prepare_draft(a, "draft_step", p, ixv, has_ix, ivec, empty);
+    if (st != PLDP_OK || empty) return st;
+    const int B = a->B;
+    const IndexView* ix = has_ix ? &ixv : nullptr;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (!a->H) return launch_draft_step<NoHidden>(p, B, s, ivec, ix);
     if (a->h_dtype == PLDP_BF16) return launch_draft_step<__nv_bfloat16>(p, B, s, ivec, ix);
     return launch_draft_step<float>(p, B, s, ivec, ix);
+}
+
+extern "C" PLDP_API pldp_status pldp_verify_greedy_draft(const pldp_verify_draft_args* a, void* stream) {
+    if (!a) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_draft: null argument block");
+    const pldp_draft_step_args& n = a->next;
+    if (!n.index) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_draft: the next draft needs a token index");
+    if (a->V < 1) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_draft: V < 1");
+    if (n.V != a->V) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_draft: the index's V differs from the logits'");
+    if (a->dtype != PLDP_F32 && a->dtype != PLDP_BF16)
+        return fail(PLDP_ERR_UNSUPPORTED, "verify_greedy_draft: unsupported dtype %d", (int)a->dtype);
+    if (n.T_cap > INT32_MAX) return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_draft: bad T_cap");
+    DraftParams p;
+    IndexView ixv = {};
+    bool has_ix = false, ivec = false, empty = false;
+    const pldp_status st = prepare_draft(&n, "verify_greedy_draft", p, ixv, has_ix, ivec, empty);
+    if (st != PLDP_OK || empty) return st;
+    const int B = n.B, K = n.K;
+    if (!a->logits || !a->draft || !a->draft_len || !a->accept_len || !a->next_token)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_draft: null pointer");
+    const size_t need = pldp_verify_workspace_size(B, K, a->V);
+    if (!a->workspace || a->workspace_bytes < need || !aligned16(a->workspace))
+        return fail(PLDP_ERR_INVALID_ARG, "verify_greedy_draft: workspace needs %zu bytes, 16-byte aligned", need);
+    // verification appends to the context the next draft reads: next.ids and next.seq_len
+    VerifyArgs va = verify_args(B, K, a->V, a->draft, a->draft_len, a->argmax, a->accept_len, a->next_token,
+                                const_cast<int32_t*>(n.ids), n.ids_stride, const_cast<int32_t*>(n.seq_len), n.T_cap,
+                                a->kv_keep_len, n.status);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const pldp_status sp = launch_verify_pass(a->logits, a->dtype, va, a->workspace, s, "verify_greedy_draft");
+    if (sp != PLDP_OK) return sp;
+    if (!n.H) return launch_verify_draft<NoHidden>(va, p, ixv, B, ivec, s);
+    if (n.h_dtype == PLDP_BF16) return launch_verify_draft<__nv_bfloat16>(va, p, ixv, B, ivec, s);
+    return launch_verify_draft<float>(va, p, ixv, B, ivec, s);
 }
 
 extern "C" PLDP_API size_t pldp_index_size(int B, int V) {

@@ -26,14 +26,26 @@ struct ScanShared {
     int nstar, offset, mine, total;
 };
 
+// How ids are read: through the read-only cache (a context that no kernel of
+// the call writes), or through L2 (a context that the same kernel has just
+// appended to, which the read-only path is not guaranteed to see).
+struct ReadOnlyIds {
+    static __device__ __forceinline__ int32_t one(const int32_t* p) { return __ldg(p); }
+    static __device__ __forceinline__ int4 four(const int4* p) { return __ldg(p); }
+};
+struct CoherentIds {
+    static __device__ __forceinline__ int32_t one(const int32_t* p) { return __ldcg(p); }
+    static __device__ __forceinline__ int4 four(const int4* p) { return __ldcg(p); }
+};
+
 // Length of the common suffix of x[0..j] and x[0..t] (x_j == x_t already known),
-// capped at n_max.  j < t, so x_{t-m} exists whenever x_{j-m} does.  Suffix
-// tokens are read through the read-only cache: every thread of the CTA reads the
-// same few of them.
+// capped at n_max.  j < t, so x_{t-m} exists whenever x_{j-m} does.  Every
+// thread of the CTA reads the same few suffix tokens.
+template <typename RD = ReadOnlyIds>
 __device__ __forceinline__ int suffix_match(const int32_t* __restrict__ row, int64_t j, int64_t t,
                                             int n_max) {
     int m = 1;
-    while (m < n_max && j - m >= 0 && __ldg(row + j - m) == __ldg(row + t - m)) ++m;
+    while (m < n_max && j - m >= 0 && RD::one(row + j - m) == RD::one(row + t - m)) ++m;
     return m;
 }
 
@@ -45,12 +57,14 @@ __device__ __forceinline__ void count_hit(int (&c)[PLDP_MAX_NGRAM], int m) {
 // Where pass 1 and pass 2 read the ids from: global memory (16-byte or 4-byte
 // loads) or a copy of the CTA's chunk staged in shared memory (`base` = ids of
 // positions c0, c0 + 1, ...).  `load4(q)` returns positions 4q .. 4q + 3.
-struct GlobalIds {
+template <typename RD>
+struct GlobalIdsT {
     const int32_t* row;
     __device__ __forceinline__ int4 load4(int64_t q) const {
-        return __ldg(reinterpret_cast<const int4*>(row) + q);
+        return RD::four(reinterpret_cast<const int4*>(row) + q);
     }
 };
+using GlobalIds = GlobalIdsT<ReadOnlyIds>;
 struct SharedIds {
     const int32_t* base;   // shared memory, 16-byte aligned
     int64_t q0;            // first int4 index of the staged chunk (c0 / 4)
@@ -62,12 +76,12 @@ struct SharedIds {
 // Pass 1 over positions [c0, c1) (c0 a multiple of 4 when VEC; all < t):
 // c[k] += number of positions whose match length exceeds k.  With VEC the ids
 // come through `src` (16-byte units); otherwise 4-byte global loads from `row`.
-template <bool VEC, typename Src>
+template <bool VEC, typename Src, typename RD = ReadOnlyIds>
 __device__ __forceinline__ void scan_count(const Src& src, const int32_t* __restrict__ row, int64_t c0,
                                            int64_t c1, int64_t t, int n_max, int (&c)[PLDP_MAX_NGRAM]) {
     if (c0 >= c1) return;
     const int tid = threadIdx.x;
-    const int32_t xt = __ldg(row + t);
+    const int32_t xt = RD::one(row + t);
     if constexpr (VEC) {
         const int64_t q0 = c0 >> 2, q1 = (c1 + 3) >> 2;
         for (int64_t qb = q0 + tid; qb < q1; qb += static_cast<int64_t>(kScanThreads) * kScanUnroll) {
@@ -85,7 +99,7 @@ __device__ __forceinline__ void scan_count(const Src& src, const int32_t* __rest
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                     const int64_t p = 4 * q + k;
-                    if (e[k] == xt && p < c1) count_hit(c, suffix_match(row, p, t, n_max));
+                    if (e[k] == xt && p < c1) count_hit(c, suffix_match<RD>(row, p, t, n_max));
                 }
             }
         }
@@ -95,12 +109,12 @@ __device__ __forceinline__ void scan_count(const Src& src, const int32_t* __rest
 #pragma unroll
             for (int u = 0; u < kScanUnroll; ++u) {
                 const int64_t p = pb + static_cast<int64_t>(u) * kScanThreads;
-                if (p < c1) v[u] = __ldg(row + p);
+                if (p < c1) v[u] = RD::one(row + p);
             }
 #pragma unroll
             for (int u = 0; u < kScanUnroll; ++u) {
                 const int64_t p = pb + static_cast<int64_t>(u) * kScanThreads;
-                if (p < c1 && v[u] == xt) count_hit(c, suffix_match(row, p, t, n_max));
+                if (p < c1 && v[u] == xt) count_hit(c, suffix_match<RD>(row, p, t, n_max));
             }
         }
     }
@@ -160,7 +174,7 @@ struct NoHook {
     __device__ __forceinline__ void operator()(int64_t) const {}
 };
 
-template <bool VEC, typename Src, typename Hook = NoHook>
+template <bool VEC, typename Src, typename Hook = NoHook, typename RD = ReadOnlyIds>
 __device__ __forceinline__ void scan_write(const Src& src, const int32_t* __restrict__ row, int64_t c0,
                                            int64_t c1, int64_t t, int n_max, ScanShared& sh,
                                            int32_t* __restrict__ dst, int C_cap,
@@ -169,7 +183,7 @@ __device__ __forceinline__ void scan_write(const Src& src, const int32_t* __rest
     int64_t out = sh.offset;
     if (!(nstar > 0 && mine > 0 && out < C_cap)) return;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int32_t xt = __ldg(row + t);
+    const int32_t xt = RD::one(row + t);
     const int64_t end = out + mine;
     constexpr int G = VEC ? 4 : 1;                       // positions per thread per tile
     const int64_t g0 = c0 / G, g1 = (c1 + G - 1) / G;
@@ -185,12 +199,12 @@ __device__ __forceinline__ void scan_write(const Src& src, const int32_t* __rest
                 e[2] = v.z;
                 e[3] = v.w;
             } else {
-                e[0] = __ldg(row + g);
+                e[0] = RD::one(row + g);
             }
 #pragma unroll
             for (int k = 0; k < G; ++k) {
                 const int64_t p = g * G + k;
-                if (e[k] == xt && p < c1 && suffix_match(row, p, t, n_max) >= nstar) mask |= 1u << k;
+                if (e[k] == xt && p < c1 && suffix_match<RD>(row, p, t, n_max) >= nstar) mask |= 1u << k;
             }
         }
         const int cnt = __popc(mask);

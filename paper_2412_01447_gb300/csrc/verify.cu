@@ -21,6 +21,7 @@
 #include <math.h>
 
 #include "pldp_internal.cuh"
+#include "pldp_verify.cuh"
 
 namespace pldp {
 namespace {
@@ -94,101 +95,6 @@ __device__ __forceinline__ void lane_argmax(const T* __restrict__ row, int64_t c
                 }
             }
         }
-    }
-}
-
-struct VerifyArgs {
-    const int32_t* draft;
-    const int32_t* draft_len;
-    int32_t* argmax;
-    int32_t* accept_len;
-    int32_t* next_token;
-    int32_t* ids;
-    int64_t ids_stride;
-    int32_t* seq_len;
-    int64_t T_cap;
-    int32_t* kv_keep_len;
-    uint32_t* status;
-    unsigned long long* row_keys;   // [B*(K+1)], zero between calls
-    int B, K, V;
-};
-
-// Where the finish reads the K+1 target tokens of a sequence: the greedy row keys
-// (argmax packed in the low word; the keys are returned to zero afterwards) or
-// the draws of sampling verification, staged in shared memory.
-struct KeyTokens {
-    unsigned long long* keys;   // [K+1] of this sequence
-    __device__ __forceinline__ int at(int i) const { return static_cast<int>(key_index(__ldcg(keys + i))); }
-    __device__ __forceinline__ void release(int K1, int lane) const {
-        for (int i = lane; i < K1; i += 32) keys[i] = 0ull;
-    }
-};
-struct SharedTokens {
-    const int32_t* tok;          // shared memory, [K+1]
-    __device__ __forceinline__ int at(int i) const { return tok[i]; }
-    __device__ __forceinline__ void release(int, int) const {}
-};
-
-// Accept/bonus/append for sequence b, by one warp, once its K+1 target tokens are
-// final.  Everything it reads is requested up front (one round trip when K < 32).
-// Sec. 4.4: n = first i < d with draft_i != target_i (else d), bonus = target_n.
-template <typename Src>
-__device__ void finish_sequence(const VerifyArgs& a, int64_t b, int lane, const Src& src) {
-    const int K1 = a.K + 1;
-    const int d_in = a.draft_len[b];
-    const int64_t L = a.seq_len ? a.seq_len[b] : 0;
-    const int t_first = lane < K1 ? src.at(lane) : 0;
-    const int tok_first = lane < a.K ? a.draft[b * a.K + lane] : 0;
-    uint32_t st = 0;
-    int d = d_in;
-    if (d < 0 || d > a.K) {
-        st |= PLDP_ST_DRAFT_LEN;
-        d = d < 0 ? 0 : a.K;
-    }
-    int n = d;
-    bool range_bad = false;
-    for (int i0 = 0; i0 < K1; i0 += 32) {
-        const int i = i0 + lane;
-        const int am = i0 == 0 ? t_first : (i < K1 ? src.at(i) : 0);
-        const int tok = i0 == 0 ? tok_first : (i < a.K ? a.draft[b * a.K + i] : 0);
-        if (i < K1 && a.argmax) a.argmax[b * K1 + i] = am;
-        const bool in_draft = i < d;
-        range_bad |= in_draft && (tok < 0 || tok >= a.V);
-        const unsigned mism = __ballot_sync(0xFFFFFFFFu, in_draft && tok != am);
-        if (n == d && mism) n = i0 + __ffs(mism) - 1;
-    }
-    if (__any_sync(0xFFFFFFFFu, range_bad)) st |= PLDP_ST_TOKEN_RANGE;
-    const int bonus = n < 32 ? __shfl_sync(0xFFFFFFFFu, t_first, n) : src.at(n);
-    __syncwarp();
-    src.release(K1, lane);
-
-    if (lane == 0) {
-        a.accept_len[b] = n;
-        a.next_token[b] = bonus;
-    }
-    if (a.seq_len) {
-        int64_t kv = -1;
-        if (L < 1 || L > a.T_cap) {
-            st |= PLDP_ST_SEQ_LEN;
-        } else {
-            kv = L + n;
-            if (L + n + 1 > a.T_cap) {
-                st |= PLDP_ST_CAPACITY;
-            } else {
-                if (a.ids) {
-                    int32_t* row = a.ids + b * a.ids_stride + L;
-                    if (lane < n) row[lane] = tok_first;
-                    for (int i = 32 + lane; i < n; i += 32) row[i] = a.draft[b * a.K + i];
-                    if (lane == 0) row[n] = bonus;
-                }
-                __syncwarp();
-                if (lane == 0) a.seq_len[b] = static_cast<int32_t>(L + n + 1);
-            }
-        }
-        if (a.kv_keep_len && lane == 0) a.kv_keep_len[b] = static_cast<int32_t>(kv);
-    }
-    if (lane == 0) {
-        if (a.status && st) a.status[b] |= st;
     }
 }
 
@@ -366,10 +272,9 @@ size_t keys_bytes(int B, int K) {
 }
 
 // Sizes the pass's grid (up to kPassWaves waves of resident CTAs, no more warps
-// than segments) and launches both kernels.  `a` has everything but the keys.
+// than segments) and launches it.  `a` has everything but the keys.
 template <typename T, int PATH>
-pldp_status launch_verify_t(const void* logits, VerifyArgs a, void* scratch, cudaStream_t s,
-                            const char* what) {
+pldp_status launch_pass_t(const void* logits, VerifyArgs& a, void* scratch, cudaStream_t s, const char* what) {
     const void* fn = reinterpret_cast<const void*>(&verify_argmax_kernel<T, PATH>);
     const int64_t N = static_cast<int64_t>(a.B) * (a.K + 1) * a.V;
     constexpr int64_t SEG = kSegBytes / static_cast<int64_t>(sizeof(T));
@@ -379,18 +284,17 @@ pldp_status launch_verify_t(const void* logits, VerifyArgs a, void* scratch, cud
     if (blocks > need) blocks = need;
     if (blocks < 1) blocks = 1;
     a.row_keys = static_cast<unsigned long long*>(scratch);
-    cudaError_t e = launch_pdl(verify_argmax_kernel<T, PATH>, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0,
-                               s, 0, static_cast<const T*>(logits), N, static_cast<int64_t>(a.V),
-                               blocks * kWarps, a.row_keys);
-    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
-    const unsigned fblocks = static_cast<unsigned>((a.B + kWarps - 1) / kWarps);
-    e = launch_pdl(verify_finish_kernel, dim3(fblocks), dim3(kThreads), 0, s, 0, a);
+    const cudaError_t e = launch_pdl(verify_argmax_kernel<T, PATH>, dim3(static_cast<unsigned>(blocks)),
+                                     dim3(kThreads), 0, s, 0, static_cast<const T*>(logits), N,
+                                     static_cast<int64_t>(a.V), blocks * kWarps, a.row_keys);
     if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
     return PLDP_OK;
 }
 
-pldp_status launch_verify(const void* logits, pldp_dtype dtype, const VerifyArgs& a, void* scratch,
-                          cudaStream_t s, const char* what) {
+}  // namespace
+
+pldp_status launch_verify_pass(const void* logits, pldp_dtype dtype, VerifyArgs& a, void* scratch,
+                               cudaStream_t s, const char* what) {
     const size_t es = dtype == PLDP_F32 ? 4 : 2;
     const bool vec = aligned16(logits) && (static_cast<size_t>(a.V) * es) % 16 == 0;
     const int64_t bytes = static_cast<int64_t>(a.B) * (a.K + 1) * a.V * static_cast<int64_t>(es);
@@ -398,13 +302,13 @@ pldp_status launch_verify(const void* logits, pldp_dtype dtype, const VerifyArgs
     const bool small = bytes / 16 < (int64_t(1) << 31);     // 32-bit vector indices
     const int path = vec ? (long_rows && small ? 0 : 1) : 2;
     if (dtype == PLDP_BF16) {
-        if (path == 0) return launch_verify_t<__nv_bfloat16, 0>(logits, a, scratch, s, what);
-        if (path == 1) return launch_verify_t<__nv_bfloat16, 1>(logits, a, scratch, s, what);
-        return launch_verify_t<__nv_bfloat16, 2>(logits, a, scratch, s, what);
+        if (path == 0) return launch_pass_t<__nv_bfloat16, 0>(logits, a, scratch, s, what);
+        if (path == 1) return launch_pass_t<__nv_bfloat16, 1>(logits, a, scratch, s, what);
+        return launch_pass_t<__nv_bfloat16, 2>(logits, a, scratch, s, what);
     }
-    if (path == 0) return launch_verify_t<float, 0>(logits, a, scratch, s, what);
-    if (path == 1) return launch_verify_t<float, 1>(logits, a, scratch, s, what);
-    return launch_verify_t<float, 2>(logits, a, scratch, s, what);
+    if (path == 0) return launch_pass_t<float, 0>(logits, a, scratch, s, what);
+    if (path == 1) return launch_pass_t<float, 1>(logits, a, scratch, s, what);
+    return launch_pass_t<float, 2>(logits, a, scratch, s, what);
 }
 
 VerifyArgs verify_args(int B, int K, int V, const int32_t* draft, const int32_t* draft_len,
@@ -427,6 +331,21 @@ VerifyArgs verify_args(int B, int K, int V, const int32_t* draft, const int32_t*
     a.K = K;
     a.V = V;
     return a;
+}
+
+
+namespace {
+
+// The pass, then the finish (one warp per sequence) behind its last wave.
+pldp_status launch_verify(const void* logits, pldp_dtype dtype, const VerifyArgs& a0, void* scratch,
+                          cudaStream_t s, const char* what) {
+    VerifyArgs a = a0;
+    const pldp_status st = launch_verify_pass(logits, dtype, a, scratch, s, what);
+    if (st != PLDP_OK) return st;
+    const unsigned fblocks = static_cast<unsigned>((a.B + kWarps - 1) / kWarps);
+    const cudaError_t e = launch_pdl(verify_finish_kernel, dim3(fblocks), dim3(kThreads), 0, s, 0, a);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
+    return PLDP_OK;
 }
 
 }  // namespace
