@@ -67,6 +67,9 @@ def parse():
                          "is built before the timed loop and kept up to date inside every timed step)")
     ap.add_argument("--separate", action="store_true",
                     help="draft with the four separate calls instead of the fused launch")
+    ap.add_argument("--two-calls", action="store_true",
+                    help="time pldp_draft_step + pldp_verify_greedy per step instead of the one "
+                         "pldp_verify_greedy_draft call (which verifies a step and drafts the next)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sample", action="store_true",
                     help="skip the separate timing of sampling verification (T = 1) on the same logits")
@@ -219,9 +222,14 @@ def profiled_traffic(kernel_srcs, profile_name):
 
 
 class Path:
-    """Device buffers and the five C-ABI calls of one step."""
+    """Device buffers and the C-ABI calls of one step.
 
-    def __init__(self, pk, loop: wl.DecodeLoop, fused=True, index=False):
+    vd (the default): one pldp_verify_greedy_draft call per step -- this step's
+    verification and the next step's drafting with the token index; the loop's
+    first draft comes from prime().  Otherwise pldp_draft_step (fused, with or
+    without the index) or the four separate drafting calls, then pldp_verify_greedy."""
+
+    def __init__(self, pk, loop: wl.DecodeLoop, fused=True, index=False, vd=False):
         self.pk, self.loop = pk, loop
         w, dev = loop.w, loop.device
         B, K, C = w.B, w.K, w.C_cap
@@ -235,21 +243,45 @@ class Path:
         self.ws = torch.zeros(pk.pldp_verify_workspace_size(B, K, w.V), dtype=torch.uint8, device=dev)
         self.dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=dev)
         self.row_idx = None   # all R rows of the chosen layers
+        self.vd = vd and fused
         self.index = (torch.empty(pk.pldp_index_size(B, w.V), dtype=torch.uint8, device=dev)
-                      if index and fused else None)
+                      if (index or self.vd) and fused else None)
         self.fused = fused
-        self.launches_per_step = 3 if fused else 6     # pldp_verify_greedy launches two kernels
-        self.kernels = (["draft_step"] if fused else
-                        ["find_candidates", "rank_hidden", "rank_attention", "extract_draft"]) + ["verify_greedy"]
+        if self.vd:
+            self.launches_per_step = 2                  # the argmax pass, then verification + next draft
+            self.kernels = ["verify_greedy_draft"]
+        else:
+            self.launches_per_step = 3 if fused else 6  # pldp_verify_greedy launches two kernels
+            self.kernels = (["draft_step"] if fused else
+                            ["find_candidates", "rank_hidden", "rank_attention", "extract_draft"]) + ["verify_greedy"]
 
     def build_index(self):
         """(Re)builds the token index for the loop's current contexts (not timed)."""
         if self.index is not None:
             self.pk.pldp_index_build(self.loop.ids, self.loop.seq_len, self.loop.w.V, self.index)
 
+    def prime(self, step=0):
+        """vd: the loop's first draft, for the current state (the prefill's draft; not timed)."""
+        if self.vd:
+            self.loop.step_inputs(step)
+            self._draft(torch.cuda.current_stream())
+
+    def inputs(self, step):
+        """Writes the inputs of step ``step`` for the current state (not timed)."""
+        if self.vd:
+            self.loop.step_inputs_next(step, self.draft, self.dlen)
+        else:
+            self.loop.step_inputs(step)
+
+    def _draft(self, s):
+        lp, w = self.loop, self.loop.w
+        self.pk.pldp_draft_step(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt, self.ml,
+                                w.K, self.draft, self.dlen, self.dws, H=lp.H, best_h=self.best_h, A=lp.A,
+                                best_a=self.best_a, row_idx=self.row_idx, draft_from="hidden",
+                                status=self.status, index=self.index, V=w.V, stream=s)
+
     def run(self, ev=None, stream=None, step_only=False):
-        """One step: the drafting half (one fused launch, or the four separate calls)
-        then verification.  ev: events recorded before the first and after every kernel
+        """One step.  ev: events recorded before the first and after every call
         (step_only: before the first and after the last only)."""
         pk, lp, w = self.pk, self.loop, self.loop.w
         s = torch.cuda.current_stream() if stream is None else stream
@@ -264,11 +296,16 @@ class Path:
                 k[0] += 1
 
         rec()
+        if self.vd:
+            pk.pldp_verify_greedy_draft(lp.logits, self.draft, self.dlen, self.acc, self.nxt, self.ws, lp.ids,
+                                        lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt, self.ml,
+                                        self.draft, self.dlen, self.index, kv_keep_len=self.kv, H=lp.H,
+                                        best_h=self.best_h, A=lp.A, best_a=self.best_a, row_idx=self.row_idx,
+                                        draft_from="hidden", status=self.status, stream=s)
+            rec()
+            return
         if self.fused:
-            pk.pldp_draft_step(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt, self.ml,
-                               w.K, self.draft, self.dlen, self.dws, H=lp.H, best_h=self.best_h, A=lp.A,
-                               best_a=self.best_a, row_idx=self.row_idx, draft_from="hidden",
-                               status=self.status, index=self.index, V=w.V, stream=s)
+            self._draft(s)
             rec()
         else:
             pk.pldp_find_candidates(lp.ids, lp.seq_len, w.ngram_min, w.ngram_max, self.cand, self.cnt,
@@ -297,6 +334,11 @@ def step_bytes(w, seq_len_mean, cand_mean):
               extract_draft=4.0 * B * w.K,
               verify_greedy=2.0 * B * (w.K + 1) * w.V)
     by["draft_step"] = by["find_candidates"] + by["rank_hidden"] + by["rank_attention"] + by["extract_draft"]
+    # drafting with the token index: x_t's 64-byte entry, <= K+1 appended ids, hidden rows,
+    # attention values and the draft (no scan)
+    by["draft_index"] = (B * (64.0 + 4 * (w.K + 1)) + by["rank_hidden"] + by["rank_attention"]
+                         + by["extract_draft"])
+    by["verify_greedy_draft"] = by["verify_greedy"] + by["draft_index"]
     return by
 
 
@@ -322,8 +364,10 @@ def run_ours(args, ws_, rank, local):
     K_steps, W_steps = args.steps, args.warmup
     t0 = time.perf_counter()
     loop = wl.DecodeLoop(w, steps=W_steps + K_steps, device=dev)
-    path = Path(pk, loop, fused=not args.separate, index=not args.scan)
+    vd = not (args.separate or args.scan or args.two_calls)
+    path = Path(pk, loop, fused=not args.separate, index=not args.scan, vd=vd)
     path.build_index()
+    path.prime(0)
     nk = len(path.kernels)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)     # 2x the 129 MB L2
     flush_sink = torch.empty((), dtype=torch.int64, device=dev)
@@ -341,7 +385,7 @@ def run_ours(args, ws_, rank, local):
     setup_s = time.perf_counter() - t0
 
     for s in range(W_steps):
-        loop.step_inputs(s)
+        path.inputs(s)
         flush_l2(s)
         path.run()
     torch.cuda.synchronize()
@@ -356,7 +400,7 @@ def run_ours(args, ws_, rank, local):
     clocks.start()
     wall0 = time.perf_counter()
     for s in range(K_steps):
-        loop.step_inputs(W_steps + s)
+        path.inputs(W_steps + s)
         len_sum += loop.seq_len.sum()
         flush_l2(s)
         path.run(evs[s], step_only=args.events == "step")
@@ -388,14 +432,26 @@ def run_ours(args, ws_, rank, local):
     L_mean = float(len_sum) / (K_steps * w.B)
     by = step_bytes(w, L_mean, cand_mean)
     peak, peak_kind = measured_peak()
-    ver_s = per_k[nk - 1] / K_steps / 1e3
     ver_bytes = by["verify_greedy"]
+    two_call = None
+    if path.vd:
+        # the verify call alone, for the roofline: the same loop with the two calls
+        two_call = time_two_call_variant(pk, loop, w, flush_l2)
+        ver_s = two_call["verify_us"] / 1e6
+        ver_src = ("verify_greedy (argmax pass + finish) per call, from the two-call variant of the same "
+                   "loop in this run (the headline call fuses it with the next draft)")
+    else:
+        ver_s = per_k[nk - 1] / K_steps / 1e3
+        ver_src = "verify_greedy (argmax pass + finish) per call in the timed loop"
     achieved = ver_bytes / ver_s / 1e9
     csrc = os.path.join(ROOT, "paper_2412_01447_gb300", "csrc")
     traffic = profiled_traffic([os.path.join(csrc, "verify.cu"), os.path.join(csrc, "pldp_internal.cuh")],
                                "verify_greedy_c5.md")
-    step_bytes_total = sum(by[k] for k in ("find_candidates", "rank_hidden", "rank_attention",
-                                            "extract_draft", "verify_greedy"))
+    if path.index is not None:
+        step_bytes_total = by["verify_greedy"] + by["draft_index"]
+    else:
+        step_bytes_total = sum(by[k] for k in ("find_candidates", "rank_hidden", "rank_attention",
+                                                "extract_draft", "verify_greedy"))
     lossless = bool(torch.equal(loop.ids[:, :w.T], loop.gt[:, :w.T]))
     L_now = loop.seq_len.long()
     pos = torch.arange(loop.T_cap, device=dev)[None]
@@ -426,11 +482,14 @@ def run_ours(args, ws_, rank, local):
                           if args.flush == "write-read" else
                           "flushed before every step: 256 MB write (cold L2 holding dirty lines)")
                          + "; per-step logits 427 MB and attention rows 1.18 GB regenerated between steps",
-                   "path": (("pldp_draft_step (incremental token index + both rankings + draft)"
+                   "path": ("pldp_verify_greedy_draft per step: this step's greedy verification, then the "
+                            "next step's drafting with the incremental token index (both rankings + draft); "
+                            "the first draft (pldp_draft_step) precedes the warm-up" if path.vd else
+                            ("pldp_draft_step (incremental token index + both rankings + draft)"
                              if path.index is not None else
                              "pldp_draft_step (fused scan + both rankings + draft)") + " + pldp_verify_greedy"
                             if path.fused else "five separate C-ABI calls"),
-                   "timing": "CUDA events around every kernel of each step on the launch stream; "
+                   "timing": "CUDA events around every C-ABI call of each step on the launch stream; "
                              "artifact generation between steps is not timed",
                    "parallelism": f"{ws_} independent replicas (batch shards)"},
         "achieved_step_gbs": round(step_bytes_total / (ms_per_step / 1e3) / 1e9, 1),
@@ -441,7 +500,7 @@ def run_ours(args, ws_, rank, local):
                               for i, k in enumerate(path.kernels)},
         "kernel_gbs": {k: round(by[k] / (per_k[i] / K_steps / 1e3) / 1e9, 1)
                        for i, k in enumerate(path.kernels)},
-        "roofline": {"kernel": "verify_greedy", "bound": "hbm", "achieved": round(achieved, 1),
+        "roofline": {"kernel": "verify_greedy", "timed": ver_src, "bound": "hbm", "achieved": round(achieved, 1),
                      "peak": peak, "peak_kind": peak_kind, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "frac_of_nominal_8tbs": round(achieved / NOMINAL_HBM_GBS, 4),
                      "traffic": traffic, "algorithmic_bytes": ver_bytes},
@@ -452,6 +511,8 @@ def run_ours(args, ws_, rank, local):
                   "lossless_vs_ground_truth": lossless, "setup_s": round(setup_s, 1),
                   "timed_loop_wall_s": round(wall, 3)},
     }
+    if two_call is not None:
+        out["two_call_variant"] = two_call
     if path.index is not None:
         out["draft_scan_variant"] = time_scan_variant(pk, loop, w, flush_l2)
     if not args.no_sample:
@@ -463,6 +524,28 @@ def run_ours(args, ws_, rank, local):
     if rank == 0 and ws_ == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline_from_loop(loop, path, w)
     return out
+
+
+def time_two_call_variant(pk, loop, w, flush_l2, steps=64, warm=3):
+    """The same loop with the drafting and the verification as two calls per step
+    (pldp_draft_step with the token index, then pldp_verify_greedy), per-call CUDA
+    events as in the timed loop, from the loop's initial state."""
+    loop.reset()
+    path = Path(pk, loop, fused=True, index=True)
+    path.build_index()
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for s in range(warm + steps):
+        loop.step_inputs(s)
+        flush_l2(s)
+        path.run(evs[s - warm] if s >= warm else None)
+    torch.cuda.synchronize()
+    d = np.array([e[0].elapsed_time(e[1]) for e in evs]) * 1e3
+    v = np.array([e[1].elapsed_time(e[2]) for e in evs]) * 1e3
+    return {"steps": steps, "us_per_step": round(float(d.sum() + v.sum()) / steps, 2),
+            "draft_us": round(float(d.mean()), 2), "verify_us": round(float(v.mean()), 2),
+            "draft_us_p50_p90": [round(float(np.percentile(d, 50)), 2), round(float(np.percentile(d, 90)), 2)],
+            "verify_us_p50_p90": [round(float(np.percentile(v, 50)), 2), round(float(np.percentile(v, 90)), 2)],
+            "path": "pldp_draft_step with the token index + pldp_verify_greedy"}
 
 
 def time_scan_variant(pk, loop, w, flush_l2, steps=64, warm=3):
@@ -598,6 +681,7 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     w, dev = loop.w, loop.device
     loop.reset()
     path.build_index()                  # the contexts were cut back: index them again
+    path.prime(0)
     B, K1 = w.B, w.K + 1
     h_logits = torch.empty(loop.logits.shape, dtype=loop.logits.dtype, pin_memory=True)
     h_A = torch.empty(loop.A.shape, dtype=loop.A.dtype, pin_memory=True)
@@ -610,7 +694,7 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     times = []
     steps = K_steps
     for s in range(W_steps + steps):
-        loop.step_inputs(s)                       # make this step's inputs ...
+        path.inputs(s)                            # make this step's inputs ...
         pos = (loop.seq_len.long()[:, None] - 1 + ar[None]).clamp(max=loop.T_cap - 1)
         h_logits.copy_(loop.logits)               # ... and park them in pinned host memory
         h_A.copy_(loop.A)
@@ -677,7 +761,8 @@ def cpu_baseline_from_loop(loop, path, w, budget_s=20.0, nseq=64, max_steps=192)
     import oracle
     oracle.build()
     loop.reset()
-    path.build_index()                  # the contexts were cut back: index them again
+    path = Path(path.pk, loop, fused=True, index=True)   # advances the GPU loop: two calls per step
+    path.build_index()
     nseq = min(nseq, w.B)
     max_steps = min(max_steps, loop.steps)
     Hs = np.zeros((nseq, loop.T_cap, w.d), np.uint16)       # zero pages until written
