@@ -688,12 +688,15 @@ __device__ __forceinline__ bool index_insert(const IndexView& ix, int b, int64_t
 // The indexed drafting of sequence b by the whole CTA, for context length L.
 // RD: how ids are read -- CoherentIds when this kernel has just appended to the
 // context (verification fused in front), else through the read-only cache.
-template <typename TH, bool IVEC, typename RD>
+// PRE: the indexed length is il_in and the ids it starts from -- is.newtok (the
+// positions appended since, when they fit) and is.suf (x_t, x_{t-1}, ...) -- are
+// already in shared memory, written before the CTA's last barrier.
+template <typename TH, bool IVEC, typename RD, bool PRE = false>
 __device__ __forceinline__ void index_draft(const DraftParams& p, const IndexView& ix, int b, int64_t L,
-                                            StepShared& sh, IndexShared& is) {
+                                            StepShared& sh, IndexShared& is, int64_t il_in = 0) {
     constexpr bool HAS_H = !std::is_same<TH, NoHidden>::value;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int64_t il = ix.ilen[b];
+    const int64_t il = PRE ? il_in : static_cast<int64_t>(ix.ilen[b]);
     const bool valid = L >= 0 && L <= p.T_cap;
     const int64_t t = L - 1;
     const int32_t* row = p.ids + static_cast<int64_t>(b) * p.ids_stride;
@@ -733,8 +736,10 @@ __device__ __forceinline__ void index_draft(const DraftParams& p, const IndexVie
     if (tid == 0 && HAS_H && t >= 2)                              // H_{t-1}: every candidate's score reads it
         prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (t - 1) * p.d) * h_es,
                          static_cast<uint32_t>(p.d * h_es));
-    if (small && tid < nnew) is.newtok[tid] = RD::one(row + il + tid);
-    if (tid < PLDP_MAX_NGRAM) is.suf[tid] = (tid < p.ngram_max && t - tid >= 0) ? RD::one(row + t - tid) : 0;
+    if (!PRE) {
+        if (small && tid < nnew) is.newtok[tid] = RD::one(row + il + tid);
+        if (tid < PLDP_MAX_NGRAM) is.suf[tid] = (tid < p.ngram_max && t - tid >= 0) ? RD::one(row + t - tid) : 0;
+    }
     __syncthreads();
     const int32_t xt = is.suf[0];
     const bool lookup = small && t >= 1 && xt >= 0 && xt < ix.V;
@@ -1021,14 +1026,37 @@ __global__ void __launch_bounds__(kThreads, 1) verify_draft_kernel(const VerifyA
     __shared__ long long L_after;
     pdl_enter();                                                  // the pass's row keys are final
     const int b = blockIdx.x;
+    const int64_t il = ix.ilen[b];                                // does not depend on the verification
     if (threadIdx.x < 32) {
-        const int64_t L1 = finish_sequence(va, b, static_cast<int>(threadIdx.x),
-                                           KeyTokens{va.row_keys + static_cast<int64_t>(b) * (va.K + 1)});
-        if (threadIdx.x == 0) L_after = L1;
+        const int lane = static_cast<int>(threadIdx.x);
+        FinishOut fo;
+        const int64_t L1 = finish_sequence(va, b, lane, KeyTokens{va.row_keys + static_cast<int64_t>(b) * (va.K + 1)},
+                                           &fo);
+        if (lane == 0) L_after = L1;
+        // The drafting's first reads come from what the finish holds: the ids appended
+        // since the index was brought up to date (il .. t-1) and the suffix x_t, x_{t-1},
+        // ...; positions the finish wrote come from its draft and bonus, older ones from L2.
+        if (L1 >= 0 && L1 <= p.T_cap) {
+            const int64_t t = L1 - 1;
+            const int64_t L0 = fo.appended ? L1 - fo.n - 1 : L1;  // the first appended position
+            const int32_t* row = p.ids + static_cast<int64_t>(b) * p.ids_stride;
+            const int32_t* dr = va.draft + static_cast<int64_t>(b) * va.K;
+            auto tok = [&](int64_t q) -> int32_t {
+                if (q >= L0) return q - L0 < fo.n ? dr[q - L0] : fo.bonus;
+                return __ldcg(row + q);
+            };
+            const bool usable = il >= 0 && il <= t;
+            const int64_t nnew = usable ? t - il : 0;
+            if (usable && nnew <= kNewCap)
+                for (int64_t k = lane; k < nnew; k += 32) is.newtok[k] = tok(il + k);
+            if (lane < PLDP_MAX_NGRAM) is.suf[lane] = (lane < p.ngram_max && t - lane >= 0) ? tok(t - lane) : 0;
+        } else if (lane < PLDP_MAX_NGRAM) {
+            is.suf[lane] = 0;                                     // no last token (as the drafting reads it)
+        }
     }
     __syncthreads();                                              // the append is visible to the whole CTA
     const int64_t L = L_after >= 0 ? static_cast<int64_t>(L_after) : static_cast<int64_t>(__ldcg(p.seq_len + b));
-    index_draft<TH, IVEC, CoherentIds>(p, ix, b, L, sh, is);
+    index_draft<TH, IVEC, CoherentIds, true>(p, ix, b, L, sh, is, il);
 }
 
 // Index build: positions 0 .. seq_len-2 of every sequence.

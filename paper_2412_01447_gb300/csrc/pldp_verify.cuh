@@ -40,6 +40,13 @@ struct SharedTokens {
     __device__ __forceinline__ void release(int, int) const {}
 };
 
+// What the finish decided, for a caller that continues with the extended context.
+struct FinishOut {
+    int n;          // accepted draft tokens
+    int bonus;      // the token emitted after them
+    bool appended;  // draft[0..n-1] and bonus were written at positions L .. L+n
+};
+
 // Accept/bonus/append for sequence b, by one warp, once its K+1 target tokens are
 // final.  Everything it reads is requested up front (one round trip when K < 32).
 // Sec. 4.4: n = first i < d with draft_i != target_i (else d), bonus = target_n.
@@ -47,7 +54,8 @@ struct SharedTokens {
 // tokens were appended, L when they were not (capacity, no ids), -1 when seq_len
 // is absent or out of range.
 template <typename Src>
-__device__ int64_t finish_sequence(const VerifyArgs& a, int64_t b, int lane, const Src& src) {
+__device__ int64_t finish_sequence(const VerifyArgs& a, int64_t b, int lane, const Src& src,
+                                   FinishOut* out = nullptr) {
     const int K1 = a.K + 1;
     const int d_in = a.draft_len[b];
     const int64_t L = a.seq_len ? a.seq_len[b] : 0;
@@ -106,6 +114,11 @@ __device__ int64_t finish_sequence(const VerifyArgs& a, int64_t b, int lane, con
     }
     if (lane == 0) {
         if (a.status && st) a.status[b] |= st;
+    }
+    if (out) {
+        out->n = n;
+        out->bonus = bonus;
+        out->appended = a.seq_len && a.ids && L_after == L + n + 1;
     }
     return L_after;
 }
