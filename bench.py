@@ -445,9 +445,8 @@ def run_ours(args, ws_, rank, local):
         ver_src = "verify_greedy (argmax pass + finish) per call in the timed loop"
     achieved = ver_bytes / ver_s / 1e9
     csrc = os.path.join(ROOT, "paper_2412_01447_gb300", "csrc")
-    traffic = profiled_traffic([os.path.join(csrc, "verify.cu"), os.path.join(csrc, "pldp_internal.cuh"),
-                                os.path.join(csrc, "pldp_verify.cuh")],
-                               "verify_greedy_c5.md")
+    traffic = profiled_traffic([os.path.join(csrc, "verify.cu"), os.path.join(csrc, "pldp_internal.cuh")],
+                               "verify_greedy_c5.md")            # the argmax pass's sources
     if path.index is not None:
         step_bytes_total = by["verify_greedy"] + by["draft_index"]
     else:
