@@ -140,3 +140,66 @@ def test_graph_capture_replays_the_step(lib, fused):
             assert np.array_equal(ga[k], gb[k]), (s, k)
         assert torch.equal(a.ids, b.ids) and torch.equal(a.seq_len, b.seq_len)
         assert int(buf_b.ws.count_nonzero()) == 0
+
+
+def test_decode_loop_c5_verify_draft(lib):
+    """The benchmark's configuration: the full c5 loop with one pldp_verify_greedy_draft
+    call per step (verification, then the next draft with the token index).  Each step
+    is compared with the oracle: verification of the GPU's draft on the pre-step state,
+    then candidates, rankings (sampled sequences) and draft on the state it leaves."""
+    import paper_2412_01447_gb300 as pk
+    w = wl.CONFIGS["c5"]
+    steps = 4
+    loop = wl.DecodeLoop(w, steps=steps, device=DEV)
+    B, K, C = w.B, w.K, w.C_cap
+    ng = (w.ngram_min, w.ngram_max)
+    buf = Buffers(B, K, w.V, C, DEV)
+    index = torch.empty(pk.pldp_index_size(B, w.V), dtype=torch.uint8, device=DEV)
+    pk.pldp_index_build(loop.ids, loop.seq_len, w.V, index)
+    sel = _sample(B, 6, 7)
+    Hs = host(loop.H[sel])
+    kw = dict(H=loop.H, best_h=buf.best_h, h_scores=buf.scores_h, best_h_score=buf.bscore_h, A=loop.A,
+              best_a=buf.best_a, a_scores=buf.scores_a, best_a_score=buf.bscore_a, draft_from="hidden",
+              status=buf.status)
+
+    def check_draft(ids0, L0, As):
+        g = snapshot(buf)
+        o_cand, o_cnt, o_ml, _ = oracle.find_candidates(ids0, L0, ng[0], ng[1], C)
+        assert np.array_equal(g["cnt"], o_cnt) and np.array_equal(g["ml"], o_ml)
+        for b in range(B):
+            n = min(o_cnt[b], C)
+            assert np.array_equal(g["cand"][b, :n], o_cand[b, :n]), b
+        o_s, o_b, _ = oracle.rank_hidden(Hs, L0[sel], o_cand[sel], o_cnt[sel])
+        check_scores(g["scores_h"][sel], o_s, o_cnt[sel], C)
+        check_choice(g["best_h"][sel], o_b, o_s, o_cand[sel], o_cnt[sel], C)
+        o_sa, o_ba, _ = oracle.rank_attention(As, L0[sel], o_cand[sel], o_cnt[sel])
+        check_scores(g["scores_a"][sel], o_sa, o_cnt[sel], C)
+        assert np.array_equal(g["best_a"][sel], o_ba)
+        o_d, o_dl = oracle.extract_draft(ids0, L0, g["best_h"], K)
+        assert np.array_equal(g["draft"], o_d) and np.array_equal(g["dlen"], o_dl)
+        return g
+
+    loop.step_inputs(0)                       # the first draft, as a prefill would make it
+    pk.pldp_draft_step(loop.ids, loop.seq_len, ng[0], ng[1], buf.cand, buf.cnt, buf.ml, K, buf.draft, buf.dlen,
+                       None, index=index, V=w.V, **kw)
+    check_draft(host(loop.ids), host(loop.seq_len), host(loop.A[sel]))
+    for s in range(steps):
+        loop.step_inputs_next(s, buf.draft, buf.dlen)
+        ids0, L0, lg = host(loop.ids), host(loop.seq_len), host(loop.logits)
+        d0, dl0 = host(buf.draft), host(buf.dlen)
+        As = host(loop.A[sel])
+        pk.pldp_verify_greedy_draft(loop.logits, buf.draft, buf.dlen, buf.acc, buf.nxt, buf.ws, loop.ids,
+                                    loop.seq_len, ng[0], ng[1], buf.cand, buf.cnt, buf.ml, buf.draft, buf.dlen,
+                                    index, argmax=buf.argmax, kv_keep_len=buf.kv, **kw)
+        ids_o, L_o = ids0.copy(), L0.copy()
+        o = oracle.verify_greedy(lg, d0, dl0, ids=ids_o, seq_len=L_o, kv_keep=True)
+        g = check_draft(ids_o, L_o, As)       # the next draft, on the state verification left
+        assert np.array_equal(g["argmax"], o["argmax"]) and np.array_equal(g["acc"], o["accept_len"])
+        assert np.array_equal(g["nxt"], o["next_token"]) and np.array_equal(g["kv"], o["kv_keep_len"])
+        assert np.array_equal(host(loop.ids), ids_o) and np.array_equal(host(loop.seq_len), L_o)
+        assert (g["status"] == 0).all()
+    L = host(loop.seq_len)
+    ids, gt = host(loop.ids), loop.gt_host
+    for b in range(B):
+        assert np.array_equal(ids[b, :L[b]], gt[b, :L[b]]), b
+    assert (L - w.T).mean() > steps * 1.5
