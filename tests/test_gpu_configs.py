@@ -142,6 +142,52 @@ def test_graph_capture_replays_the_step(lib, fused):
         assert int(buf_b.ws.count_nonzero()) == 0
 
 
+def test_graph_capture_replays_verify_draft(lib):
+    """One pldp_verify_greedy_draft call captured in a CUDA graph and replayed step after
+    step gives the eager call's results, with the token index kept up to date by the
+    replays; the verify workspace returns to zero between replays."""
+    import paper_2412_01447_gb300 as pk
+    w = wl.CONFIGS["c5"].replace(B=16, prompt_len=3000, out_len=1000, V=32000, d=1024)
+    ng = (w.ngram_min, w.ngram_max)
+    loops = [wl.DecodeLoop(w, steps=6, device=DEV) for _ in range(2)]
+    bufs = [Buffers(w.B, w.K, w.V, w.C_cap, DEV) for _ in range(2)]
+    idx = [torch.empty(pk.pldp_index_size(w.B, w.V), dtype=torch.uint8, device=DEV) for _ in range(2)]
+
+    def kw(lp, buf):
+        return dict(H=lp.H, best_h=buf.best_h, A=lp.A, best_a=buf.best_a, draft_from="hidden", status=buf.status)
+
+    def call(i, stream=None):
+        lp, buf = loops[i], bufs[i]
+        pk.pldp_verify_greedy_draft(lp.logits, buf.draft, buf.dlen, buf.acc, buf.nxt, buf.ws, lp.ids, lp.seq_len,
+                                    ng[0], ng[1], buf.cand, buf.cnt, buf.ml, buf.draft, buf.dlen, idx[i],
+                                    argmax=buf.argmax, kv_keep_len=buf.kv, stream=stream, **kw(lp, buf))
+
+    for i in range(2):                        # the index and the first draft of each copy
+        lp, buf = loops[i], bufs[i]
+        pk.pldp_index_build(lp.ids, lp.seq_len, w.V, idx[i])
+        lp.step_inputs(0)
+        pk.pldp_draft_step(lp.ids, lp.seq_len, ng[0], ng[1], buf.cand, buf.cnt, buf.ml, w.K, buf.draft, buf.dlen,
+                           None, index=idx[i], V=w.V, **kw(lp, buf))
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream()
+    stream.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        call(1, stream=torch.cuda.current_stream())
+    for s in range(6):
+        for i in range(2):
+            loops[i].step_inputs_next(s, bufs[i].draft, bufs[i].dlen)
+        call(0)
+        graph.replay()
+        torch.cuda.synchronize()
+        ga, gb = snapshot(bufs[0]), snapshot(bufs[1])
+        for k in ("cnt", "ml", "best_h", "best_a", "draft", "dlen", "acc", "nxt", "argmax", "kv", "status"):
+            assert np.array_equal(ga[k], gb[k]), (s, k)
+        assert torch.equal(loops[0].ids, loops[1].ids) and torch.equal(loops[0].seq_len, loops[1].seq_len)
+        assert torch.equal(idx[0][:4 * w.B], idx[1][:4 * w.B])
+        assert int(bufs[1].ws.count_nonzero()) == 0
+
+
 def test_decode_loop_c5_verify_draft(lib):
     """The benchmark's configuration: the full c5 loop with one pldp_verify_greedy_draft
     call per step (verification, then the next draft with the token index).  Each step
