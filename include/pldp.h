@@ -240,7 +240,7 @@ PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
  *                        [0, V).  With it, a step looks up the occurrences of
  *                        x_t instead of scanning the context, and appends the
  *                        positions added since the last step; results are the
- *                        same as without it (a token with more than 7 earlier
+ *                        same as without it (a token with more than 15 earlier
  *                        occurrences, or a sequence whose index is unusable,
  *                        is scanned).  The index must only ever see the
  *                        contexts grow by appending: a sequence whose length
@@ -302,12 +302,12 @@ PLDP_API size_t pldp_draft_workspace_size(int B);
  * The incremental token index of pldp_draft_step (no counterpart in the paper:
  * it is a way to find the occurrences of Eq. 1 without rescanning the context).
  * Per sequence and token it holds the number of occurrences among the indexed
- * positions and up to 7 of them (one 32-byte entry); per sequence the number of
+ * positions and up to 15 of them (one 64-byte entry); per sequence the number of
  * positions indexed.
  * pldp_index_build clears `index` and indexes positions 0 .. seq_len[b]-2 of
  * every sequence (all but the last token, which the next draft step looks up).
  * Token ids outside [0, V) mark that sequence's index unusable (TOKEN_RANGE);
- * seq_len outside [0, T_cap] too (SEQ_LEN).  Memory: about B * V * 32 bytes.
+ * seq_len outside [0, T_cap] too (SEQ_LEN).  Memory: about B * V * 64 bytes.
  */
 PLDP_API size_t pldp_index_size(int B, int V);
 PLDP_API pldp_status pldp_index_build(const int32_t* ids, int64_t ids_stride, const int32_t* seq_len,
