@@ -1,8 +1,15 @@
 // pldp_draft_step: the drafting half of a PLD+ step -- candidate search (Eq. 1
 // with the longest-suffix n-gram rule), ranking by hidden states (Eq. 3) and/or
-// by attentions (Eq. 2), and draft extraction (Sec. 4.3) -- in one launch.
+// by attentions (Eq. 2), and draft extraction (Sec. 4.3) -- in one launch; and
+// pldp_verify_greedy_draft: greedy verification (Sec. 4.4) followed by the next
+// step's drafting.  Three kernels:
+//  * draft_step_kernel scans the contexts (below);
+//  * draft_index_kernel looks the occurrences up in the incremental token index
+//    (further down), one CTA per sequence;
+//  * verify_draft_kernel runs the finish of greedy verification and then the
+//    indexed drafting in the same CTA.
 //
-// A flat grid of (chunk, sequence) CTAs.  Each CTA
+// The scanning kernel: a flat grid of (chunk, sequence) CTAs.  Each CTA
 //  1. streams its chunk of the context with 16-byte loads and, for every
 //     occurrence j of x_t, takes the suffix-match length m and a slot in a short
 //     per-sequence list held in the workspace;
