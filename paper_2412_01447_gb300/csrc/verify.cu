@@ -474,8 +474,16 @@ __device__ __forceinline__ float warp_max_f(float v) {
     return v;
 }
 
+// The float of an ordered key (inverse of ordered_key).
+__device__ __forceinline__ float ordered_value(uint32_t o) {
+    return __uint_as_float((o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o);
+}
+
 // 1. per-piece (max, sum of weights).  Units u = row * npieces + piece, warp w of W
 // takes units w, w + W, ...; piece k of row r covers elements [k P, min((k+1) P, V)).
+// Each lane sums its elements' weights against its own maximum m, so the
+// exponentials do not wait for the piece's maximum M (one redux over ordered
+// keys); the lane's sum is then scaled by 2^((m - M) / T log2 e) and the warp adds.
 template <typename T, bool VEC>
 __global__ void __launch_bounds__(kThreads, VEC ? kPassBlocksPerSm : 4)
 sample_stats_kernel(const T* __restrict__ logits, int64_t V, int64_t rows, int npieces, int P, float c,
@@ -504,18 +512,20 @@ sample_stats_kernel(const T* __restrict__ logits, int64_t V, int64_t rows, int n
 #pragma unroll
             for (int q = 0; q < kSegLoads; ++q)
                 if (static_cast<int64_t>(lane + 32 * q) * VW < n) m = fmaxf(m, vmax(raw[q], T()));
-            M = warp_max_f(m);
-            if (M > -INFINITY) {
-                const float mc = M * c;
+            if (m > -INFINITY) {
+                const float mc = m * c;
 #pragma unroll
                 for (int q = 0; q < kSegLoads; ++q) {
                     if (static_cast<int64_t>(lane + 32 * q) * VW >= n) continue;
                     float e[8];
                     unpack(raw[q], e, T());
 #pragma unroll
-                    for (int j = 0; j < VW; ++j) sum += ex2_approx(fmaf(e[j], c, -mc));
+                    for (int j = 0; j < VW; j += 2)                // pairs: half the dependent adds
+                        sum += ex2_approx(fmaf(e[j], c, -mc)) + ex2_approx(fmaf(e[j + 1], c, -mc));
                 }
             }
+            M = ordered_value(__reduce_max_sync(0xFFFFFFFFu, ordered_key(m)));
+            if (sum > 0.f) sum *= ex2_approx((m - M) * c);
         } else {
             constexpr int PER = static_cast<int>(kPieceBytes / sizeof(T)) / 32;
             float x[PER];
@@ -525,13 +535,14 @@ sample_stats_kernel(const T* __restrict__ logits, int64_t V, int64_t rows, int n
                 x[q] = ei < n ? to_f32(piece[ei]) : -INFINITY;
                 m = fmaxf(m, x[q]);
             }
-            M = warp_max_f(m);
-            if (M > -INFINITY) {
-                const float mc = M * c;
+            if (m > -INFINITY) {
+                const float mc = m * c;
 #pragma unroll
                 for (int q = 0; q < PER; ++q)
                     if (x[q] > -INFINITY) sum += ex2_approx(fmaf(x[q], c, -mc));
             }
+            M = ordered_value(__reduce_max_sync(0xFFFFFFFFu, ordered_key(m)));
+            if (sum > 0.f) sum *= ex2_approx((m - M) * c);
         }
         sum = warp_sum(sum);
         if (lane == 0) stats[u] = make_float2(M, sum);
@@ -645,16 +656,18 @@ __device__ int sample_row(const T* __restrict__ logits, const SampleArgs& a, int
     if (!(u >= 0.f)) u = 0.f;
     if (u >= 1.f) u = __uint_as_float(0x3F7FFFFFu);               // largest float below 1
     PiecePick pk = pick_piece(st, np, a.c, u, lane);
-    if (pk.k < 0) {                                               // rounding: the last piece with weight
+    float f;                                                      // fraction of the piece to pass
+    if (pk.k < 0) {
+        // u Z rounded up to Z (u within 2^-24 of 1): the end of the last piece with weight
         int k = np - 1;
         for (; k > 0; --k)
             if (__ldcg(st + k).y > 0.f) break;
         pk.k = k;
-        pk.before = pk.target;
-        pk.w = 1.f;
         pk.Mk = __ldcg(st + k).x;
+        f = 1.f;
+    } else {
+        f = pk.w > 0.f ? (pk.target - pk.before) / pk.w : 0.f;
     }
-    float f = pk.w > 0.f ? (pk.target - pk.before) / pk.w : 0.f;  // fraction of the piece to pass
     f = fminf(fmaxf(f, 0.f), __uint_as_float(0x3F7FFFFFu));
     const int ks = pk.k;
     // the piece, lane L holding its elements [L E, (L+1) E) in index order
@@ -724,6 +737,12 @@ __global__ void __launch_bounds__(32 * kFinishWarps, 1) sample_finish_kernel(con
     const int64_t b = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int K1 = a.v.K + 1;
+    if (warp == kFinishWarps - 1) {                              // what the finish reads, on its way to L1
+        for (int i = lane; i < a.v.K; i += 32)
+            asm volatile("prefetch.global.L1 [%0];" ::"l"(a.v.draft + b * a.v.K + i));
+        if (lane == 0) asm volatile("prefetch.global.L1 [%0];" ::"l"(a.v.draft_len + b));
+        if (lane == 1 && a.v.seq_len) asm volatile("prefetch.global.L1 [%0];" ::"l"(a.v.seq_len + b));
+    }
     for (int i = warp; i < K1; i += kFinishWarps) {
         const int y = sample_row<T, VEC>(logits, a, b * K1 + i, lane);
         if (lane == 0) draws[i] = y;
