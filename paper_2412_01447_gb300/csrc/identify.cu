@@ -14,7 +14,9 @@
 //     (ov << 32 | ~j).
 //  2. The R rows of query p-1 are reduced to their first maximum, one warp per
 //     row (16-byte streaming loads where rows allow, packed (value, ~key)
-//     maxima), and a row whose maximum is at r* adds one to counts[r].
+//     maxima), and a row whose maximum is at r* adds one to counts[r].  The rows
+//     are read first (they do not depend on r*, and they are the bandwidth); the
+//     latency-bound scan of step 1 follows.
 // pldp_top_heads: one CTA ranks the counts and writes the k rows with the most
 // (ties to the smaller row index) -- the row_idx of pldp_rank_attention.
 #include "pldp_internal.cuh"
@@ -59,7 +61,8 @@ __device__ __forceinline__ unsigned long long row_first_max_vec(const T* row, in
             bi = k;
         }
     }
-    return bi < 0 ? 0ull : warp_max_u64(pack_key(bv, static_cast<uint32_t>(bi)));
+    // every lane takes part in the reduction; a lane without elements offers 0 (no key)
+    return warp_max_u64(bi < 0 ? 0ull : pack_key(bv, static_cast<uint32_t>(bi)));
 }
 
 template <typename T>
@@ -73,7 +76,8 @@ __device__ __forceinline__ unsigned long long row_first_max_elem(const T* row, i
             bi = k;
         }
     }
-    return bi < 0 ? 0ull : warp_max_u64(pack_key(bv, static_cast<uint32_t>(bi)));
+    // every lane takes part in the reduction; a lane without elements offers 0 (no key)
+    return warp_max_u64(bi < 0 ? 0ull : pack_key(bv, static_cast<uint32_t>(bi)));
 }
 
 template <bool VEC>
@@ -115,6 +119,18 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
     }
     const int32_t* x = ids + static_cast<int64_t>(b) * ids_stride;
     const int32_t xp = __ldg(x + p);
+    // 2 (first: it does not depend on r*, and it is the bandwidth). The first maximum of
+    // each of this CTA's rows, two rows per warp.
+    constexpr int RW = kRowsPerCta / kWarps;
+    const size_t es = a_bf16 ? 2 : 4;
+    const char* ab = static_cast<const char*>(A) + static_cast<int64_t>(b) * seq_stride * es;
+    const int r1 = r0 + kRowsPerCta < R ? r0 + kRowsPerCta : R;
+    unsigned long long rk[RW];
+#pragma unroll
+    for (int i = 0; i < RW; ++i) {
+        const int r = r0 + warp + i * kWarps;
+        rk[i] = r < r1 ? row_first_max<VEC>(ab + static_cast<int64_t>(r) * row_stride * es, a_bf16, p, lane) : 0ull;
+    }
     // 1. the copy source r*: positions [0, p) in tiles, eight loads in flight per thread
     unsigned long long best = 0;
     constexpr int U = 8;
@@ -166,13 +182,11 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
     const int64_t rs = best ? static_cast<int64_t>(0xFFFFFFFFu - static_cast<uint32_t>(best & 0xFFFFFFFFull)) : -1;
     if (tid == 0 && blockIdx.y == 0 && r_star) r_star[b] = static_cast<int32_t>(rs);
     if (rs < 0) return;
-    // 2. the rows whose maximum is at r*
-    const size_t es = a_bf16 ? 2 : 4;
-    const char* ab = static_cast<const char*>(A) + static_cast<int64_t>(b) * seq_stride * es;
-    const int r1 = r0 + kRowsPerCta < R ? r0 + kRowsPerCta : R;
-    for (int r = r0 + warp; r < r1; r += kWarps) {
-        const unsigned long long k = row_first_max<VEC>(ab + static_cast<int64_t>(r) * row_stride * es, a_bf16, p, lane);
-        if (lane == 0 && k && static_cast<int64_t>(key_index(k)) == rs) atomicAdd(counts + r, 1u);
+    // the rows whose maximum is at r* count
+#pragma unroll
+    for (int i = 0; i < RW; ++i) {
+        const int r = r0 + warp + i * kWarps;
+        if (lane == 0 && r < r1 && rk[i] && static_cast<int64_t>(key_index(rk[i])) == rs) atomicAdd(counts + r, 1u);
     }
 }
 
