@@ -490,6 +490,7 @@ PLDP_API size_t pldp_verify_workspace_size(int B, int K, int V);
  * attention peaks.  Run it over many observations, then keep the rows with the
  * most counts (pldp_top_heads).
  *
+ *  B          observations, at most 65535 (else PLDP_ERR_UNSUPPORTED).
  *  ids, ids_stride, T_cap   int32 contexts [B, ids_stride], T_cap <= ids_stride.
  *  pos        int32 [B]; outside [1, T_cap - 1]: SEQ_LEN, nothing counted.
  *  max_suffix >= 1: cap on ov(j).

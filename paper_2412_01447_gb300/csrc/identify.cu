@@ -6,7 +6,7 @@
 // that over many observations and keeping the rows with the most counts gives
 // G* x L*.
 //
-// pldp_identify_heads: a (observation, group of kRowsPerCta rows) grid of CTAs.
+// pldp_identify_heads: a (group of kRowsPerCta rows, observation) grid of CTAs.
 //  1. The context before x_p is scanned for x_p (by every CTA of the observation:
 //     4 bytes per position against 2 R bytes of attention); every occurrence j gets its
 //     overlap ov(j) (the length of the common suffix of x[..j] and x[..p]) and
@@ -27,7 +27,7 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxTopRows = 8192;   // counts staged in shared memory by pldp_top_heads
-constexpr int kRowsPerCta = 16;     // attention rows per CTA (two per warp)
+constexpr int kRowsPerCta = 8;      // attention rows per CTA (one per warp)
 
 // The first maximum of elements [0, n) of one attention row, by one warp, as a
 // packed (value, ~key) key.  Each lane keeps a running (max, first key) over its
@@ -106,12 +106,12 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
                       int32_t* __restrict__ r_star, uint32_t* __restrict__ status) {
     __shared__ unsigned long long wkey[kWarps];
     pdl_enter();
-    const int b = blockIdx.x;
-    const int r0 = blockIdx.y * kRowsPerCta;
+    const int b = blockIdx.y;                                     // the CTAs of one observation are adjacent:
+    const int r0 = blockIdx.x * kRowsPerCta;                      // its ids are read once from DRAM, then L2
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int64_t p = pos[b];
     if (p < 1 || p >= T_cap) {
-        if (tid == 0 && blockIdx.y == 0) {
+        if (tid == 0 && blockIdx.x == 0) {
             if (r_star) r_star[b] = -1;
             if (status) atomicOr(status + b, PLDP_ST_SEQ_LEN);
         }
@@ -180,7 +180,7 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
 #pragma unroll
     for (int w = 0; w < kWarps; ++w) best = wkey[w] > best ? wkey[w] : best;
     const int64_t rs = best ? static_cast<int64_t>(0xFFFFFFFFu - static_cast<uint32_t>(best & 0xFFFFFFFFull)) : -1;
-    if (tid == 0 && blockIdx.y == 0 && r_star) r_star[b] = static_cast<int32_t>(rs);
+    if (tid == 0 && blockIdx.x == 0 && r_star) r_star[b] = static_cast<int32_t>(rs);
     if (rs < 0) return;
     // the rows whose maximum is at r* count
 #pragma unroll
@@ -226,6 +226,7 @@ extern "C" PLDP_API pldp_status pldp_identify_heads(const int32_t* ids, int64_t 
     if (row_stride < T_cap) return fail(PLDP_ERR_INVALID_ARG, "identify_heads: row_stride < T_cap");
     if (seq_stride < static_cast<int64_t>(R) * row_stride)
         return fail(PLDP_ERR_INVALID_ARG, "identify_heads: seq_stride < R*row_stride");
+    if (B > 65535) return fail(PLDP_ERR_UNSUPPORTED, "identify_heads: B > 65535");
     if (B == 0) return PLDP_OK;
     if (!ids || !pos || !A || !counts) return fail(PLDP_ERR_INVALID_ARG, "identify_heads: null pointer");
     const size_t es = dtype == PLDP_F32 ? 4 : 2;
@@ -233,7 +234,7 @@ extern "C" PLDP_API pldp_status pldp_identify_heads(const int32_t* ids, int64_t 
     const bool bf16 = dtype == PLDP_BF16;
     const bool ivec = aligned16(ids) && ids_stride % 4 == 0;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const dim3 grid(static_cast<unsigned>(B), static_cast<unsigned>((R + kRowsPerCta - 1) / kRowsPerCta));
+    const dim3 grid(static_cast<unsigned>((R + kRowsPerCta - 1) / kRowsPerCta), static_cast<unsigned>(B));
     cudaError_t e;
 #define PLDP_IDENTIFY_LAUNCH(V, I)                                                                          \
     launch_pdl(identify_heads_kernel<V, I>, grid, dim3(kThreads), 0, s, 0, ids, ids_stride, pos, T_cap, max_suffix, \
