@@ -102,16 +102,28 @@ def _planted_logits(draft, dlen, V, gen, accept):
     (4096, 3000, 16, "both", True), (8000, 300, 12, "hidden", False), (2048, 20, 10, "attention", True),
     (30000, 20000, 8, "both", False)])
 def test_verify_draft_equals_separate_calls(lib, T, V, B, mode, shared):
-    rng = np.random.default_rng(T + V)
+    _verify_draft_case(T, V, B, mode, shared, K=10, C=64, ngram=(1, 3), dt=torch.bfloat16)
+
+
+@pytest.mark.parametrize("K,C,ngram,dt", [(40, 64, (1, 3), torch.bfloat16), (6, 2, (2, 4), torch.float32),
+                                          (33, 8, (1, 8), torch.float32)])
+def test_verify_draft_other_shapes(lib, K, C, ngram, dt):
+    """Drafts longer than the staged window (K > 32), short candidate lists, other
+    n-gram ranges, and fp32 hidden rows and attention values."""
+    _verify_draft_case(6000, 2000, 12, "both", True, K=K, C=C, ngram=ngram, dt=dt)
+
+
+def _verify_draft_case(T, V, B, mode, shared, K, C, ngram, dt):
+    rng = np.random.default_rng(T + V + K)
     gen = torch.Generator(device=DEV).manual_seed(T + 3)
-    K, C, d, R, ngram = 10, 64, 128, 12, (1, 3)
-    T_cap = T + 120
+    d, R = 128, 12
+    T_cap = T + 12 * (K + 1)
     ids = rng.integers(0, V, size=(B, T_cap)).astype(np.int32)
     lens = rng.integers(2, T + 1, size=B)
-    lens[0] = T_cap - 15                      # runs out of room within a few steps (CAPACITY)
+    lens[0] = T_cap - 1                       # full within two steps (CAPACITY)
     lens[1] = T_cap + 5                       # out of range throughout (SEQ_LEN)
-    H = torch.randn((B, T_cap, d), generator=gen, device=DEV).to(torch.bfloat16) if mode != "attention" else None
-    A = torch.rand((B, R, T_cap), generator=gen, device=DEV).to(torch.bfloat16) if mode != "hidden" else None
+    H = torch.randn((B, T_cap, d), generator=gen, device=DEV).to(dt) if mode != "attention" else None
+    A = torch.rand((B, R, T_cap), generator=gen, device=DEV).to(dt) if mode != "hidden" else None
     draft_from = "attention" if mode == "attention" else "hidden"
     ids_a, L_a = i32(ids), i32(lens)
     ids_b, L_b = ids_a.clone(), L_a.clone()
