@@ -122,6 +122,8 @@ def _verify_draft_case(T, V, B, mode, shared, K, C, ngram, dt):
     lens = rng.integers(2, T + 1, size=B)
     lens[0] = T_cap - 1                       # full within two steps (CAPACITY)
     lens[1] = T_cap + 5                       # out of range throughout (SEQ_LEN)
+    lens[3] = 1                               # x_t alone: no H_{t-1}, nothing before it
+    lens[4] = 0                               # empty: verification refuses it (SEQ_LEN), drafting finds nothing
     H = torch.randn((B, T_cap, d), generator=gen, device=DEV).to(dt) if mode != "attention" else None
     A = torch.rand((B, R, T_cap), generator=gen, device=DEV).to(dt) if mode != "hidden" else None
     draft_from = "attention" if mode == "attention" else "hidden"
@@ -148,6 +150,7 @@ def _verify_draft_case(T, V, B, mode, shared, K, C, ngram, dt):
         _same_index(ix_a, ix_b, B, V)
     st = host(b_.status).view(np.uint32)
     assert st[0] & pk.PLDP_ST_CAPACITY and st[1] & pk.PLDP_ST_SEQ_LEN and st[2] & pk.PLDP_ST_DRAFT_LEN
+    assert st[4] & pk.PLDP_ST_SEQ_LEN and host(L_b)[4] == 0 and host(L_b)[3] > 1
     assert (host(b_.ws) == 0).all()           # the verification workspace is left zero
 
 
