@@ -16,12 +16,20 @@
  *      (Sec. 4.3)                                         -> pldp_extract_draft
  *   4. verifies the draft greedily against the target
  *      model's K+1 next-token distributions (Sec. 4.4)    -> pldp_verify_greedy
+ *      or by sampling at temperature T                    -> pldp_verify_sample
+ *
+ * Fused forms: pldp_draft_step runs 1-3 in one launch (scanning the contexts, or
+ * with the incremental token index of pldp_index_build); pldp_verify_greedy_draft
+ * runs 4 for the current step and then 1-3 for the next step.  Offline:
+ * pldp_rank_hidden_avg (App. B.2) and pldp_identify_heads / pldp_top_heads
+ * (Sec. 4.2.1).
  *
  * Conventions shared by every call
  *  - Every pointer argument is a DEVICE pointer owned by the caller; the
  *    library allocates nothing and keeps no state between calls, except the
- *    caller-provided verification workspace described at pldp_verify_greedy
- *    and the fixed scratch area of pldp_verify_greedy_noalloc.
+ *    caller-provided verification workspace described at pldp_verify_greedy,
+ *    the caller-provided token index that the indexed drafting calls keep up
+ *    to date, and the fixed scratch area of pldp_verify_greedy_noalloc.
  *  - All work is enqueued asynchronously on `stream` (a cudaStream_t; NULL is
  *    the legacy default stream).  No call synchronises the device or reads
  *    device memory on the host, so every call may be captured in a CUDA graph.
