@@ -339,22 +339,31 @@ class DecodeLoop:
             gen_attention(w, self.seq_len, s_last, self.T_cap, self.device, self.gen, out=self.A)
         gen_logits(w, targets, self.device, self.gen, out=self.logits)
 
+    def next_lengths(self, draft: torch.Tensor, draft_len: torch.Tensor) -> torch.Tensor:
+        """The context lengths greedy verification of ``draft`` will leave: the
+        logits plant gt[L + i] as row i's argmax, so n = the first i < draft_len with
+        draft[i] != gt[L + i] (else draft_len), and L + n + 1 when that fits T_cap."""
+        w = self.w
+        L = self.seq_len.long()
+        ar = torch.arange(w.K + 1, device=self.device)
+        targets = self.gt.gather(1, (L[:, None] + ar[None]).clamp(max=self.T_cap - 1))
+        d = draft_len.long().clamp(0, w.K)
+        mism = (draft.long() != targets[:, :w.K]) | (ar[None, :w.K] >= d[:, None])
+        n = torch.where(mism.any(dim=1), mism.int().argmax(dim=1), d)
+        return torch.where(L + n + 1 <= self.T_cap, L + n + 1, L)
+
     def step_inputs_next(self, step: int, draft: torch.Tensor, draft_len: torch.Tensor):
         """Inputs of a step that verifies ``draft`` and drafts the next step in one
         call: logits for the current state, and attention rows for the query of the
         state verification will leave (the forward pass that produces this step's
-        logits also produces those rows).  The accepted length is that of greedy
-        verification against the planted targets, computed here on the device."""
+        logits also produces those rows), from next_lengths."""
         w = self.w
         self.gen.manual_seed(self.seed * 100003 + step)
         L = self.seq_len.long()
-        ar = torch.arange(w.K + 1, device=self.device)
-        idx = (L[:, None] + ar[None]).clamp(max=self.T_cap - 1)
+        idx = (L[:, None] + torch.arange(w.K + 1, device=self.device)[None]).clamp(max=self.T_cap - 1)
         targets = self.gt.gather(1, idx)
         if self.A is not None:
-            mism = (draft.long() != targets[:, :w.K]) | (ar[None, :w.K] >= draft_len.long()[:, None])
-            n = torch.where(mism.any(dim=1), mism.int().argmax(dim=1), draft_len.long().clamp(0, w.K))
-            L_next = torch.where(L + n + 1 <= self.T_cap, L + n + 1, L)
+            L_next = self.next_lengths(draft, draft_len)
             s_last = self.src.gather(1, (L_next - 1).clamp(min=0)[:, None])[:, 0]
             gen_attention(w, L_next.to(torch.int32), s_last, self.T_cap, self.device, self.gen, out=self.A)
         gen_logits(w, targets, self.device, self.gen, out=self.logits)
