@@ -1,0 +1,43 @@
+"""Host-side pieces of bench.py on the CPU: the traffic record read from a profile
+summary is used only while the profiled sources are unchanged, and the algorithmic
+byte counts follow the per-unit figures of the measurement section."""
+import os
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+import workloads as wl  # noqa: E402
+
+
+def test_profiled_traffic_needs_matching_sources(tmp_path, monkeypatch):
+    src = tmp_path / "k.cu"
+    src.write_text("__global__ void k() {}\n")
+    prof = tmp_path / "profiles"
+    prof.mkdir()
+    sha = bench.source_sha256([str(src)])
+    (prof / "k.md").write_text(f"# k\n\ntraffic_bytes_per_launch: 1234\nsource_sha256: {sha}\n")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench.profiled_traffic([str(src)], "k.md") == 1234.0
+    src.write_text("__global__ void k() { }\n")                 # the kernel changed: no record
+    assert bench.profiled_traffic([str(src)], "k.md") is None
+    assert bench.profiled_traffic([str(src)], "missing.md") is None
+
+
+def test_step_bytes_follow_the_per_unit_figures():
+    w = wl.CONFIGS["c5"]
+    L, cand = 33716.6, 1.15
+    by = bench.step_bytes(w, L, cand)
+    B = w.B
+    assert by["verify_greedy"] == 2 * B * (w.K + 1) * w.V                  # the logits, bf16
+    assert by["find_candidates"] == pytest.approx(4 * B * L)                # ids scanned
+    assert by["rank_hidden"] == pytest.approx(2 * B * (cand + 1) * w.d)     # H_{j-1} rows and H_{t-1}
+    assert by["rank_attention"] == pytest.approx(2 * B * cand * w.R)
+    assert by["draft_step"] == pytest.approx(by["find_candidates"] + by["rank_hidden"] + by["rank_attention"]
+                                             + by["extract_draft"])
+    # the indexed drafting reads no context: an index entry and the appended ids instead
+    assert by["draft_index"] < by["draft_step"] - by["find_candidates"] + B * 64 * 2
+    assert by["verify_greedy_draft"] == pytest.approx(by["verify_greedy"] + by["draft_index"])
+    assert 426e6 < by["verify_greedy"] < 427e6
