@@ -51,7 +51,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=256)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="c5")
+    ap.add_argument("--workload", default="decode_loop_b128_ctx32k")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--slack-us", type=float, default=300.0,
                     help="GPU spin after each flush, outside the timed region, so that a step's launches "
@@ -359,7 +359,7 @@ def run_ours(args, ws_, rank, local):
     dev = torch.device("cuda", local)
     w = workload(args)
     if w.steps <= 1:
-        raise SystemExit("the benchmark workload is the sustained decode loop (c5)")
+        raise SystemExit("the benchmark workload is the sustained decode loop")
     w = w.replace(seed=shard_seed(w.seed, rank))      # each rank its own shard of sequences
     K_steps, W_steps = args.steps, args.warmup
     t0 = time.perf_counter()
@@ -446,7 +446,7 @@ def run_ours(args, ws_, rank, local):
     achieved = ver_bytes / ver_s / 1e9
     csrc = os.path.join(ROOT, "paper_2412_01447_gb300", "csrc")
     traffic = profiled_traffic([os.path.join(csrc, "verify.cu"), os.path.join(csrc, "pldp_internal.cuh")],
-                               "verify_greedy_c5.md")            # the argmax pass's sources
+                               "verify_greedy_decode_loop.md")            # the argmax pass's sources
     if path.index is not None:
         step_bytes_total = by["verify_greedy"] + by["draft_index"]
     else:

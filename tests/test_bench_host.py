@@ -27,7 +27,7 @@ def test_profiled_traffic_needs_matching_sources(tmp_path, monkeypatch):
 
 
 def test_step_bytes_follow_the_per_unit_figures():
-    w = wl.CONFIGS["c5"]
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"]
     L, cand = 33716.6, 1.15
     by = bench.step_bytes(w, L, cand)
     B = w.B

@@ -21,7 +21,8 @@ def _sample(B, k, seed):
 
 
 @pytest.mark.parametrize("fused", [False, True], ids=["calls", "fused"])
-@pytest.mark.parametrize("name", ["c1", "c2", "c3", "c4"])
+@pytest.mark.parametrize("name", ["one_step_b1_ctx512", "hidden_b8_ctx4k", "hidden_b64_ctx16k",
+                                  "attention_b32_ctx8k"])
 def test_single_step_config(lib, name, fused):
     w = wl.CONFIGS[name]
     inp = wl.single_step(w, device=DEV)
@@ -62,15 +63,15 @@ def test_single_step_config(lib, name, fused):
     # the planted structure is recovered: the planted accept length on (nearly) every sequence
     hit = float(np.mean(g["acc"] == inp["planted_accept"]))
     assert hit >= 0.8, hit
-    if name == "c1":
+    if name == "one_step_b1_ctx512":
         assert g["acc"].tolist() == [6]
 
 
 @pytest.mark.parametrize("fused", [False, True], ids=["calls", "fused"])
-def test_decode_loop_c5(lib, fused):
+def test_decode_loop_full(lib, fused):
     """The sustained loop: every step compared with the oracle run on the same
     pre-step state; the emitted streams equal the ground truth (losslessness)."""
-    w = wl.CONFIGS["c5"]
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"]
     steps = 5
     loop = wl.DecodeLoop(w, steps=steps, device=DEV)
     B, K, C = w.B, w.K, w.C_cap
@@ -115,7 +116,7 @@ def test_decode_loop_c5(lib, fused):
 def test_graph_capture_replays_the_step(lib, fused):
     """The five calls captured in one CUDA graph give the eager results, and the
     verify workspace returns to zero between replays."""
-    w = wl.CONFIGS["c5"].replace(B=16, prompt_len=3000, out_len=1000, V=32000, d=1024)
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"].replace(B=16, prompt_len=3000, out_len=1000, V=32000, d=1024)
     a = wl.DecodeLoop(w, steps=6, device=DEV)
     b = wl.DecodeLoop(w, steps=6, device=DEV)
     buf_a = Buffers(w.B, w.K, w.V, w.C_cap, DEV)
@@ -147,7 +148,7 @@ def test_graph_capture_replays_verify_draft(lib):
     step gives the eager call's results, with the token index kept up to date by the
     replays; the verify workspace returns to zero between replays."""
     import paper_2412_01447_gb300 as pk
-    w = wl.CONFIGS["c5"].replace(B=16, prompt_len=3000, out_len=1000, V=32000, d=1024)
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"].replace(B=16, prompt_len=3000, out_len=1000, V=32000, d=1024)
     ng = (w.ngram_min, w.ngram_max)
     loops = [wl.DecodeLoop(w, steps=6, device=DEV) for _ in range(2)]
     bufs = [Buffers(w.B, w.K, w.V, w.C_cap, DEV) for _ in range(2)]
@@ -188,13 +189,13 @@ def test_graph_capture_replays_verify_draft(lib):
         assert int(bufs[1].ws.count_nonzero()) == 0
 
 
-def test_decode_loop_c5_verify_draft(lib):
-    """The benchmark's configuration: the full c5 loop with one pldp_verify_greedy_draft
-    call per step (verification, then the next draft with the token index).  Each step
-    is compared with the oracle: verification of the GPU's draft on the pre-step state,
-    then candidates, rankings (sampled sequences) and draft on the state it leaves."""
+def test_decode_loop_full_verify_draft(lib):
+    """The benchmark's configuration: the full decode loop (batch 128, context 32768)
+    with one pldp_verify_greedy_draft call per step (verification, then the next draft
+    with the token index).  Each step is compared with the oracle: verification of the
+    GPU's draft on the pre-step state, then candidates, rankings (sampled sequences) and draft on the state it leaves."""
     import paper_2412_01447_gb300 as pk
-    w = wl.CONFIGS["c5"]
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"]
     steps = 4
     loop = wl.DecodeLoop(w, steps=steps, device=DEV)
     B, K, C = w.B, w.K, w.C_cap

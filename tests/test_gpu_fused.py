@@ -84,7 +84,7 @@ def test_draft_step_rows_threshold_long_draft(lib, agg):
 @pytest.mark.parametrize("draft_from", ["hidden", "attention"])
 def test_draft_step_matches_separate_calls(lib, draft_from):
     """Same integer results as the four separate calls on a planted workload."""
-    w = wl.CONFIGS["c4"].replace(B=24, prompt_len=3000, out_len=1000, V=8000, d=1024, layers=2,
+    w = wl.CONFIGS["attention_b32_ctx8k"].replace(B=24, prompt_len=3000, out_len=1000, V=8000, d=1024, layers=2,
                                  heads=8, planted_heads=2, C_cap=128)
     inp = wl.single_step(w, device=DEV)
     outs = []

@@ -120,7 +120,7 @@ def test_index_marks_tokens_it_cannot_hold(lib):
 def test_indexed_decode_loop(lib):
     """A sustained loop (batch 32, context 4096, V 128256): each step drafts with and
     without the index on the same state, then verifies greedily with append."""
-    w = wl.CONFIGS["c5"].replace(B=32, prompt_len=3072, out_len=1024, d=512)
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"].replace(B=32, prompt_len=3072, out_len=1024, d=512)
     steps = 6
     loop = wl.DecodeLoop(w, steps=steps, device=DEV)
     B, K, C = w.B, w.K, w.C_cap

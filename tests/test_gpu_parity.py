@@ -246,7 +246,7 @@ def test_verify_without_bookkeeping_and_large_batch(lib):
 # ----------------------------------------------------------------------------
 @pytest.mark.parametrize("draft_from", ["hidden", "attention"])
 def test_small_step_end_to_end(lib, draft_from):
-    w = wl.CONFIGS["c4"].replace(B=6, prompt_len=900, out_len=300, V=3000, d=512, layers=2,
+    w = wl.CONFIGS["attention_b32_ctx8k"].replace(B=6, prompt_len=900, out_len=300, V=3000, d=512, layers=2,
                                  heads=8, planted_heads=2, C_cap=128)
     inp = wl.single_step(w, device=DEV)
     ids0, L0 = host(inp["ids"]), host(inp["seq_len"])

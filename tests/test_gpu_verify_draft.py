@@ -158,7 +158,7 @@ def test_verify_draft_decode_loop(lib):
     """The sustained loop (batch 32, context 4096, V 128256): each step verifies and
     drafts the next with the fused call on one copy of the state and with the two
     calls on another; the emitted streams are the ground truth."""
-    w = wl.CONFIGS["c5"].replace(B=32, prompt_len=3072, out_len=1024, d=512)
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"].replace(B=32, prompt_len=3072, out_len=1024, d=512)
     steps = 6
     loop = wl.DecodeLoop(w, steps=steps, device=DEV)
     B, K, C = w.B, w.K, w.C_cap

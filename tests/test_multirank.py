@@ -35,7 +35,7 @@ def _rank_main(rank, world, port, outdir):
     bench.barrier(ws)
     elapsed_ms = 3.0 + 2.0 * rank                       # this rank's device time over its steps
     worst = bench.max_over_ranks(elapsed_ms, ws)
-    w = wl.CONFIGS["c5"].replace(B=2, prompt_len=64, out_len=32)
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"].replace(B=2, prompt_len=64, out_len=32)
     tok, _ = wl.token_streams(w, w.T, bench.shard_seed(w.seed, rank))
     bench.barrier(ws)
     with open(os.path.join(outdir, f"rank{rank}.json"), "w") as f:

@@ -464,7 +464,7 @@ def test_identify_heads_recovers_planted_heads(orc):
     """Copied spans; rows of 3 planted heads per layer put extra attention on the
     true copy source of the generated token: they are exactly the top heads."""
     import workloads as wl
-    w = wl.CONFIGS["c4"].replace(B=24, prompt_len=600, out_len=400, V=5000, layers=2, heads=8,
+    w = wl.CONFIGS["attention_b32_ctx8k"].replace(B=24, prompt_len=600, out_len=400, V=5000, layers=2, heads=8,
                                  planted_heads=3)
     tok, src = wl.token_streams(w, w.T, 77)
     rng = np.random.default_rng(78)

@@ -11,7 +11,7 @@ from tests._parity import host
 
 
 def test_next_lengths_match_oracle_verification():
-    w = wl.CONFIGS["c5"].replace(B=6, prompt_len=192, out_len=64, V=100, d=16, layers=1, heads=4,
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"].replace(B=6, prompt_len=192, out_len=64, V=100, d=16, layers=1, heads=4,
                                  planted_heads=2)
     loop = wl.DecodeLoop(w, steps=6, device="cpu")
     K, T_cap = w.K, loop.T_cap

@@ -89,34 +89,34 @@ def _round_up(x, m):
     return (x + m - 1) // m * m
 
 
-CONFIGS = {
+CONFIGS = {w.name: w for w in (
     # batch 1, one step: 384-token prompt + 128 output tokens (70% copied, spans 4-16),
     # V = 32000, max n-gram 3, K = 10, fp32 hidden [512, 4096], fp32 logits with the first
     # 6 draft tokens accepted.
-    "c1": Workload("c1", B=1, prompt_len=384, out_len=128, V=32000, K=10, copy_frac=0.7,
-                   span_min=4, span_max=16, d=4096, h_dtype="f32", logits_dtype="f32",
-                   accept="fixed:6", seed=1001),
+    Workload("one_step_b1_ctx512", B=1, prompt_len=384, out_len=128, V=32000, K=10, copy_frac=0.7,
+             span_min=4, span_max=16, d=4096, h_dtype="f32", logits_dtype="f32",
+             accept="fixed:6", seed=1001),
     # batch 8, context 4096 (3072 + 1024, 60% copied, spans 2-32), V = 32000, bf16 hidden
     # [8, 4096, 4096], K = 10, bf16 logits with accept length U{0..10}.
-    "c2": Workload("c2", B=8, prompt_len=3072, out_len=1024, V=32000, K=10, copy_frac=0.6,
-                   span_min=2, span_max=32, d=4096, seed=1002),
+    Workload("hidden_b8_ctx4k", B=8, prompt_len=3072, out_len=1024, V=32000, K=10, copy_frac=0.6,
+             span_min=2, span_max=32, d=4096, seed=1002),
     # batch 64, context 16384 (12288 + 4096, 50% copied, spans 2-64), V = 32000, bf16 hidden
     # width 5120, K = 16, bf16 logits [64, 17, 32000].
-    "c3": Workload("c3", B=64, prompt_len=12288, out_len=4096, V=32000, K=16, copy_frac=0.5,
-                   span_min=2, span_max=64, d=5120, seed=1003),
+    Workload("hidden_b64_ctx16k", B=64, prompt_len=12288, out_len=4096, V=32000, K=16, copy_frac=0.5,
+             span_min=2, span_max=64, d=5120, seed=1003),
     # attention ranking: batch 32, context 8192 (6144 + 2048, 60% copied, spans 2-32),
     # bf16 attention rows [32, 4 layers, 32 heads, 8192] with mass planted on the copy
     # source in 8 heads per layer, K = 10, bf16 logits [32, 11, 128256].
-    "c4": Workload("c4", B=32, prompt_len=6144, out_len=2048, V=128256, K=10, copy_frac=0.6,
-                   span_min=2, span_max=32, layers=4, heads=32, planted_heads=8, seed=1004),
+    Workload("attention_b32_ctx8k", B=32, prompt_len=6144, out_len=2048, V=128256, K=10, copy_frac=0.6,
+             span_min=2, span_max=32, layers=4, heads=32, planted_heads=8, seed=1004),
     # sustained decode loop: batch 128, context 32768 (24576 + 8192), 256 steps; the ground
     # truth copies prompt spans (2-32) with probability 0.6 per segment, else a uniform
     # token; bf16 hidden width 4096 and attention rows [4 layers x 32 heads] both ranked;
     # V = 128256, K = 12.
-    "c5": Workload("c5", B=128, prompt_len=24576, out_len=8192, V=128256, K=12,
-                   p_copy_per_segment=0.6, span_min=2, span_max=32, d=4096, layers=4,
-                   heads=32, planted_heads=8, accept="ground_truth", steps=256, seed=1005),
-}
+    Workload("decode_loop_b128_ctx32k", B=128, prompt_len=24576, out_len=8192, V=128256, K=12,
+             p_copy_per_segment=0.6, span_min=2, span_max=32, d=4096, layers=4,
+             heads=32, planted_heads=8, accept="ground_truth", steps=256, seed=1005),
+)}
 
 
 def torch_dtype(name):
@@ -249,7 +249,7 @@ def gen_logits(w: Workload, targets: torch.Tensor, device, gen: torch.Generator,
 # complete inputs
 # ----------------------------------------------------------------------------
 def single_step(w: Workload, device="cpu", seed: Optional[int] = None) -> dict:
-    """All inputs of one decode step of a single-step config (c1-c4 or a variant).
+    """All inputs of one decode step of a single-step config (a one-step workload or a variant).
 
     Returns a dict of tensors on ``device``: ids [B, T_cap] int32, seq_len [B] int32,
     H or None, A or None, logits; plus host numpy: src, expected_draft [B, K] (the
@@ -289,7 +289,7 @@ def single_step(w: Workload, device="cpu", seed: Optional[int] = None) -> dict:
 
 
 class DecodeLoop:
-    """Sustained decode loop inputs (c5 or a variant).
+    """Sustained decode loop inputs (the decode loop or a variant).
 
     The ground-truth stream ``gt`` [B, T_cap] is fixed up front; the context starts as
     its first w.T tokens.  Before every step, ``step_inputs`` writes fresh attention
