@@ -12,7 +12,16 @@ PLD+ (arXiv 2412.01447), per decode step and per sequence:
   * ``pldp_rank_hidden``     -- Eq. 3 (Sec. 4.2.2): cosine of hidden states;
   * ``pldp_rank_attention``  -- Eq. 2 (Sec. 4.2.1): max attention of selected heads;
   * ``pldp_extract_draft``   -- Sec. 4.3: the K tokens after the best occurrence;
-  * ``pldp_verify_greedy``   -- Sec. 4.4: greedy accept against the target argmax.
+  * ``pldp_verify_greedy``   -- Sec. 4.4: greedy accept against the target argmax;
+  * ``pldp_verify_sample``   -- Sec. 4.4 with sampling, from caller uniforms.
+The fused calls: ``pldp_draft_step`` (the first four in one launch, optionally
+with the token index of ``pldp_index_build``) and ``pldp_verify_greedy_draft``
+(verification, then the next step's draft).  Also ``pldp_rank_hidden_avg``
+(App. B.2) and ``pldp_identify_heads`` / ``pldp_top_heads`` (Sec. 4.2.1).
+
+Device buffers are passed as raw pointers, so the binding checks what the C
+side cannot: every tensor is a CUDA tensor of the stated dtype, dense where
+the call wants it, and holds at least the elements the call will touch.
 """
 from __future__ import annotations
 
@@ -29,8 +38,14 @@ __all__ = [
     "PLDP_F32", "PLDP_BF16", "PLDP_AGG_MAX", "PLDP_AGG_SUM",
     "PLDP_ST_CAND_OVERFLOW", "PLDP_ST_TOKEN_RANGE", "PLDP_ST_CAPACITY", "PLDP_ST_SEQ_LEN",
     "PLDP_ST_DRAFT_LEN", "PLDP_ST_ROW_INDEX", "PLDP_ST_TIMEOUT",
+    "PLDP_OK", "PLDP_ERR_INVALID_ARG", "PLDP_ERR_UNSUPPORTED", "PLDP_ERR_CUDA", "PLDP_ERR_TIMEOUT",
     "pldp_find_candidates", "pldp_rank_hidden", "pldp_rank_attention", "pldp_extract_draft",
-    "pldp_draft_step", "pldp_draft_step_args", "pldp_draft_workspace_size", "pldp_verify_greedy", "pldp_verify_greedy_noalloc", "pldp_verify_workspace_size",
+    "pldp_verify_greedy", "pldp_verify_workspace_size", "pldp_verify_greedy_noalloc",
+    "pldp_verify_sample", "pldp_verify_sample_workspace_size",
+    "pldp_draft_step", "pldp_draft_step_args", "pldp_draft_workspace_size",
+    "pldp_index_size", "pldp_index_build",
+    "pldp_verify_greedy_draft", "pldp_verify_draft_args",
+    "pldp_rank_hidden_avg", "pldp_identify_heads", "pldp_top_heads",
     "pldp_version", "pldp_last_error",
 ]
 
@@ -185,17 +200,38 @@ def _dev(t, name, dtype=None, allow_none=False):
     return ctypes.c_void_p(t.data_ptr())
 
 
-def _dense(t, name, dtype=None, allow_none=False):
-    if t is not None and not t.is_contiguous():
-        raise ValueError(f"{name} must be contiguous")
+_WORD = (torch.int32, getattr(torch, "uint32", torch.int32))
+
+
+def _dense(t, name, dtype=None, allow_none=False, n=None):
+    """A contiguous tensor of at least n elements (the call reads or writes n).
+    dtype _WORD: any 4-byte integer type (status bits, counts)."""
+    if t is not None:
+        if not isinstance(t, torch.Tensor):
+            raise ValueError(f"{name} must be a CUDA tensor")
+        if not t.is_contiguous():
+            raise ValueError(f"{name} must be contiguous")
+        if n is not None and t.numel() < n:
+            raise ValueError(f"{name} needs {n} elements, has {t.numel()}")
+        if dtype is _WORD:
+            if t.dtype not in _WORD:
+                raise ValueError(f"{name} must be int32 or uint32, got {t.dtype}")
+            dtype = None
     return _dev(t, name, dtype, allow_none)
 
 
-def _rows(t, name):
-    """A [B, T] int32 tensor whose rows may be strided (unit inner stride)."""
-    if t.dim() != 2 or t.stride(1) != 1:
+def _rows(t, name, B=None, T_cap=None):
+    """A [B, T] int32 tensor whose rows may be strided (unit inner stride), with at
+    least B rows; returns (pointer, row stride, T_cap), T_cap at most T (default T)."""
+    if not isinstance(t, torch.Tensor) or t.dim() != 2 or t.stride(1) != 1:
         raise ValueError(f"{name} must be 2-D with unit inner stride")
-    return _dev(t, name, torch.int32), t.stride(0), t.shape[1]
+    if B is not None and t.shape[0] < B:
+        raise ValueError(f"{name} has {t.shape[0]} rows, the call needs {B}")
+    if T_cap is None:
+        T_cap = t.shape[1]
+    elif not 0 <= T_cap <= t.shape[1]:
+        raise ValueError(f"T_cap = {T_cap} is outside [0, {name}.shape[1] = {t.shape[1]}]")
+    return _dev(t, name, torch.int32), t.stride(0), int(T_cap)
 
 
 def _code(x):
@@ -219,14 +255,14 @@ def pldp_find_candidates(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_coun
     """Eq. 1 with the longest-suffix n-gram rule.  ids: int32 [B, T] (rows may be
     strided), seq_len int32 [B]; outputs cand_pos int32 [B, C_cap], cand_count and
     match_len int32 [B], status uint32-as-int32 [B] (optional)."""
-    p_ids, stride, T = _rows(ids, "ids")
+    p_ids, stride, T = _rows(ids, "ids", T_cap=T_cap)
     B = ids.shape[0]
     C_cap = cand_pos.shape[1] if cand_pos is not None and cand_pos.dim() == 2 else 0
     _check("pldp_find_candidates", _load().pldp_find_candidates(
-        p_ids, stride, _dense(seq_len, "seq_len", torch.int32), B, T if T_cap is None else T_cap,
-        ngram_min, ngram_max, _dense(cand_pos, "cand_pos", torch.int32, allow_none=True), C_cap,
-        _dense(cand_count, "cand_count", torch.int32), _dense(match_len, "match_len", torch.int32),
-        _dense(status, "status", None, allow_none=True), _stream(stream)))
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, n=B), B, T,
+        ngram_min, ngram_max, _dense(cand_pos, "cand_pos", torch.int32, allow_none=True, n=B * C_cap), C_cap,
+        _dense(cand_count, "cand_count", torch.int32, n=B), _dense(match_len, "match_len", torch.int32, n=B),
+        _dense(status, "status", _WORD, allow_none=True, n=B), _stream(stream)))
 
 
 def pldp_rank_hidden(H, seq_len, cand_pos, cand_count, best_pos, scores=None, best_score=None,
@@ -239,12 +275,12 @@ def pldp_rank_hidden(H, seq_len, cand_pos, cand_count, best_pos, scores=None, be
     B, T_cap, d = H.shape
     C_cap = cand_pos.shape[1]
     _check("pldp_rank_hidden", _load().pldp_rank_hidden(
-        _dev(H, "H"), _code(H.dtype), d, H.stride(0), _dense(seq_len, "seq_len", torch.int32), B,
-        T_cap, _dense(cand_pos, "cand_pos", torch.int32), _dense(cand_count, "cand_count", torch.int32),
-        C_cap, float(threshold), _dense(scores, "scores", torch.float32, allow_none=True),
-        _dense(best_pos, "best_pos", torch.int32),
-        _dense(best_score, "best_score", torch.float32, allow_none=True),
-        _dense(status, "status", None, allow_none=True), _stream(stream)))
+        _dev(H, "H"), _code(H.dtype), d, H.stride(0), _dense(seq_len, "seq_len", torch.int32, n=B), B,
+        T_cap, _dense(cand_pos, "cand_pos", torch.int32, n=B * C_cap), _dense(cand_count, "cand_count", torch.int32, n=B),
+        C_cap, float(threshold), _dense(scores, "scores", torch.float32, allow_none=True, n=B * C_cap),
+        _dense(best_pos, "best_pos", torch.int32, n=B),
+        _dense(best_score, "best_score", torch.float32, allow_none=True, n=B),
+        _dense(status, "status", _WORD, allow_none=True, n=B), _stream(stream)))
 
 
 def pldp_rank_hidden_avg(H, seq_len, cand_pos, cand_count, best_pos, m, scores=None, best_score=None,
@@ -256,12 +292,12 @@ def pldp_rank_hidden_avg(H, seq_len, cand_pos, cand_count, best_pos, m, scores=N
     B, T_cap, d = H.shape
     C_cap = cand_pos.shape[1]
     _check("pldp_rank_hidden_avg", _load().pldp_rank_hidden_avg(
-        _dev(H, "H"), _code(H.dtype), d, H.stride(0), int(m), _dense(seq_len, "seq_len", torch.int32), B,
-        T_cap, _dense(cand_pos, "cand_pos", torch.int32), _dense(cand_count, "cand_count", torch.int32),
-        C_cap, float(threshold), _dense(scores, "scores", torch.float32, allow_none=True),
-        _dense(best_pos, "best_pos", torch.int32),
-        _dense(best_score, "best_score", torch.float32, allow_none=True),
-        _dense(status, "status", None, allow_none=True), _stream(stream)))
+        _dev(H, "H"), _code(H.dtype), d, H.stride(0), int(m), _dense(seq_len, "seq_len", torch.int32, n=B), B,
+        T_cap, _dense(cand_pos, "cand_pos", torch.int32, n=B * C_cap), _dense(cand_count, "cand_count", torch.int32, n=B),
+        C_cap, float(threshold), _dense(scores, "scores", torch.float32, allow_none=True, n=B * C_cap),
+        _dense(best_pos, "best_pos", torch.int32, n=B),
+        _dense(best_score, "best_score", torch.float32, allow_none=True, n=B),
+        _dense(status, "status", _WORD, allow_none=True, n=B), _stream(stream)))
 
 
 def pldp_identify_heads(ids, pos, A, counts, max_suffix=64, r_star=None, status=None, stream=None):
@@ -269,21 +305,24 @@ def pldp_identify_heads(ids, pos, A, counts, max_suffix=64, r_star=None, status=
     generated token's position p); A [B, R, T_cap] float32/bfloat16, the attention
     rows of query p-1 (unit inner stride); counts int32/uint32 [R] CUDA tensor,
     added to.  r_star int32 [B] out (optional)."""
-    p_ids, stride, T_cap = _rows(ids, "ids")
     if A.dim() != 3 or A.stride(2) != 1:
         raise ValueError("A must be [B, R, T_cap] with unit inner stride")
     B, R = A.shape[0], A.shape[1]
+    p_ids, stride, T_cap = _rows(ids, "ids", B)
+    if A.shape[2] < T_cap:
+        raise ValueError("A must cover the T_cap = ids.shape[1] key positions")
     _check("pldp_identify_heads", _load().pldp_identify_heads(
-        p_ids, stride, _dense(pos, "pos", torch.int32), B, T_cap, int(max_suffix), _dev(A, "A"), _code(A.dtype),
-        R, A.stride(1), A.stride(0), _dense(counts, "counts", None), _dense(r_star, "r_star", torch.int32,
-                                                                             allow_none=True),
-        _dense(status, "status", None, allow_none=True), _stream(stream)))
+        p_ids, stride, _dense(pos, "pos", torch.int32, n=B), B, T_cap, int(max_suffix), _dev(A, "A"), _code(A.dtype),
+        R, A.stride(1), A.stride(0), _dense(counts, "counts", _WORD, n=R),
+        _dense(r_star, "r_star", torch.int32, allow_none=True, n=B),
+        _dense(status, "status", _WORD, allow_none=True, n=B), _stream(stream)))
 
 
 def pldp_top_heads(counts, k, row_idx, stream=None):
     """The k rows with the most counts (ties to the smaller index) into row_idx int32 [k]."""
-    _check("pldp_top_heads", _load().pldp_top_heads(_dense(counts, "counts", None), counts.numel(), int(k),
-                                                    _dense(row_idx, "row_idx", torch.int32), _stream(stream)))
+    _check("pldp_top_heads", _load().pldp_top_heads(_dense(counts, "counts", _WORD), counts.numel(), int(k),
+                                                    _dense(row_idx, "row_idx", torch.int32, n=int(k)),
+                                                    _stream(stream)))
 
 
 def pldp_rank_attention(A, seq_len, cand_pos, cand_count, best_pos, row_idx=None, agg=PLDP_AGG_MAX,
@@ -298,22 +337,22 @@ def pldp_rank_attention(A, seq_len, cand_pos, cand_count, best_pos, row_idx=None
     _check("pldp_rank_attention", _load().pldp_rank_attention(
         _dev(A, "A"), _code(A.dtype), R, A.stride(1), A.stride(0),
         _dense(row_idx, "row_idx", torch.int32, allow_none=True), n_sel, int(agg),
-        _dense(seq_len, "seq_len", torch.int32), B, T_cap, _dense(cand_pos, "cand_pos", torch.int32),
-        _dense(cand_count, "cand_count", torch.int32), C_cap,
-        _dense(scores, "scores", torch.float32, allow_none=True),
-        _dense(best_pos, "best_pos", torch.int32),
-        _dense(best_score, "best_score", torch.float32, allow_none=True),
-        _dense(status, "status", None, allow_none=True), _stream(stream)))
+        _dense(seq_len, "seq_len", torch.int32, n=B), B, T_cap, _dense(cand_pos, "cand_pos", torch.int32, n=B * C_cap),
+        _dense(cand_count, "cand_count", torch.int32, n=B), C_cap,
+        _dense(scores, "scores", torch.float32, allow_none=True, n=B * C_cap),
+        _dense(best_pos, "best_pos", torch.int32, n=B),
+        _dense(best_score, "best_score", torch.float32, allow_none=True, n=B),
+        _dense(status, "status", _WORD, allow_none=True, n=B), _stream(stream)))
 
 
 def pldp_extract_draft(ids, seq_len, best_pos, draft, draft_len, T_cap=None, stream=None):
     """Sec. 4.3.  draft int32 [B, K] and draft_len int32 [B] are written."""
-    p_ids, stride, T = _rows(ids, "ids")
     B, K = draft.shape
+    p_ids, stride, T = _rows(ids, "ids", B, T_cap)
     _check("pldp_extract_draft", _load().pldp_extract_draft(
-        p_ids, stride, _dense(seq_len, "seq_len", torch.int32), T if T_cap is None else T_cap,
-        _dense(best_pos, "best_pos", torch.int32), B, K, _dense(draft, "draft", torch.int32),
-        _dense(draft_len, "draft_len", torch.int32), _stream(stream)))
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, n=B), T,
+        _dense(best_pos, "best_pos", torch.int32, n=B), B, K, _dense(draft, "draft", torch.int32, n=B * K),
+        _dense(draft_len, "draft_len", torch.int32, n=B), _stream(stream)))
 
 
 def pldp_draft_workspace_size(B) -> int:
@@ -326,40 +365,44 @@ def _draft_args(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_
                 a_scores=None, best_a_score=None, draft_from="hidden", status=None, T_cap=None,
                 index=None, V=None):
     """The argument block of pldp_draft_step (marshalling only)."""
-    p_ids, stride, T = _rows(ids, "ids")
+    p_ids, stride, T = _rows(ids, "ids", T_cap=T_cap)
     B = ids.shape[0]
     a = pldp_draft_step_args()
-    a.ids, a.ids_stride, a.seq_len, a.B = p_ids, stride, _dense(seq_len, "seq_len", torch.int32), B
-    a.T_cap = T if T_cap is None else T_cap
+    a.ids, a.ids_stride, a.seq_len, a.B = p_ids, stride, _dense(seq_len, "seq_len", torch.int32, n=B), B
+    a.T_cap = T
     a.ngram_min, a.ngram_max = ngram_min, ngram_max
-    a.cand_pos = _dense(cand_pos, "cand_pos", torch.int32, allow_none=True)
-    a.C_cap = cand_pos.shape[1] if cand_pos is not None and cand_pos.dim() == 2 else 0
-    a.cand_count = _dense(cand_count, "cand_count", torch.int32)
-    a.match_len = _dense(match_len, "match_len", torch.int32)
+    a.C_cap = C_cap = cand_pos.shape[1] if cand_pos is not None and cand_pos.dim() == 2 else 0
+    a.cand_pos = _dense(cand_pos, "cand_pos", torch.int32, allow_none=True, n=B * C_cap)
+    a.cand_count = _dense(cand_count, "cand_count", torch.int32, n=B)
+    a.match_len = _dense(match_len, "match_len", torch.int32, n=B)
     if H is not None:
         if H.dim() != 3 or H.stride(2) != 1 or H.stride(1) != H.shape[2]:
             raise ValueError("H must be [B, T_cap, d] with contiguous rows")
+        if H.shape[0] < B or H.shape[1] < T:
+            raise ValueError(f"H must cover [B, T_cap] = [{B}, {T}] positions")
         a.H, a.h_dtype, a.d, a.h_seq_stride = _dev(H, "H"), _code(H.dtype), H.shape[2], H.stride(0)
         a.threshold = float(threshold)
-        a.h_scores = _dense(h_scores, "h_scores", torch.float32, allow_none=True)
-        a.best_h = _dense(best_h, "best_h", torch.int32)
-        a.best_h_score = _dense(best_h_score, "best_h_score", torch.float32, allow_none=True)
+        a.h_scores = _dense(h_scores, "h_scores", torch.float32, allow_none=True, n=B * C_cap)
+        a.best_h = _dense(best_h, "best_h", torch.int32, n=B)
+        a.best_h_score = _dense(best_h_score, "best_h_score", torch.float32, allow_none=True, n=B)
     if A is not None:
         if A.dim() != 3 or A.stride(2) != 1:
             raise ValueError("A must be [B, R, T_cap] with unit inner stride")
+        if A.shape[0] < B or A.shape[2] < T:
+            raise ValueError(f"A must cover [B, T_cap] = [{B}, {T}] positions")
         a.A, a.a_dtype, a.R = _dev(A, "A"), _code(A.dtype), A.shape[1]
         a.a_row_stride, a.a_seq_stride = A.stride(1), A.stride(0)
         a.row_idx = _dense(row_idx, "row_idx", torch.int32, allow_none=True)
         a.n_sel = A.shape[1] if row_idx is None else row_idx.numel()
         a.agg = int(agg)
-        a.a_scores = _dense(a_scores, "a_scores", torch.float32, allow_none=True)
-        a.best_a = _dense(best_a, "best_a", torch.int32)
-        a.best_a_score = _dense(best_a_score, "best_a_score", torch.float32, allow_none=True)
+        a.a_scores = _dense(a_scores, "a_scores", torch.float32, allow_none=True, n=B * C_cap)
+        a.best_a = _dense(best_a, "best_a", torch.int32, n=B)
+        a.best_a_score = _dense(best_a_score, "best_a_score", torch.float32, allow_none=True, n=B)
     a.draft_from = {"hidden": 0, "attention": 1, 0: 0, 1: 1}[draft_from]
     a.K = K
-    a.draft = _dense(draft, "draft", torch.int32)
-    a.draft_len = _dense(draft_len, "draft_len", torch.int32)
-    a.status = _dense(status, "status", None, allow_none=True)
+    a.draft = _dense(draft, "draft", torch.int32, n=B * K)
+    a.draft_len = _dense(draft_len, "draft_len", torch.int32, n=B)
+    a.status = _dense(status, "status", _WORD, allow_none=True, n=B)
     if workspace is not None:
         a.workspace = _dense(workspace, "workspace")
         a.workspace_bytes = workspace.numel() * workspace.element_size()
@@ -399,16 +442,18 @@ def pldp_verify_greedy_draft(logits, draft, draft_len, accept_len, next_token, w
     K = K1 - 1
     if draft.shape != (B, K) or next_draft.shape != (B, K):
         raise ValueError("draft and next_draft must be [B, K] with K = logits.shape[1] - 1")
+    if not isinstance(ids, torch.Tensor) or ids.dim() != 2 or ids.shape[0] != B:
+        raise ValueError("ids must be [B, T_cap] with B = logits.shape[0]")
     a = pldp_verify_draft_args()
     a.next = _draft_args(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, next_draft,
                          next_draft_len, None, index=index, V=V, **kw)
     a.logits, a.dtype, a.V = _dense(logits, "logits"), _code(logits.dtype), V
-    a.draft = _dense(draft, "draft", torch.int32)
-    a.draft_len = _dense(draft_len, "draft_len", torch.int32)
-    a.argmax = _dense(argmax, "argmax", torch.int32, allow_none=True)
-    a.accept_len = _dense(accept_len, "accept_len", torch.int32)
-    a.next_token = _dense(next_token, "next_token", torch.int32)
-    a.kv_keep_len = _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True)
+    a.draft = _dense(draft, "draft", torch.int32, n=B * K)
+    a.draft_len = _dense(draft_len, "draft_len", torch.int32, n=B)
+    a.argmax = _dense(argmax, "argmax", torch.int32, allow_none=True, n=B * K1)
+    a.accept_len = _dense(accept_len, "accept_len", torch.int32, n=B)
+    a.next_token = _dense(next_token, "next_token", torch.int32, n=B)
+    a.kv_keep_len = _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True, n=B)
     a.workspace = _dense(workspace, "workspace")
     a.workspace_bytes = workspace.numel() * workspace.element_size()
     _check("pldp_verify_greedy_draft", _load().pldp_verify_greedy_draft(ctypes.byref(a), _stream(stream)))
@@ -422,12 +467,12 @@ def pldp_index_build(ids, seq_len, V, index, status=None, T_cap=None, stream=Non
     """Builds the incremental token index of pldp_draft_step over positions
     0 .. seq_len[b]-2 of every sequence.  index: uint8 CUDA tensor of
     pldp_index_size(B, V) bytes (cleared by the call)."""
-    p_ids, stride, T = _rows(ids, "ids")
+    p_ids, stride, T = _rows(ids, "ids", T_cap=T_cap)
     B = ids.shape[0]
     _check("pldp_index_build", _load().pldp_index_build(
-        p_ids, stride, _dense(seq_len, "seq_len", torch.int32), B, T if T_cap is None else T_cap, int(V),
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, n=B), B, T, int(V),
         _dense(index, "index"), index.numel() * index.element_size(),
-        _dense(status, "status", None, allow_none=True), _stream(stream)))
+        _dense(status, "status", _WORD, allow_none=True, n=B), _stream(stream)))
 
 
 def pldp_verify_workspace_size(B, K, V) -> int:
@@ -445,17 +490,17 @@ def pldp_verify_greedy(logits, draft, draft_len, accept_len, next_token, workspa
     K = K1 - 1
     if draft.shape != (B, K):
         raise ValueError("draft must be [B, K] with K = logits.shape[1] - 1")
-    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids")
+    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids", B, T_cap)
     if T_cap is None:
         T_cap = T
     _check("pldp_verify_greedy", _load().pldp_verify_greedy(
-        _dense(logits, "logits"), _code(logits.dtype), B, K, V, _dense(draft, "draft", torch.int32),
-        _dense(draft_len, "draft_len", torch.int32),
-        _dense(argmax, "argmax", torch.int32, allow_none=True),
-        _dense(accept_len, "accept_len", torch.int32), _dense(next_token, "next_token", torch.int32),
-        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True), T_cap,
-        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True),
-        _dense(status, "status", None, allow_none=True), _dense(workspace, "workspace"),
+        _dense(logits, "logits"), _code(logits.dtype), B, K, V, _dense(draft, "draft", torch.int32, n=B * K),
+        _dense(draft_len, "draft_len", torch.int32, n=B),
+        _dense(argmax, "argmax", torch.int32, allow_none=True, n=B * K1),
+        _dense(accept_len, "accept_len", torch.int32, n=B), _dense(next_token, "next_token", torch.int32, n=B),
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True, n=B), T_cap,
+        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True, n=B),
+        _dense(status, "status", _WORD, allow_none=True, n=B), _dense(workspace, "workspace"),
         workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
@@ -476,17 +521,17 @@ def pldp_verify_sample(logits, uniforms, draft, draft_len, accept_len, next_toke
         raise ValueError("draft must be [B, K] with K = logits.shape[1] - 1")
     if uniforms.shape != (B, K1):
         raise ValueError("uniforms must be [B, K+1]")
-    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids")
+    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids", B, T_cap)
     if T_cap is None:
         T_cap = T
     _check("pldp_verify_sample", _load().pldp_verify_sample(
         _dense(logits, "logits"), _code(logits.dtype), B, K, V, float(temperature),
-        _dense(uniforms, "uniforms", torch.float32), _dense(draft, "draft", torch.int32),
-        _dense(draft_len, "draft_len", torch.int32), _dense(sampled, "sampled", torch.int32, allow_none=True),
-        _dense(accept_len, "accept_len", torch.int32), _dense(next_token, "next_token", torch.int32),
-        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True), T_cap,
-        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True),
-        _dense(status, "status", None, allow_none=True), _dense(workspace, "workspace"),
+        _dense(uniforms, "uniforms", torch.float32), _dense(draft, "draft", torch.int32, n=B * K),
+        _dense(draft_len, "draft_len", torch.int32, n=B), _dense(sampled, "sampled", torch.int32, allow_none=True, n=B * K1),
+        _dense(accept_len, "accept_len", torch.int32, n=B), _dense(next_token, "next_token", torch.int32, n=B),
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True, n=B), T_cap,
+        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True, n=B),
+        _dense(status, "status", _WORD, allow_none=True, n=B), _dense(workspace, "workspace"),
         workspace.numel() * workspace.element_size(), _stream(stream)))
 
 
@@ -500,17 +545,17 @@ def pldp_verify_greedy_noalloc(logits, draft, draft_len, accept_len, next_token,
     K = K1 - 1
     if draft.shape != (B, K):
         raise ValueError("draft must be [B, K] with K = logits.shape[1] - 1")
-    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids")
+    p_ids, stride, T = (None, 0, 0) if ids is None else _rows(ids, "ids", B, T_cap)
     if T_cap is None:
         T_cap = T
     _check("pldp_verify_greedy_noalloc", _load().pldp_verify_greedy_noalloc(
-        _dense(logits, "logits"), _code(logits.dtype), B, K, V, _dense(draft, "draft", torch.int32),
-        _dense(draft_len, "draft_len", torch.int32),
-        _dense(argmax, "argmax", torch.int32, allow_none=True),
-        _dense(accept_len, "accept_len", torch.int32), _dense(next_token, "next_token", torch.int32),
-        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True), T_cap,
-        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True),
-        _dense(status, "status", None, allow_none=True), _stream(stream)))
+        _dense(logits, "logits"), _code(logits.dtype), B, K, V, _dense(draft, "draft", torch.int32, n=B * K),
+        _dense(draft_len, "draft_len", torch.int32, n=B),
+        _dense(argmax, "argmax", torch.int32, allow_none=True, n=B * K1),
+        _dense(accept_len, "accept_len", torch.int32, n=B), _dense(next_token, "next_token", torch.int32, n=B),
+        p_ids, stride, _dense(seq_len, "seq_len", torch.int32, allow_none=True, n=B), T_cap,
+        _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True, n=B),
+        _dense(status, "status", _WORD, allow_none=True, n=B), _stream(stream)))
 
 
 def pldp_version() -> int:

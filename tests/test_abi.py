@@ -207,3 +207,25 @@ def test_verify_draft_host_checks(so):
     assert call(a) == pk.PLDP_ERR_INVALID_ARG and "workspace" in pk.pldp_last_error()
     a = block(); a.next.B = 0
     assert call(a) == pk.PLDP_OK
+
+
+def test_binding_checks_element_counts_and_shapes():
+    """The binding passes raw pointers, so it refuses, before any call, a buffer
+    with fewer elements than the call touches, a status buffer that is not 4-byte
+    words, an ids tensor with too few rows, and a T_cap beyond the ids rows."""
+    import torch
+    with pytest.raises(ValueError, match="needs 4 elements"):
+        pk._dense(torch.zeros(3, dtype=torch.int32), "x", torch.int32, n=4)
+    with pytest.raises(ValueError, match="int32 or uint32"):
+        pk._dense(torch.zeros(4, dtype=torch.int64), "status", pk._WORD, n=4)
+    with pytest.raises(ValueError, match="contiguous"):
+        pk._dense(torch.zeros((4, 4), dtype=torch.int32)[:, :2], "x", torch.int32, n=4)
+    with pytest.raises(ValueError, match="rows"):
+        pk._rows(torch.zeros((2, 5), dtype=torch.int32), "ids", B=3)
+    with pytest.raises(ValueError, match="T_cap"):
+        pk._rows(torch.zeros((2, 5), dtype=torch.int32), "ids", T_cap=6)
+    with pytest.raises(ValueError, match="unit inner stride"):
+        pk._rows(torch.zeros((5, 2), dtype=torch.int32).t(), "ids")
+    # a tensor of the right size still has to be on the device
+    with pytest.raises(ValueError, match="CUDA"):
+        pk._dense(torch.zeros(4, dtype=torch.int32), "x", torch.int32, n=4)
