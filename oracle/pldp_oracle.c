@@ -1,7 +1,6 @@
 /*
  * pldp_oracle.c -- plain, slow, single-threaded CPU oracle of the PLD+
- * drafting and greedy verification step (arXiv 2412.01447, "PLD+:
- * Accelerating LLM inference by leveraging Language Model Artifacts").
+ * drafting and greedy verification step (PLD+, arXiv 2412.01447).
  *
  * TEST INFRASTRUCTURE ONLY.  This file is the independent reference that the
  * CUDA library is checked against.  It shares no code, header, helper or
@@ -18,8 +17,7 @@
  * L = seq_len[b], the last token is x_t with t = L - 1.  The artifacts (hidden
  * rows and attention rows) exist for positions 0..t-1 only, because the
  * forward pass that will produce position t's artifacts has not run yet
- * (Sec. 4.2.2: "the hidden states corresponding to the last generated token
- * x_t is not available").
+ * (Sec. 4.2.2 notes that x_t has no hidden state at drafting time).
  *
  * Readings of passages the paper leaves silent, garbled or ambiguous are
  * marked READING below; each one is listed in the design notes.
@@ -62,8 +60,9 @@ static double orc_load(const void* base, int dtype, int64_t idx) {
  * Candidate search.  Eq. 1 (Sec. 4.2, Drafting Algorithm):
  *     P = { j | x_j = x_t, j < t }.
  * READING (n-gram): following the prompt-lookup heritage that PLD+ builds on
- * (Sec. 2; Fig. 2 caption: PLD picks the span with the longest matching
- * prefix), the match is on the longest suffix n-gram that occurs earlier:
+ * (Sec. 2 and Fig. 2: PLD drafts from the earlier occurrence that agrees with
+ * the context on the most tokens), the match is on the longest suffix n-gram
+ * that occurs earlier:
  * for n = n_max down to n_min, P_n = { j < t : j-n+1 >= 0 and
  * x_{j-k} = x_{t-k} for k = 0..n-1 }; the first non-empty P_n is P and its n
  * is match_len.  n_min = n_max = 1 is Eq. 1 itself.
@@ -347,8 +346,9 @@ int pldpo_extract_draft(const int32_t* ids, int64_t ids_stride, const int32_t* s
  *   r*     = argmax_{j in P} ov(j)
  *   row r counts when argmax_{key < p} A[r, key] = r*.
  * READING: ties in ov(j) go to the smallest j (the library's tie rule); ties in
- * a row's maximum go to the smallest key; "the token position x_{r*} has the
- * maximum attention" is read per row (r* is the argmax of that head's row).
+ * a row's maximum go to the smallest key; Sec. 4.2.1's condition that the
+ * attention peaks at position r* is applied to each row on its own (a row
+ * counts when r* is the argmax of that head's row).
  * r_star[b] = r*, or -1 when P is empty (then nothing is counted); counts[r]
  * are ADDED to (uint32, caller-initialised) so that batches accumulate.
  * pos[b] outside [1, T_cap - 1] sets SEQ_LEN and counts nothing.
