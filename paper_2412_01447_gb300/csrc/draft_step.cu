@@ -623,13 +623,13 @@ __global__ void __launch_bounds__(kThreads, 4) draft_step_kernel(const DraftPara
 // ---------------------------------------------------------------------------
 // The incremental token index: drafting without rescanning the context.
 //
-// Per sequence b and token v the index holds one 32-byte entry: how often v
-// occurs among the indexed positions, then up to kIndexSlots of those positions
-// (in no particular order); ilen[b] is the number of positions indexed (0 ..
-// ilen-1), -1 when the index of b is unusable.  A step with t = seq_len - 1:
-//  * reads x_t's entry in one sector; when the count is at most kIndexSlots the
-//    slots are every occurrence before ilen, and the positions appended since
-//    (ilen .. t-1, read anyway) supply the rest;
+// Per sequence b and token v the index holds one 64-byte entry (half a line): how
+// often v occurs among the indexed positions, then up to kIndexSlots of those
+// positions (in no particular order); ilen[b] is the number of positions indexed
+// (0 .. ilen-1), -1 when the index of b is unusable.  A step with t = seq_len - 1:
+//  * reads x_t's entry in one request (a word per lane); when the count is at
+//    most kIndexSlots the slots are every occurrence before ilen, and the
+//    positions appended since (ilen .. t-1, read anyway) supply the rest;
 //  * otherwise (a frequent token, a stale or unusable index) falls back to the
 //    ordered rescan of the context, so results are those of the scan either way;
 //  * appends positions ilen .. t-1 to the index and sets ilen = t.  Each
