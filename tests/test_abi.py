@@ -229,3 +229,45 @@ def test_binding_checks_element_counts_and_shapes():
     # a tensor of the right size still has to be on the device
     with pytest.raises(ValueError, match="CUDA"):
         pk._dense(torch.zeros(4, dtype=torch.int32), "x", torch.int32, n=4)
+
+
+def _c_kind(decl):
+    """('ptr',) for a pointer, (kind, bytes) for a scalar C parameter or return type."""
+    decl = re.sub(r"/\*.*?\*/", "", decl).strip()
+    if "*" in decl:
+        return ("ptr",)
+    words = [w for w in re.split(r"\s+", decl) if w not in ("const", "unsigned", "signed")]
+    base = words[0]
+    scalar = {"int": ("int", 4), "int32_t": ("int", 4), "uint32_t": ("int", 4), "int64_t": ("int", 8),
+              "size_t": ("int", 8), "float": ("float", 4), "double": ("float", 8),
+              "pldp_dtype": ("int", 4), "pldp_agg": ("int", 4), "pldp_status": ("int", 4)}
+    return scalar[base]
+
+
+def _ctypes_kind(t):
+    if t is None:
+        return None
+    if t in (ctypes.c_void_p, ctypes.c_char_p) or issubclass(t, ctypes._Pointer):
+        return ("ptr",)
+    if t in (ctypes.c_float, ctypes.c_double):
+        return ("float", ctypes.sizeof(t))
+    return ("int", ctypes.sizeof(t))
+
+
+def test_binding_signatures_match_the_header(so):
+    """Every call's ctypes argtypes and restype in the binding agree with the
+    prototype in include/pldp.h: the same number of parameters, a pointer where the
+    header has one, and integer and floating scalars of the header's width."""
+    src = re.sub(r"//[^\n]*", "", open(HEADER).read())
+    protos = re.findall(r"PLDP_API\s+([\w\s\*]+?)\b(pldp_\w+)\s*\(([^;]*?)\)\s*;", src, flags=re.S)
+    assert len(protos) == len(declared_symbols())
+    lib = pk._load()
+    for ret, name, params in protos:
+        params = re.sub(r"/\*.*?\*/", "", params, flags=re.S).strip()
+        want = [] if params in ("", "void") else [_c_kind(re.sub(r"\b\w+\s*$", "", p.strip()) or p)
+                                                  for p in params.split(",")]
+        fn = getattr(lib, name)
+        got = [_ctypes_kind(t) for t in (fn.argtypes or [])]
+        assert got == want, (name, got, want)
+        want_ret = ("ptr",) if "*" in ret else _c_kind(ret)
+        assert _ctypes_kind(fn.restype) == want_ret, (name, fn.restype, want_ret)
