@@ -353,6 +353,13 @@ def workload(args):
     return w
 
 
+def workload_name(w):
+    """The workload as the JSON line names it (both arms)."""
+    return (f"sustained decode loop: batch {w.B}, context {w.T} ({w.prompt_len}+{w.out_len}), vocab {w.V}, "
+            f"K={w.K}, max n-gram {w.ngram_max}, bf16 hidden {w.d} + attention {w.layers}x{w.heads} heads, "
+            "both rankings every step")
+
+
 def run_ours(args, ws_, rank, local):
     import paper_2412_01447_gb300 as pk
     pk.build()
@@ -472,10 +479,7 @@ def run_ours(args, ws_, rank, local):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (seeded; copied-span contexts, planted hidden/attention/logit structure)",
-        "config": {"workload": f"sustained decode loop: batch {w.B}, context {w.T} "
-                               f"({w.prompt_len}+{w.out_len}), vocab {w.V}, K={w.K}, max n-gram "
-                               f"{w.ngram_max}, bf16 hidden {w.d} + attention {w.layers}x{w.heads} "
-                               "heads, both rankings every step",
+        "config": {"workload": workload_name(w),
                    "batch_per_gpu": w.B, "context": w.T, "vocab": w.V, "K": w.K, "d": w.d,
                    "attention_rows": w.R, "C_cap": w.C_cap,
                    "l2": ("flushed before every step: 256 MB write then 256 MB read (cold, clean L2)"
@@ -826,9 +830,7 @@ def run_reference(args, ws_, rank):
             "n_gpus": ws_, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(per_step_full * 1e3, 2), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic (same generator as our arm)",
-            "config": {"workload": "sustained decode loop: batch 128, context 32768 (24576+8192), "
-                                   "vocab 128256, K=12, max n-gram 3, bf16 hidden 4096 + attention "
-                                   "4x32 heads, both rankings every step"},
+            "config": {"workload": workload_name(w)},
             "cpu_baseline": {"value": round(value, 4), "unit": "steps/s", "cores": 1, "kind": "oracle",
                              "sample": f"{S} of {w.B} sequences per step, scaled to the full batch"},
             "e2e": {"value": round(value, 4), "unit": "steps/s", "h2d_bytes_per_step": 0,
