@@ -1,6 +1,7 @@
 """Host-side pieces of bench.py on the CPU: the traffic record read from a profile
-summary is used only while the profiled sources are unchanged, and the algorithmic
-byte counts follow the per-unit figures of the measurement section."""
+summary is used only while the profiled sources are unchanged, the algorithmic
+byte counts follow the per-unit figures of the measurement section, and the
+reference arm's line carries the keys of the benchmark's contract."""
 import os
 import sys
 
@@ -41,3 +42,25 @@ def test_step_bytes_follow_the_per_unit_figures():
     assert by["draft_index"] < by["draft_step"] - by["find_candidates"] + B * 64 * 2
     assert by["verify_greedy_draft"] == pytest.approx(by["verify_greedy"] + by["draft_index"])
     assert 426e6 < by["verify_greedy"] < 427e6
+
+
+def test_reference_arm_line_has_the_contract_keys(monkeypatch):
+    """bench.py --impl reference on a shrunken decode loop (the oracle on the host):
+    one JSON-ready dict with the reference arm's keys, its own timing as value, and a
+    cpu_baseline and an e2e that describe this run (no host-device copies)."""
+    small = wl.CONFIGS["decode_loop_b128_ctx32k"].replace(B=4, prompt_len=192, out_len=64, V=300, d=32,
+                                                          layers=1, heads=4, planted_heads=1)
+    monkeypatch.setattr(bench, "workload", lambda args: small)
+    monkeypatch.setattr(sys, "argv", ["bench.py", "--impl", "reference", "--steps", "3", "--warmup", "3"])
+    out = bench.run_reference(bench.parse(), 1, 0)
+    for k in ("impl", "metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+              "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
+        assert k in out, k
+    assert out["impl"] == "reference" and out["unit"] == "steps/s" and out["value"] > 0
+    assert out["steps"] == 3 and out["warmup"] == 3 and out["metric"] == bench.METRIC
+    assert out["config"]["workload"] == bench.workload_name(small)
+    cb = out["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] == out["value"] and "sample" in cb
+    e = out["e2e"]
+    assert e["value"] == out["value"] and e["unit"] == out["unit"]
+    assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
