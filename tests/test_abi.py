@@ -271,3 +271,18 @@ def test_binding_signatures_match_the_header(so):
         assert got == want, (name, got, want)
         want_ret = ("ptr",) if "*" in ret else _c_kind(ret)
         assert _ctypes_kind(fn.restype) == want_ret, (name, fn.restype, want_ret)
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """Without libpldp.so every call raises: there is no CPU path to fall back to."""
+    import torch
+    monkeypatch.setattr(pk._build, "LIB", str(tmp_path / "libpldp.so"))
+    monkeypatch.setattr(pk, "_lib", None)
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        pk.pldp_version()
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        pk.pldp_verify_workspace_size(2, 4, 100)
+    x = torch.zeros((2, 8), dtype=torch.int32)
+    with pytest.raises((RuntimeError, ValueError)):
+        pk.pldp_find_candidates(x, torch.zeros(2, dtype=torch.int32), 1, 3, torch.zeros((2, 4), dtype=torch.int32),
+                                torch.zeros(2, dtype=torch.int32), torch.zeros(2, dtype=torch.int32))
