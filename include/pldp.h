@@ -465,12 +465,15 @@ PLDP_API size_t pldp_verify_sample_workspace_size(int B, int K, int V, pldp_dtyp
  * allocates nothing: it clears the part of the area it uses with
  * cudaMemsetAsync on `stream`, then launches the verification kernels.
  *
- * The first call on each device looks up the area's device address (once per
- * device, on the current device); make that first call before any stream
- * capture.  All calls on a device share the one area, which keeps whatever the
- * last call left there: calls that can overlap on the GPU (different streams,
- * or threads without ordering between them) race on it and must be serialised
- * by the caller.
+ * Every call looks up the area's device address in the CUDA context current on
+ * the calling thread (cudaGetSymbolAddress, which allocates nothing), so a
+ * switch of context or a device reset between calls never leaves it a stale
+ * address.  The first call in a context also makes the runtime load the
+ * library's device code there; make that first call before any stream capture.
+ * All calls on a device share the one area, which keeps whatever the last call
+ * left there: calls that can overlap on the GPU (different streams, or threads
+ * without ordering between them) race on it and must be serialised by the
+ * caller.
  */
 PLDP_API pldp_status pldp_verify_greedy_noalloc(const void* logits, pldp_dtype dtype, int B,
                                                 int K, int V, const int32_t* draft,

@@ -823,7 +823,7 @@ __device__ __forceinline__ void index_draft(const DraftParams& p, const IndexVie
             if (p.status && bad) atomicOr(p.status + b, PLDP_ST_ROW_INDEX);
             // the index now covers 0 .. t-1 (or is unusable: a token it cannot hold, or stale)
             if (usable) ix.ilen[b] = is.bad_token ? -1 : static_cast<int32_t>(t);
-            else if (il > t) ix.ilen[b] = -1;
+            else if (il > t && il > 0) ix.ilen[b] = -1;         // shrunk (an empty context keeps il = 0)
         }
     };
 

@@ -421,39 +421,24 @@ extern "C" PLDP_API pldp_status pldp_verify_greedy(
 // library.  Every GPU that loads the library holds that area until the process
 // exits.
 // ---------------------------------------------------------------------------
-#include <mutex>
-
 namespace pldp {
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = size_t(1) << 20;   // 1 MiB: B*(K+1) up to ~130k rows
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-std::mutex g_noalloc_mutex;
-void* g_noalloc_ptr[kMaxDevices] = {};
-
-// Device address of g_noalloc_scratch on the current device, looked up once per
-// device.  In host code the array's name only stands in for the symbol; the
-// kernel must be given this address instead.
+// Device address of g_noalloc_scratch in the CUDA context current on this thread.
+// In host code the array's name only stands in for the symbol; the kernels must
+// be given this address instead.  It is looked up on every call, not cached: the
+// address belongs to a context, and a caller may switch contexts or reset the
+// device between calls.  cudaGetSymbolAddress allocates nothing.
 pldp_status noalloc_scratch(void** out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess)
-        return fail(PLDP_ERR_CUDA, "verify_greedy_noalloc: cudaGetDevice: %s", cudaGetErrorString(e));
-    if (dev < 0 || dev >= kMaxDevices)
-        return fail(PLDP_ERR_UNSUPPORTED, "verify_greedy_noalloc: device %d beyond %d", dev, kMaxDevices);
-    std::lock_guard<std::mutex> lock(g_noalloc_mutex);
-    if (!g_noalloc_ptr[dev]) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess || !p)
-            return fail(PLDP_ERR_CUDA, "verify_greedy_noalloc: cudaGetSymbolAddress: %s",
-                        cudaGetErrorString(e));
-        g_noalloc_ptr[dev] = p;
-    }
-    *out = g_noalloc_ptr[dev];
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess || !p)
+        return fail(PLDP_ERR_CUDA, "verify_greedy_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+    *out = p;
     return PLDP_OK;
 }
 

@@ -92,6 +92,43 @@ def gpu_step(buf, ids, seq_len, logits, ngram=(1, 3), H=None, A=None, row_idx=No
                               stream=stream)
 
 
+def oracle_rows(H, A, seq_len, cand, cnt):
+    """Host copies of H [B, T_cap, d] and A [B, R, T_cap] (device tensors, or None)
+    that hold exactly what the oracle's rankings read for these candidate lists: per
+    sequence the query row H_{t-1} and each listed candidate's H_{j-1}, and each
+    listed candidate's key column A[:, j].  The rest of each host array is zero
+    pages that are never touched, so full-size tensors fit in host memory.  The
+    candidate lists are the oracle's own (never the GPU's)."""
+    B = len(seq_len)
+    bh, rh, ba, ja = [], [], [], []
+    for b in range(B):
+        L = int(seq_len[b])
+        T_cap = (H if H is not None else A).shape[1 if H is not None else 2]
+        t = L - 1
+        if t < 1 or L > T_cap:
+            continue
+        n = max(0, min(int(cnt[b]), cand.shape[1]))
+        js = cand[b, :n].astype(np.int64)
+        js = js[(js >= 0) & (js < t)]
+        rows = np.unique(np.concatenate([js[js >= 1] - 1, [t - 1]]))
+        bh += [b] * rows.size
+        rh += rows.tolist()
+        ba += [b] * js.size
+        ja += js.tolist()
+    Hs = As = None
+    if H is not None:
+        Hs = np.zeros(tuple(H.shape), np.uint16 if H.dtype == torch.bfloat16 else np.float32)
+        if bh:
+            bi, ri = np.asarray(bh), np.asarray(rh)
+            Hs[bi, ri] = host(H[torch.as_tensor(bi, device=H.device), torch.as_tensor(ri, device=H.device)])
+    if A is not None:
+        As = np.zeros(tuple(A.shape), np.uint16 if A.dtype == torch.bfloat16 else np.float32)
+        if ba:
+            bi, ji = np.asarray(ba), np.asarray(ja)
+            As[bi, :, ji] = host(A[torch.as_tensor(bi, device=A.device), :, torch.as_tensor(ji, device=A.device)])
+    return Hs, As
+
+
 def snapshot(buf):
     torch.cuda.synchronize()
     return {k: host(v) for k, v in vars(buf).items() if k not in ("ws", "dws")}

@@ -1,11 +1,13 @@
 """The incremental token index of pldp_draft_step: every output must equal the
 scanning step's bit for bit (same candidates, counts, match lengths, scores,
-choices, drafts, status), over random contexts, a decode loop with greedy
-appends, long appends, shrunk contexts and tokens the index cannot hold."""
+choices, drafts, status), and the oracle's at every step, over random contexts,
+a decode loop with greedy appends, long appends, shrunk and empty contexts and
+tokens the index cannot hold."""
 import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2412_01447_gb300 as pk
 import workloads as wl
 from tests._parity import Buffers, gpu_step, host, snapshot
@@ -67,6 +69,8 @@ def _indexed_case(T, V, B, mode, C, K, ngram):
     lens = rng.integers(0, T + 1, size=B)
     lens[:3] = [T, 1, 2]
     lens[3] = T_cap + 3                                              # invalid length
+    if B > 6:
+        lens[6] = 0                                                  # empty, then grows
     H = torch.randn((B, T_cap, d), generator=gen, device=DEV).to(torch.bfloat16) if mode != "attention" else None
     A = torch.rand((B, R, T_cap), generator=gen, device=DEV).to(torch.bfloat16) if mode != "hidden" else None
     draft_from = "attention" if mode == "attention" else "hidden"
@@ -80,8 +84,7 @@ def _indexed_case(T, V, B, mode, C, K, ngram):
         g_scan = _draft(a, ids_g, L_g, K, H, A, ngram=ngram, draft_from=draft_from)
         g_idx = _draft(b_, ids_g, L_g, K, H, A, index=index, V=V, ngram=ngram, draft_from=draft_from)
         _same(g_scan, g_idx)
-        if step == 0:
-            _compare(g_idx, ids, lens, H, A, None, 0, ngram, C, K, draft_from)
+        _compare(g_idx, ids, lens, H, A, None, 0, ngram, C, K, draft_from)     # every step against the oracle
         # the contexts grow: 1..13 tokens, one long append, one sequence cut back
         L = host(L_g).astype(np.int64)
         for s in range(B):
@@ -98,6 +101,8 @@ def _indexed_case(T, V, B, mode, C, K, ngram):
         L_g.copy_(i32(lens))
     il = _ilen(index, B)
     assert il[3] == -1 and il[5] == -1
+    if B > 6:
+        assert il[6] >= 0                                            # the context that was empty kept its index
 
 
 def test_index_marks_tokens_it_cannot_hold(lib):
@@ -129,10 +134,15 @@ def test_indexed_decode_loop(lib):
     a, b_ = Buffers(B, K, w.V, C, DEV), Buffers(B, K, w.V, C, DEV)
     for s in range(steps):
         loop.step_inputs(s)
-        _same(_draft(a, loop.ids, loop.seq_len, K, loop.H, loop.A),
-              _draft(b_, loop.ids, loop.seq_len, K, loop.H, loop.A, index=index, V=w.V))
+        ids0, L0 = host(loop.ids), host(loop.seq_len)
+        g_idx = _draft(b_, loop.ids, loop.seq_len, K, loop.H, loop.A, index=index, V=w.V)
+        _same(_draft(a, loop.ids, loop.seq_len, K, loop.H, loop.A), g_idx)
+        _compare(g_idx, ids0, L0, loop.H, loop.A, None, 0, (w.ngram_min, w.ngram_max), C, K, "hidden")
         pk.pldp_verify_greedy(loop.logits, b_.draft, b_.dlen, b_.acc, b_.nxt, b_.ws, ids=loop.ids,
                               seq_len=loop.seq_len, kv_keep_len=b_.kv, status=b_.status)
+        o = oracle.verify_greedy(host(loop.logits), g_idx["draft"], g_idx["dlen"], ids=ids0, seq_len=L0)
+        assert np.array_equal(host(b_.acc), o["accept_len"]) and np.array_equal(host(b_.nxt), o["next_token"])
+        assert np.array_equal(host(loop.ids), ids0) and np.array_equal(host(loop.seq_len), L0)
     torch.cuda.synchronize()
     L = host(loop.seq_len)
     il = _ilen(index, B)

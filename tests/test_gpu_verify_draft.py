@@ -151,6 +151,8 @@ def _verify_draft_case(T, V, B, mode, shared, K, C, ngram, dt):
     st = host(b_.status).view(np.uint32)
     assert st[0] & pk.PLDP_ST_CAPACITY and st[1] & pk.PLDP_ST_SEQ_LEN and st[2] & pk.PLDP_ST_DRAFT_LEN
     assert st[4] & pk.PLDP_ST_SEQ_LEN and host(L_b)[4] == 0 and host(L_b)[3] > 1
+    for ix in (ix_a, ix_b):                   # the empty context's index stays usable (nothing indexed)
+        assert host(ix[:4 * B].view(torch.int32))[4] == 0
     assert (host(b_.ws) == 0).all()           # the verification workspace is left zero
 
 
