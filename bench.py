@@ -72,7 +72,10 @@ def parse():
                          "pldp_verify_greedy_draft call (which verifies a step and drafts the next)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sample", action="store_true",
-                    help="skip the separate timing of sampling verification (T = 1) on the same logits")
+                    help="skip the separate timings on the loop's tensors (rank stress, sampling verification, "
+                         "averaged ranking, head identification)")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the per-call timing of the four single-step workloads")
     ap.add_argument("--ref-seqs", type=int, default=2, help="sequences per oracle step (reference arm)")
     ap.add_argument("--batch", type=int, default=None, help="override the batch (not the headline)")
     ap.add_argument("--hidden-width", type=int, default=None,
@@ -360,6 +363,19 @@ def workload_name(w):
             "both rankings every step")
 
 
+def bench_config(w, args, ws_):
+    """The JSON line's ``config``: the workload and the timing protocol, the same dict
+    on both arms."""
+    return {"workload": workload_name(w),
+            "batch_per_gpu": w.B, "context": w.T, "vocab": w.V, "K": w.K, "d": w.d,
+            "attention_rows": w.R, "C_cap": w.C_cap,
+            "l2": ("flushed before every step: 256 MB write then 256 MB read (cold, clean L2)"
+                   if args.flush == "write-read" else
+                   "flushed before every step: 256 MB write (cold L2 holding dirty lines)")
+                  + "; per-step logits 427 MB and attention rows 1.18 GB regenerated between steps",
+            "parallelism": f"{ws_} independent replicas (batch shards)"}
+
+
 def run_ours(args, ws_, rank, local):
     import paper_2412_01447_gb300 as pk
     pk.build()
@@ -479,23 +495,16 @@ def run_ours(args, ws_, rank, local):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (seeded; copied-span contexts, planted hidden/attention/logit structure)",
-        "config": {"workload": workload_name(w),
-                   "batch_per_gpu": w.B, "context": w.T, "vocab": w.V, "K": w.K, "d": w.d,
-                   "attention_rows": w.R, "C_cap": w.C_cap,
-                   "l2": ("flushed before every step: 256 MB write then 256 MB read (cold, clean L2)"
-                          if args.flush == "write-read" else
-                          "flushed before every step: 256 MB write (cold L2 holding dirty lines)")
-                         + "; per-step logits 427 MB and attention rows 1.18 GB regenerated between steps",
-                   "path": ("pldp_verify_greedy_draft per step: this step's greedy verification, then the "
-                            "next step's drafting with the incremental token index (both rankings + draft); "
-                            "the first draft (pldp_draft_step) precedes the warm-up" if path.vd else
-                            ("pldp_draft_step (incremental token index + both rankings + draft)"
-                             if path.index is not None else
-                             "pldp_draft_step (fused scan + both rankings + draft)") + " + pldp_verify_greedy"
-                            if path.fused else "five separate C-ABI calls"),
-                   "timing": "CUDA events around every C-ABI call of each step on the launch stream; "
-                             "artifact generation between steps is not timed",
-                   "parallelism": f"{ws_} independent replicas (batch shards)"},
+        "config": bench_config(w, args, ws_),
+        "path": ("pldp_verify_greedy_draft per step: this step's greedy verification, then the next step's "
+                 "drafting with the incremental token index (both rankings + draft); the first draft "
+                 "(pldp_draft_step) precedes the warm-up" if path.vd else
+                 ("pldp_draft_step (incremental token index + both rankings + draft)"
+                  if path.index is not None else
+                  "pldp_draft_step (fused scan + both rankings + draft)") + " + pldp_verify_greedy"
+                 if path.fused else "five separate C-ABI calls"),
+        "timing": "CUDA events around every C-ABI call of each step on the launch stream; "
+                  "artifact generation between steps is not timed",
         "achieved_step_gbs": round(step_bytes_total / (ms_per_step / 1e3) / 1e9, 1),
         "frac_step_of_nominal_8tbs": round(step_bytes_total / (ms_per_step / 1e3) / 1e9 / NOMINAL_HBM_GBS, 4),
         "kernel_us": {k: round(per_k[i] / K_steps * 1e3, 2) for i, k in enumerate(path.kernels)},
@@ -520,9 +529,12 @@ def run_ours(args, ws_, rank, local):
     if path.index is not None:
         out["draft_scan_variant"] = time_scan_variant(pk, loop, w, flush_l2)
     if not args.no_sample:
+        out["rank_stress"] = time_rank_stress(pk, loop, w, flush_l2, peak)
         out["sampling_verify"] = time_sampling_verify(pk, loop, w, flush_l2, peak)
         out["rank_hidden_avg"] = time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak)
         out["identify_heads"] = time_identify_heads(pk, loop, w, flush_l2, peak)
+    if not args.no_configs:
+        out["configs"] = time_single_step_configs(pk, flush_l2, peak)
     if not args.no_e2e:
         out["e2e"] = run_e2e(pk, loop, path, K_steps, W_steps, ws_)
     if rank == 0 and ws_ == 1 and not args.no_cpu_baseline:
@@ -670,6 +682,159 @@ def time_identify_heads(pk, loop, w, flush_l2, peak, calls=16, warm=2):
             "achieved_gbs": round(by / (us * 1e-6) / 1e9, 1), "peak_gbs": peak,
             "frac": round(by / (us * 1e-6) / 1e9 / peak, 4), "top_rows_are_the_planted_heads": recovered,
             "timing": "CUDA events around pldp_identify_heads + pldp_top_heads, L2 flushed before each"}
+
+
+def _time_calls(calls, flush_l2, iters, warm, reset=None):
+    """Times a sequence of C-ABI calls: before each iteration ``reset()`` (not timed)
+    and an L2 flush, then CUDA events on the launch stream before the first call and
+    after every call.  Returns {name: [us per iteration]}."""
+    s = torch.cuda.current_stream()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(calls) + 1)] for _ in range(iters)]
+    for i in range(warm + iters):
+        if reset is not None:
+            reset()
+        flush_l2(i)
+        e = ev[i - warm] if i >= warm else None
+        if e is not None:
+            e[0].record(s)
+        for k, (_, fn) in enumerate(calls):
+            fn()
+            if e is not None:
+                e[k + 1].record(s)
+    torch.cuda.synchronize()
+    return {name: [e[k].elapsed_time(e[k + 1]) * 1e3 for e in ev] for k, (name, _) in enumerate(calls)}
+
+
+def _call_stats(us, by, peak):
+    m = float(np.mean(us))
+    return {"us": round(m, 2), "us_p50": round(float(np.percentile(us, 50)), 2), "algorithmic_bytes": by,
+            "gbs": round(by / (m * 1e-6) / 1e9, 1), "frac": round(by / (m * 1e-6) / 1e9 / peak, 4)}
+
+
+SINGLE_STEP = ("one_step_b1_ctx512", "hidden_b8_ctx4k", "hidden_b64_ctx16k", "attention_b32_ctx8k")
+
+
+def time_single_step_configs(pk, flush_l2, peak, iters=32, warm=3):
+    """The four single-step workloads: one decode step each (the state restored before
+    every iteration), timed per C-ABI call and for the whole step with CUDA events,
+    L2 flushed before each step.  Two forms of the step: the five separate calls
+    (candidate search, the workload's ranking, draft, greedy verification with append)
+    and the fused drafting launch + verification.  Algorithmic bytes per call are the
+    per-unit figures: 4 B per context position scanned, (|P| + 1) * d * s of hidden
+    rows, |P| * R * 2 B of attention values (32 B sectors in practice), K * 4 B of
+    draft, (K + 1) * V * s of logits."""
+    dev = torch.device("cuda", torch.cuda.current_device())
+    out = {}
+    for name in SINGLE_STEP:
+        w = wl.CONFIGS[name]
+        inp = wl.single_step(w, device=dev)
+        B, K, C = w.B, w.K, w.C_cap
+        ids, L = inp["ids"], inp["seq_len"]
+        ids0, L0 = ids.clone(), L.clone()
+        H, A, logits = inp["H"], inp["A"], inp["logits"]
+        i32 = dict(dtype=torch.int32, device=dev)
+        cand, cnt, ml, st = torch.zeros((B, C), **i32), torch.zeros(B, **i32), torch.zeros(B, **i32), \
+            torch.zeros(B, **i32)
+        best_h, best_a = torch.zeros(B, **i32), torch.zeros(B, **i32)
+        draft, dlen = torch.zeros((B, K), **i32), torch.zeros(B, **i32)
+        acc, nxt, kv = torch.zeros(B, **i32), torch.zeros(B, **i32), torch.zeros(B, **i32)
+        ws = torch.zeros(pk.pldp_verify_workspace_size(B, K, w.V), dtype=torch.uint8, device=dev)
+        dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=dev)
+        best = best_h if H is not None else best_a
+
+        def reset():
+            ids.copy_(ids0)
+            L.copy_(L0)
+
+        def verify():
+            pk.pldp_verify_greedy(logits, draft, dlen, acc, nxt, ws, ids=ids, seq_len=L, kv_keep_len=kv,
+                                  status=st)
+        calls = [("find_candidates", lambda: pk.pldp_find_candidates(ids, L, w.ngram_min, w.ngram_max, cand, cnt,
+                                                                     ml, st))]
+        if H is not None:
+            calls.append(("rank_hidden", lambda: pk.pldp_rank_hidden(H, L, cand, cnt, best_h, status=st)))
+        if A is not None:
+            calls.append(("rank_attention", lambda: pk.pldp_rank_attention(A, L, cand, cnt, best_a, status=st)))
+        calls += [("extract_draft", lambda: pk.pldp_extract_draft(ids, L, best, draft, dlen)),
+                  ("verify_greedy", verify)]
+        sep = _time_calls(calls, flush_l2, iters, warm, reset)
+        fused = _time_calls([("draft_step", lambda: pk.pldp_draft_step(
+            ids, L, w.ngram_min, w.ngram_max, cand, cnt, ml, K, draft, dlen, dws, H=H, best_h=best_h if H is not None
+            else None, A=A, best_a=best_a if A is not None else None,
+            draft_from="hidden" if H is not None else "attention", status=st)), ("verify_greedy", verify)],
+            flush_l2, iters, warm, reset)
+        torch.cuda.synchronize()
+        n_list = float(cnt.clamp(0, C).sum().item())
+        s_h = H.element_size() if H is not None else 0
+        by = {"find_candidates": 4.0 * float(L0.double().sum().item()),
+              "rank_hidden": (n_list + B) * (w.d or 0) * s_h,
+              "rank_attention": n_list * w.R * 2.0,
+              "extract_draft": 4.0 * B * K,
+              "verify_greedy": float(B * (K + 1) * w.V * logits.element_size())}
+        by["draft_step"] = by["find_candidates"] + by["extract_draft"] + (
+            by["rank_hidden"] if H is not None else by["rank_attention"])
+        rec = {"B": B, "context": w.T, "V": w.V, "K": K, "candidates_listed": int(n_list),
+               "separate_calls": {k: _call_stats(v, by[k], peak) for k, v in sep.items()},
+               "fused": {k: _call_stats(v, by[k], peak) for k, v in fused.items()}}
+        for form, times in (("separate_calls", sep), ("fused", fused)):
+            step = np.sum([np.asarray(v) for v in times.values()], axis=0)
+            tot = sum(by[k] for k in times)
+            rec[form]["step"] = _call_stats(step, tot, peak)
+        if A is not None:
+            rec["separate_calls"]["rank_attention"]["sector_bytes"] = n_list * w.R * 32.0
+        out[name] = rec
+        del inp, H, A, logits, ids, L, ids0, L0
+        torch.cuda.empty_cache()
+    out["timing"] = ("CUDA events before the first and after every call of one step, state restored and L2 "
+                     "flushed before each step; us = mean over the timed steps")
+    return out
+
+
+def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
+    """Candidate-heavy ranking, reported apart from the headline: the decode loop's
+    batch, context and artifacts (bf16 hidden rows of width d, R attention rows) with
+    contexts drawn from a small vocabulary and Eq. 1's unigram match (n-gram 1..1),
+    so that x_t has hundreds of earlier occurrences and the rankings have bytes to
+    move.  Each call timed with CUDA events, L2 flushed before each; the candidate
+    lists come from one untimed pldp_find_candidates call."""
+    dev = loop.device
+    B, T, C = w.B, w.T, w.C_cap
+    T_cap = loop.T_cap
+    i32 = dict(dtype=torch.int32, device=dev)
+    L = torch.full((B,), T, **i32)
+    cand, cnt, ml = torch.zeros((B, C), **i32), torch.zeros(B, **i32), torch.zeros(B, **i32)
+    best_h, best_a = torch.zeros(B, **i32), torch.zeros(B, **i32)
+    draft, dlen = torch.zeros((B, w.K), **i32), torch.zeros(B, **i32)
+    dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=dev)
+    out = {}
+    for V in (256, 64):
+        g = torch.Generator(device=dev).manual_seed(w.seed + V)
+        ids = torch.randint(0, V, (B, T_cap), generator=g, device=dev, dtype=torch.int32)
+        pk.pldp_find_candidates(ids, L, 1, 1, cand, cnt, ml)
+        torch.cuda.synchronize()
+        n_list = float(cnt.clamp(0, C).sum().item())
+        calls = [("rank_hidden", lambda: pk.pldp_rank_hidden(loop.H, L, cand, cnt, best_h)),
+                 ("rank_attention", lambda: pk.pldp_rank_attention(loop.A, L, cand, cnt, best_a))]
+        times = {}
+        for c in calls:
+            times.update(_time_calls([c], flush_l2, iters, warm))
+        by = {"rank_hidden": (n_list + B) * w.d * 2.0, "rank_attention": n_list * w.R * 2.0}
+        rec = {"vocab": V, "ngram": [1, 1], "mean_candidates_listed": round(n_list / B, 1),
+               **{k: _call_stats(v, by[k], peak) for k, v in times.items()}}
+        rec["rank_attention"]["sector_bytes"] = n_list * w.R * 32.0
+        rec["rank_attention"]["sector_gbs"] = round(n_list * w.R * 32.0 / (rec["rank_attention"]["us"] * 1e-6) / 1e9, 1)
+        if V == 256:      # at most 256 occurrences per sequence: the launch's own scoring path
+            t = _time_calls([("draft_step", lambda: pk.pldp_draft_step(
+                ids, L, 1, 1, cand, cnt, ml, w.K, draft, dlen, dws, H=loop.H, best_h=best_h, A=loop.A,
+                best_a=best_a, draft_from="hidden"))], flush_l2, iters, warm)
+            by_d = 4.0 * B * T + by["rank_hidden"] + by["rank_attention"] + 4.0 * B * w.K
+            rec["draft_step"] = _call_stats(t["draft_step"], by_d, peak)
+        out[f"vocab{V}"] = rec
+        del ids
+    out.update({"batch": B, "context": T, "d": w.d, "attention_rows": w.R, "C_cap": C,
+                "timing": "CUDA events around each call, L2 flushed before each; hidden rows and attention "
+                          "values are the decode loop's own tensors"})
+    return out
 
 
 def path_draft(loop, w):
@@ -830,7 +995,9 @@ def run_reference(args, ws_, rank):
             "n_gpus": ws_, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(per_step_full * 1e3, 2), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic (same generator as our arm)",
-            "config": {"workload": workload_name(w)},
+            "config": bench_config(w, args, ws_),
+            "timing": "host wall clock around each oracle step on host-resident inputs (the config's L2 "
+                      "protocol is the GPU arm's)",
             "cpu_baseline": {"value": round(value, 4), "unit": "steps/s", "cores": 1, "kind": "oracle",
                              "sample": f"{S} of {w.B} sequences per step, scaled to the full batch"},
             "e2e": {"value": round(value, 4), "unit": "steps/s", "h2d_bytes_per_step": 0,

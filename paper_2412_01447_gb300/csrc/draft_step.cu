@@ -106,10 +106,6 @@ __device__ __forceinline__ uint4* seq_entries(unsigned char* ws, int b) {
     return reinterpret_cast<uint4*>(ws + static_cast<size_t>(b) * kSeqWs + 16);
 }
 
-__device__ __forceinline__ void prefetch_l2_bulk(const void* ptr, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
-}
-
 struct Hit {
     int32_t j, m;
 };

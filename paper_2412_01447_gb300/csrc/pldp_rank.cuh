@@ -7,9 +7,12 @@
 // S CTAs serve a sequence; candidate i belongs to CTA i mod S.  A CTA scores its
 // candidates P at a time (P = 1, 2, 4 or 8, the largest not above its count)
 // with 8 / P warps per candidate, each warp taking an interleaved share of the
-// row, so that one candidate is read by the whole CTA in one DRAM round trip
-// while many candidates stream with one warp each.  Partial sums meet in shared
-// memory and are combined in a fixed order: results are deterministic.
+// row, so that one candidate is read by the whole CTA in one DRAM round trip.
+// Partial sums meet in shared memory and are combined in a fixed order: results
+// are deterministic.  With 8 or more candidates per CTA (one warp per candidate)
+// the warps run on their own instead: each streams its candidates in turn with
+// no CTA barrier between them, and keeps the rows of its next candidates coming
+// into L2 with bulk prefetches, so that many rows are in flight per SM.
 //
 // Argmax keys pack (score, position): the larger score wins, equal scores go to
 // the smaller position, whatever the order of reduction.
@@ -24,6 +27,18 @@ namespace pldp {
 constexpr int kRankThreads = 256;
 constexpr int kRankWarps = kRankThreads / 32;
 constexpr int kRowUnroll = 8;                 // 16-byte loads in flight per lane
+constexpr int kLookahead = 2;                 // candidates per warp whose rows are prefetched into L2
+#ifdef PLDP_TEST_STUCK_QUERY_WAIT
+constexpr uint32_t kQueryPolls = 1u << 12;    // test build: a short bound on the wait for the query row
+#else
+constexpr uint32_t kQueryPolls = kMbarPolls;
+#endif
+
+// Brings `bytes` (a multiple of 16, 16-byte aligned) at ptr into L2: one bulk
+// prefetch, no registers held, no completion to wait for.
+__device__ __forceinline__ void prefetch_l2_bulk(const void* ptr, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(ptr), "r"(bytes) : "memory");
+}
 
 struct RankShared {
     float part[kRankWarps][3];                 // per-warp partial sums of the current batch
@@ -117,6 +132,95 @@ __device__ __forceinline__ float finish_cosine(float dot, float na, float nq) {
     return dot * rsqrtf(na) * rsqrtf(nq);
 }
 
+// Position of this CTA's k-th candidate (list index i): the first batch's from
+// `jpre` (shared), the others from the candidate row.
+template <bool CANDS_SHARED>
+__device__ __forceinline__ int64_t cand_at(const int32_t* __restrict__ cands, const int32_t* jpre, int k, int i,
+                                           int P) {
+    if (k < P && jpre) return jpre[k];
+    return CANDS_SHARED ? cands[i] : __ldcg(cands + i);
+}
+
+// Eq. 3 with one warp per candidate (G = 1): warp `slot` scores candidates slot,
+// slot + P, ... of this CTA on its own.  Lane 0 keeps the rows of the warp's next
+// kLookahead candidates on their way into L2; their positions are read one
+// iteration before they are needed, so the prefetches never wait.
+template <typename T, bool CANDS_SHARED>
+__device__ __forceinline__ void hidden_rank_warp(const T* __restrict__ hb, int64_t d, int64_t t,
+                                                 const int32_t* __restrict__ cands, int S, int rank,
+                                                 const int32_t* jpre, const T* q_sh, uint64_t* bar, bool q_pending,
+                                                 float threshold, float* __restrict__ scores_row, RankShared& sh,
+                                                 const Batch& bt) {
+    constexpr int E = 16 / sizeof(T);
+    const int lane = threadIdx.x & 31;
+    const int P = bt.P;
+    const int64_t nch = d / E;
+    const uint32_t row_bytes = static_cast<uint32_t>(d * sizeof(T));
+    auto cand = [&](int k) -> int64_t { return cand_at<CANDS_SHARED>(cands, jpre, k, rank + S * k, P); };
+    auto prefetch_row = [&](int64_t j) {
+        if (j >= 1 && j < t) prefetch_l2_bulk(hb + (j - 1) * d, row_bytes);
+    };
+    int64_t jnext = -1;                                   // lane 0: position of candidate k + kLookahead * P
+    if (lane == 0) {
+        for (int a = 1; a < kLookahead; ++a)
+            if (bt.slot + a * P < bt.n_local) prefetch_row(cand(bt.slot + a * P));
+        if (bt.slot + kLookahead * P < bt.n_local) jnext = cand(bt.slot + kLookahead * P);
+    }
+    bool q_ready = !q_pending, timed_out = false;
+    unsigned long long best = 0;
+    for (int k = bt.slot; k < bt.n_local; k += P) {
+        const int i = rank + S * k;
+        const int64_t j = cand(k);
+        if (lane == 0) {
+            prefetch_row(jnext);
+            const int kn = k + (kLookahead + 1) * P;
+            jnext = kn < bt.n_local ? cand(kn) : -1;
+        }
+        const bool ok = j >= 1 && j < t;
+        float dot = 0.f, na = 0.f, nq = 0.f;
+        if (ok) {
+            const T* row = hb + (j - 1) * d;              // H_{j-1}
+            for (int64_t c0 = lane; c0 < nch; c0 += 32 * kRowUnroll) {
+                uint4 a[kRowUnroll];
+#pragma unroll
+                for (int u = 0; u < kRowUnroll; ++u) {
+                    const int64_t c = c0 + 32 * u;
+                    if (c < nch) a[u] = ld_stream16(row + c * E);
+                }
+                if (!q_ready) {
+                    if (!mbar_wait(bar, 0, kQueryPolls)) timed_out = true;
+                    q_ready = true;
+                }
+                if (timed_out) break;
+#pragma unroll
+                for (int u = 0; u < kRowUnroll; ++u) {
+                    const int64_t c = c0 + 32 * u;
+                    if (c < nch) {
+                        const uint4 q = *reinterpret_cast<const uint4*>(q_sh + c * E);
+                        accum16<T>(a[u], q, dot, na, nq);
+                    }
+                }
+            }
+        }
+        if (__any_sync(0xFFFFFFFFu, timed_out)) {
+            if (lane == 0) sh.err = 1;
+            break;
+        }
+        dot = warp_sum(dot);
+        na = warp_sum(na);
+        nq = warp_sum(nq);
+        if (lane == 0) {
+            const float s = ok ? finish_cosine(0.f + dot, 0.f + na, 0.f + nq) : -INFINITY;   // as the CTA path sums
+            if (scores_row) scores_row[i] = s;
+            if (ok && s > threshold) {
+                const unsigned long long key = pack_key(s, static_cast<uint32_t>(j));
+                best = key > best ? key : best;
+            }
+        }
+    }
+    if (lane == 0 && best > sh.slot_key[bt.slot]) sh.slot_key[bt.slot] = best;
+}
+
 // Eq. 3 for this CTA's candidates.  `hb` is the sequence's hidden slice, `cands`
 // its candidate row, `q_sh` the query row H_{t-1} in shared memory -- complete,
 // or (q_pending) still arriving through `bar`, waited for before its first use.
@@ -134,6 +238,14 @@ __device__ __forceinline__ void hidden_rank_cta(const T* __restrict__ hb, int64_
                                                 const WarpGroup& wg = whole_cta()) {
     const int lane = threadIdx.x & 31, warp = wg.warp();
     const Batch bt = batch_shape(n, S, rank, wg);
+    if constexpr (VEC) {
+        if (bt.G == 1) {                                  // one warp per candidate: no barriers
+            hidden_rank_warp<T, CANDS_SHARED>(hb, d, t, cands, S, rank, jpre, q_sh, bar, q_pending, threshold,
+                                              scores_row, sh, bt);
+            wg.sync();
+            return;
+        }
+    }
     bool q_ready = !q_pending, timed_out = false;
     for (int k0 = 0; k0 < bt.n_local; k0 += bt.P) {
         const int k = k0 + bt.slot;
@@ -157,7 +269,7 @@ __device__ __forceinline__ void hidden_rank_cta(const T* __restrict__ hb, int64_
                         if (c < nch) a[u] = ld_stream16(row + c * E);
                     }
                     if (!q_ready) {
-                        if (!mbar_wait(bar, 0, kMbarPolls)) timed_out = true;
+                        if (!mbar_wait(bar, 0, kQueryPolls)) timed_out = true;
                         q_ready = true;
                     }
                     if (timed_out) break;
@@ -217,6 +329,70 @@ __device__ __forceinline__ float load_attn(const void* base, int64_t idx, bool a
     return static_cast<const float*>(base)[idx];
 }
 
+// Eq. 2 with one warp per candidate (G = 1): warp `slot` takes candidates slot,
+// slot + P, ... of this CTA two at a time, on its own (no CTA barrier), so twice
+// the scattered values are in flight.  Lane sums run in the order of the CTA path.
+template <bool CANDS_SHARED>
+__device__ __forceinline__ void attention_rank_warp(const void* ab, bool a_bf16, const int64_t* rows_sh, int n_sel,
+                                                    int64_t t, const int32_t* __restrict__ cands, int S, int rank,
+                                                    const int32_t* jpre, bool is_max, float* __restrict__ scores_row,
+                                                    RankShared& sh, const Batch& bt) {
+    const int lane = threadIdx.x & 31;
+    const int P = bt.P;
+    constexpr int U = 4;
+    unsigned long long best = 0;
+    for (int k = bt.slot; k < bt.n_local; k += 2 * P) {
+        int64_t j[2];
+        bool act[2], ok[2];
+        float acc[2];
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+            const int kk = k + c * P;
+            act[c] = kk < bt.n_local;
+            j[c] = act[c] ? cand_at<CANDS_SHARED>(cands, jpre, kk, rank + S * kk, P) : -1;
+            ok[c] = act[c] && j[c] >= 0 && j[c] < t;
+            acc[c] = is_max ? -INFINITY : 0.0f;
+        }
+        for (int r0 = lane; r0 < n_sel; r0 += 32 * U) {
+            float v[2][U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int r = r0 + 32 * u;
+                const int64_t off = (r < n_sel) ? rows_sh[r] : -1;
+#pragma unroll
+                for (int c = 0; c < 2; ++c) v[c][u] = (ok[c] && off >= 0) ? load_attn(ab, off + j[c], a_bf16) : NAN;
+            }
+#pragma unroll
+            for (int c = 0; c < 2; ++c)
+#pragma unroll
+                for (int u = 0; u < U; ++u)
+                    if (v[c][u] == v[c][u]) acc[c] = is_max ? fmaxf(acc[c], v[c][u]) : acc[c] + v[c][u];
+        }
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+            if (is_max) {
+#pragma unroll
+                for (int o = 16; o > 0; o >>= 1) acc[c] = fmaxf(acc[c], __shfl_xor_sync(0xFFFFFFFFu, acc[c], o));
+            } else {
+                acc[c] = warp_sum(acc[c]);
+            }
+        }
+        if (lane == 0) {
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                if (!act[c]) continue;
+                const float s = ok[c] ? acc[c] : -INFINITY;
+                if (scores_row) scores_row[rank + S * (k + c * P)] = s;
+                if (ok[c]) {
+                    const unsigned long long key = pack_key(s, static_cast<uint32_t>(j[c]));
+                    best = key > best ? key : best;
+                }
+            }
+        }
+    }
+    if (lane == 0 && best > sh.slot_key[bt.slot]) sh.slot_key[bt.slot] = best;
+}
+
 // Eq. 2 for this CTA's candidates.  `rows_sh` (shared) holds the element offset
 // of each selected row, or -1 for an invalid one.  Same conventions as
 // hidden_rank_cta; every candidate in [0, t) is eligible.  With CANDS_SHARED
@@ -230,6 +406,12 @@ __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
                                                    const WarpGroup& wg = whole_cta()) {
     const int lane = threadIdx.x & 31, warp = wg.warp();
     const Batch bt = batch_shape(n, S, rank, wg);
+    if (bt.G == 1) {                                      // one warp per candidate: no barriers
+        attention_rank_warp<CANDS_SHARED>(ab, a_bf16, rows_sh, n_sel, t, cands, S, rank, jpre, is_max, scores_row,
+                                          sh, bt);
+        wg.sync();
+        return;
+    }
     constexpr int U = 4;
     for (int k0 = 0; k0 < bt.n_local; k0 += bt.P) {
         const int k = k0 + bt.slot;

@@ -98,6 +98,15 @@ rank_hidden_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride,
     __shared__ RankShared sh;
     __shared__ CtaBest mine;
     __shared__ __align__(8) uint64_t bar;
+#ifdef PLDP_TEST_STUCK_QUERY_WAIT
+    // Test build only: the scoring warps wait for the query on a barrier that
+    // nothing arrives on, so that their bounded wait runs out (the TIMEOUT path);
+    // the copy itself still completes on `bar`, which is waited for before exit.
+    __shared__ __align__(8) uint64_t stuck;
+    uint64_t* const wait_bar = &stuck;
+#else
+    uint64_t* const wait_bar = &bar;
+#endif
 
     pdl_enter();
     const int b = blockIdx.x / S;
@@ -126,6 +135,7 @@ rank_hidden_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride,
         if constexpr (VEC) {
             if (tid == 0) {
                 mbar_init(&bar, 1);
+                if (wait_bar != &bar) mbar_init(wait_bar, 1);
                 fence_mbar_init();
                 mbar_arrive_expect_tx(&bar, static_cast<uint32_t>(d * sizeof(T)));
                 bulk_g2s(q_sh, qg, static_cast<uint32_t>(d * sizeof(T)), &bar);
@@ -136,7 +146,7 @@ rank_hidden_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride,
     }
     __syncthreads();               // mbarrier initialised; shared state visible
     hidden_rank_cta<T, VEC>(hb, d, t, cand_pos + static_cast<int64_t>(b) * C_cap, n, S, rank, sh.jpre,
-                            q_sh, &bar, need_query && VEC, threshold,
+                            q_sh, wait_bar, need_query && VEC, threshold,
                             scores ? scores + static_cast<int64_t>(b) * C_cap : nullptr, sh);
     if constexpr (VEC) {
         // The copy into this CTA's shared memory must have landed before exit (bounded).
@@ -334,10 +344,11 @@ rank_attention_kernel(const void* __restrict__ A, bool a_bf16, int R, int64_t ro
     store_best<CLUSTER>(sh, mine, b, best_pos, best_score, status, PLDP_ST_TIMEOUT);
 }
 
-// CTAs per sequence: 1 when the batch fills the GPU, else up to a cluster of 8
-// (never more than the candidate capacity).
-int pick_split(int B, int C_cap) {
-    int s = sm_count() / (B > 0 ? B : 1);
+// CTAs per sequence: as many as the kernel's resident CTA slots allow for the
+// batch (all of its CTAs in one wave), up to a cluster of 8, never more than the
+// candidate capacity.  `kernel` is the variant launched when S > 1.
+int pick_split(int B, int C_cap, const void* kernel, size_t smem) {
+    int s = resident_blocks(kernel, kThreads, smem) / (B > 0 ? B : 1);
     if (s > C_cap) s = C_cap;
     return s < 1 ? 1 : (s > kMaxCluster ? kMaxCluster : s);
 }
@@ -435,8 +446,9 @@ extern "C" PLDP_API pldp_status pldp_rank_hidden_avg(const void* H, pldp_dtype d
         return fail(PLDP_ERR_INVALID_ARG, "rank_hidden_avg: null pointer");
 
     const bool vec = aligned16(H) && (d * es) % 16 == 0 && (seq_stride * es) % 16 == 0;
-    const int S = pick_split(B, C_cap);
     const size_t smem = (static_cast<size_t>(d) * sizeof(float) + 127) / 128 * 128;
+    const int S = pick_split(B, C_cap, reinterpret_cast<const void*>(&rank_hidden_avg_kernel<__nv_bfloat16, true, true>),
+                             smem);
     cudaError_t e;
     if (dtype == PLDP_BF16) {
         const __nv_bfloat16* h = static_cast<const __nv_bfloat16*>(H);
@@ -480,8 +492,9 @@ extern "C" PLDP_API pldp_status pldp_rank_hidden(const void* H, pldp_dtype dtype
         return fail(PLDP_ERR_INVALID_ARG, "rank_hidden: null pointer");
 
     const bool vec = aligned16(H) && (d * es) % 16 == 0 && (seq_stride * es) % 16 == 0;
-    const int S = pick_split(B, C_cap);
     const size_t smem = (static_cast<size_t>(d) * es + 127) / 128 * 128;
+    const int S = pick_split(B, C_cap, reinterpret_cast<const void*>(&rank_hidden_kernel<__nv_bfloat16, true, true>),
+                             smem);
     cudaError_t e;
     if (dtype == PLDP_BF16) {
         const __nv_bfloat16* h = static_cast<const __nv_bfloat16*>(H);
@@ -532,8 +545,8 @@ extern "C" PLDP_API pldp_status pldp_rank_attention(const void* A, pldp_dtype dt
     if (!A || !seq_len || !cand_count || !best_pos || (C_cap > 0 && !cand_pos))
         return fail(PLDP_ERR_INVALID_ARG, "rank_attention: null pointer");
 
-    const int S = pick_split(B, C_cap);
     const size_t smem = static_cast<size_t>(sel) * sizeof(int64_t);
+    const int S = pick_split(B, C_cap, reinterpret_cast<const void*>(&rank_attention_kernel<true>), smem);
     cudaError_t e;
     e = launch_attention(B, S, smem, stream, A, dtype == PLDP_BF16, R, row_stride, seq_stride, row_idx,
                          sel, static_cast<int>(agg), seq_len, T_cap, cand_pos, cand_count, C_cap,

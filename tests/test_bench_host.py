@@ -59,6 +59,7 @@ def test_reference_arm_line_has_the_contract_keys(monkeypatch):
     assert out["impl"] == "reference" and out["unit"] == "steps/s" and out["value"] > 0
     assert out["steps"] == 3 and out["warmup"] == 3 and out["metric"] == bench.METRIC
     assert out["config"]["workload"] == bench.workload_name(small)
+    assert out["config"] == bench.bench_config(small, bench.parse(), 1)       # the same dict as our arm's
     cb = out["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] == 1 and cb["value"] == out["value"] and "sample" in cb
     e = out["e2e"]

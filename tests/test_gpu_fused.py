@@ -17,13 +17,16 @@ def i32(x):
     return torch.as_tensor(np.asarray(x, np.int32), device=DEV)
 
 
-def _compare(g, ids0, L0, H, A, row_idx, agg, ngram, C, K, draft_from, thr=float("-inf")):
+def _compare(g, ids0, L0, H, A, row_idx, agg, ngram, C, K, draft_from, thr=float("-inf"), status0=None):
+    """The drafting outputs in g against the oracle on the state (ids0, L0); status0
+    (the oracle's bits of an earlier part of the same call) is OR-ed into the status
+    expected."""
     o_cand, o_cnt, o_ml, o_st = oracle.find_candidates(ids0, L0, ngram[0], ngram[1], C)
     assert np.array_equal(g["cnt"], o_cnt) and np.array_equal(g["ml"], o_ml)
     for b in range(len(L0)):
         n = min(o_cnt[b], C)
         assert np.array_equal(g["cand"][b, :n], o_cand[b, :n]), b
-    st = o_st.copy()
+    st = o_st.copy() if status0 is None else o_st | status0
     valid = np.array([0 <= l <= ids0.shape[1] for l in L0])
     if H is not None:
         o_s, o_b, _ = oracle.rank_hidden(host(H), L0, o_cand, o_cnt, threshold=thr, status=st)

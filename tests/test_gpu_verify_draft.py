@@ -1,7 +1,9 @@
 """pldp_verify_greedy_draft (verification of a step, then the next step's drafting
 with the token index, in one call) against pldp_verify_greedy followed by
 pldp_draft_step on the same state: every output, the extended contexts and the
-index must agree bit for bit, step after step.  Covers random contexts (few and
+index must agree bit for bit, step after step, and every output equals the
+oracle's (verification on the pre-step state, then the next draft on the state
+it leaves).  Covers random contexts (few and
 many occurrences, the rescan fallback), a context that runs out of capacity, an
 out-of-range length, an out-of-range draft length, the draft buffers shared
 between the two halves or not, and a sustained decode loop."""
@@ -9,9 +11,11 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2412_01447_gb300 as pk
 import workloads as wl
 from tests._parity import Buffers, host, snapshot
+from tests.test_gpu_fused import _compare
 
 pytestmark = pytest.mark.gpu
 DEV = "cuda"
@@ -83,6 +87,18 @@ def _same_index(x, y, B, V):
     assert torch.equal(sx, sy)
 
 
+def _oracle_step(g, pre, ids, L, H, A, ngram, C, K, draft_from):
+    """The fused call's outputs g against the oracle: greedy verification of the
+    pre-step draft on the pre-step state, then the next draft on the state that
+    verification leaves (every status bit of both halves)."""
+    ids_o, L_o = pre["ids"].copy(), pre["L"].copy()
+    o = oracle.verify_greedy(pre["logits"], pre["draft"], pre["dlen"], ids=ids_o, seq_len=L_o, kv_keep=True)
+    for k_g, k_o in (("argmax", "argmax"), ("acc", "accept_len"), ("nxt", "next_token"), ("kv", "kv_keep_len")):
+        assert np.array_equal(g[k_g], o[k_o]), k_g
+    assert np.array_equal(host(ids), ids_o) and np.array_equal(host(L), L_o)
+    _compare(g, ids_o, L_o, H, A, None, 0, ngram, C, K, draft_from, status0=o["status"])
+
+
 def _planted_logits(draft, dlen, V, gen, accept):
     """bf16 logits [B, K+1, V]: N(0,1), with row i's maximum moved onto draft[b, i] for
     i < accept[b] (the step accepts min(accept, draft_len) tokens, fewer where a draft
@@ -136,19 +152,25 @@ def _verify_draft_case(T, V, B, mode, shared, K, C, ngram, dt):
     a, b_ = Buffers(B, K, V, C, DEV), Buffers(B, K, V, C, DEV)
     _draft(a, ids_a, L_a, ix_a, V, H, A, ngram, draft_from)
     _draft(b_, ids_b, L_b, ix_b, V, H, A, ngram, draft_from)
+    st = np.zeros(B, np.uint32)
     for step in range(6):
         accept = torch.as_tensor(rng.integers(0, K + 1, size=B), device=DEV)
         if step == 2:
             a.dlen[2] = K + 3                 # an out-of-range draft length (DRAFT_LEN, clamped)
             b_.dlen[2] = K + 3
         logits = _planted_logits(a.draft, a.dlen, V, gen, accept)
+        pre = dict(ids=host(ids_b), L=host(L_b), logits=host(logits), draft=host(b_.draft), dlen=host(b_.dlen))
+        a.status.zero_()
+        b_.status.zero_()
         _separate(a, logits, ids_a, L_a, ix_a, V, H, A, ngram, draft_from)
         _fused(b_, logits, ids_b, L_b, ix_b, V, H, A, ngram, draft_from, shared=shared)
         torch.cuda.synchronize()
-        _same(_snap(a), _snap(b_), step)
+        g = _snap(b_)
+        _same(_snap(a), g, step)
         assert torch.equal(ids_a, ids_b) and torch.equal(L_a, L_b), step
         _same_index(ix_a, ix_b, B, V)
-    st = host(b_.status).view(np.uint32)
+        _oracle_step(g, pre, ids_b, L_b, H, A, ngram, C, K, draft_from)
+        st |= g["status"].view(np.uint32)
     assert st[0] & pk.PLDP_ST_CAPACITY and st[1] & pk.PLDP_ST_SEQ_LEN and st[2] & pk.PLDP_ST_DRAFT_LEN
     assert st[4] & pk.PLDP_ST_SEQ_LEN and host(L_b)[4] == 0 and host(L_b)[3] > 1
     for ix in (ix_a, ix_b):                   # the empty context's index stays usable (nothing indexed)
@@ -173,15 +195,21 @@ def test_verify_draft_decode_loop(lib):
     loop.step_inputs(0)
     _draft(a, loop.ids, loop.seq_len, ix_a, w.V, loop.H, loop.A, (w.ngram_min, w.ngram_max), "hidden")
     _draft(b_, ids_b, L_b, ix_b, w.V, loop.H, loop.A, (w.ngram_min, w.ngram_max), "hidden")
+    ng = (w.ngram_min, w.ngram_max)
     for s in range(steps):
         loop.step_inputs(s)                   # logits for this step (and attention rows, shared by both)
-        _separate(a, loop.logits, loop.ids, loop.seq_len, ix_a, w.V, loop.H, loop.A, (w.ngram_min, w.ngram_max),
-                  "hidden")
-        _fused(b_, loop.logits, ids_b, L_b, ix_b, w.V, loop.H, loop.A, (w.ngram_min, w.ngram_max), "hidden")
+        pre = dict(ids=host(ids_b), L=host(L_b), logits=host(loop.logits), draft=host(b_.draft),
+                   dlen=host(b_.dlen))
+        a.status.zero_()
+        b_.status.zero_()
+        _separate(a, loop.logits, loop.ids, loop.seq_len, ix_a, w.V, loop.H, loop.A, ng, "hidden")
+        _fused(b_, loop.logits, ids_b, L_b, ix_b, w.V, loop.H, loop.A, ng, "hidden")
         torch.cuda.synchronize()
-        _same(_snap(a), _snap(b_), s)
+        g = _snap(b_)
+        _same(_snap(a), g, s)
         assert torch.equal(loop.ids, ids_b) and torch.equal(loop.seq_len, L_b)
         _same_index(ix_a, ix_b, B, w.V)
+        _oracle_step(g, pre, ids_b, L_b, loop.H, loop.A, ng, C, K, "hidden")
     L = host(L_b)
     ids, gt = host(ids_b), loop.gt_host
     for b in range(B):
