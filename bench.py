@@ -531,6 +531,8 @@ def run_ours(args, ws_, rank, local):
     if not args.no_sample:
         out["rank_stress"] = time_rank_stress(pk, loop, w, flush_l2, peak)
         out["sampling_verify"] = time_sampling_verify(pk, loop, w, flush_l2, peak)
+        if path.vd:
+            out["sampling_verify_draft"] = time_sample_draft_loop(pk, loop, path, w, flush_l2, peak)
         out["rank_hidden_avg"] = time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak)
         out["identify_heads"] = time_identify_heads(pk, loop, w, flush_l2, peak)
     if not args.no_configs:
@@ -613,6 +615,49 @@ def time_sampling_verify(pk, loop, w, flush_l2, peak, calls=64, warm=4, temperat
             "frac": round(by / (us * 1e-6) / 1e9 / peak, 4), "algorithmic_bytes": by,
             "launches_per_call": 2,
             "timing": "CUDA events around each pldp_verify_sample call, L2 flushed before each"}
+
+
+def time_sample_draft_loop(pk, loop, path, w, flush_l2, peak, steps=64, warm=3, temperature=1.0):
+    """Sampling verification at T = 1 followed by the next draft, one
+    pldp_verify_sample_draft call per step, on the same loop from its initial state
+    (index and first draft as in the timed loop): per-call CUDA events, L2 flushed
+    before each step.  The attention rows each step's drafting ranks with are those
+    of the step's own state (step_inputs): the acceptance of sampling is not known
+    to the input generator."""
+    dev = loop.device
+    B, K1 = w.B, w.K + 1
+    loop.reset()
+    path.build_index()
+    path.prime(0)
+    gen = torch.Generator(device=dev).manual_seed(w.seed + 29)
+    ws = torch.empty(pk.pldp_verify_sample_draft_workspace_size(B, w.K, w.V, loop.logits.dtype), dtype=torch.uint8,
+                     device=dev)
+    u = torch.empty((B, K1), dtype=torch.float32, device=dev)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    s = torch.cuda.current_stream()
+    acc = torch.zeros((), dtype=torch.int64, device=dev)
+    for i in range(warm + steps):
+        loop.step_inputs(i)
+        u.uniform_(generator=gen)
+        flush_l2(i)
+        if i >= warm:
+            ev[i - warm][0].record(s)
+        pk.pldp_verify_sample_draft(loop.logits, u, path.draft, path.dlen, path.acc, path.nxt, ws, loop.ids,
+                                    loop.seq_len, w.ngram_min, w.ngram_max, path.cand, path.cnt, path.ml, path.draft,
+                                    path.dlen, path.index, temperature=temperature, kv_keep_len=path.kv, H=loop.H,
+                                    best_h=path.best_h, A=loop.A, best_a=path.best_a, draft_from="hidden",
+                                    status=path.status)
+        if i >= warm:
+            ev[i - warm][1].record(s)
+            acc += path.acc.sum()
+    torch.cuda.synchronize()
+    us = np.array([a.elapsed_time(b) for a, b in ev]) * 1e3
+    by = 2.0 * B * K1 * w.V
+    return {"temperature": temperature, "steps": steps, "us_per_step": round(float(us.mean()), 2),
+            "us_p50_p90": [round(float(np.percentile(us, 50)), 2), round(float(np.percentile(us, 90)), 2)],
+            "logits_bytes": by, "logits_gbs": round(by / (us.mean() * 1e-6) / 1e9, 1),
+            "mean_accept": round(float(acc) / (steps * B), 3), "launches_per_step": 3,
+            "timing": "CUDA events around each pldp_verify_sample_draft call, L2 flushed before each step"}
 
 
 def time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak, m=4, calls=64, warm=4):
@@ -845,15 +890,19 @@ def path_draft(loop, w):
 
 def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     """The same loop through the public API with host buffers: each step copies its
-    inputs (logits, attention rows, the hidden rows of the positions the step's forward
-    pass produced) from pinned host memory and reads back its results."""
+    logits and the hidden rows of the positions the step's forward pass produced from
+    pinned host memory, and reads back its results.  The attention rows stay in pinned
+    host memory and the drafting reads them in place (the API takes host-resident
+    attention rows): only the selected rows' values at the candidate keys cross the
+    link, counted here as one 32-byte sector each."""
     w, dev = loop.w, loop.device
     loop.reset()
     path.build_index()                  # the contexts were cut back: index them again
     path.prime(0)
     B, K1 = w.B, w.K + 1
+    A_dev = loop.A
     h_logits = torch.empty(loop.logits.shape, dtype=loop.logits.dtype, pin_memory=True)
-    h_A = torch.empty(loop.A.shape, dtype=loop.A.dtype, pin_memory=True)
+    h_A = torch.empty(A_dev.shape, dtype=A_dev.dtype, pin_memory=True)
     h_H = torch.empty((B, K1, w.d), dtype=loop.H.dtype, pin_memory=True)
     d_H = torch.empty((B, K1, w.d), dtype=loop.H.dtype, device=dev)
     res = torch.empty((B, 3 + w.K), dtype=torch.int32, device=dev)
@@ -861,34 +910,42 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     ar = torch.arange(K1, device=dev)
     bi = torch.arange(B, device=dev)[:, None]
     times = []
+    sectors = 0.0
     steps = K_steps
-    for s in range(W_steps + steps):
-        path.inputs(s)                            # make this step's inputs ...
-        pos = (loop.seq_len.long()[:, None] - 1 + ar[None]).clamp(max=loop.T_cap - 1)
-        h_logits.copy_(loop.logits)               # ... and park them in pinned host memory
-        h_A.copy_(loop.A)
-        h_H.copy_(loop.H[bi, pos])
-        torch.cuda.synchronize()
-        t0 = time.perf_counter()
-        loop.logits.copy_(h_logits, non_blocking=True)
-        loop.A.copy_(h_A, non_blocking=True)
-        d_H.copy_(h_H, non_blocking=True)
-        loop.H[bi, pos] = d_H
-        path.run()
-        res[:, 0], res[:, 1], res[:, 2] = path.acc, path.nxt, loop.seq_len
-        res[:, 3:] = path.draft
-        h_res.copy_(res, non_blocking=True)
-        torch.cuda.synchronize()
-        if s >= W_steps:
-            times.append(time.perf_counter() - t0)
+    try:
+        for s in range(W_steps + steps):
+            loop.A = A_dev
+            path.inputs(s)                            # make this step's inputs ...
+            pos = (loop.seq_len.long()[:, None] - 1 + ar[None]).clamp(max=loop.T_cap - 1)
+            h_logits.copy_(loop.logits)               # ... and park them in pinned host memory
+            h_A.copy_(A_dev)
+            h_H.copy_(loop.H[bi, pos])
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            loop.logits.copy_(h_logits, non_blocking=True)
+            d_H.copy_(h_H, non_blocking=True)
+            loop.H[bi, pos] = d_H
+            loop.A = h_A                              # read in place by the drafting
+            path.run()
+            res[:, 0], res[:, 1], res[:, 2] = path.acc, path.nxt, loop.seq_len
+            res[:, 3:] = path.draft
+            h_res.copy_(res, non_blocking=True)
+            torch.cuda.synchronize()
+            if s >= W_steps:
+                times.append(time.perf_counter() - t0)
+                sectors += float(path.cnt.clamp(0, w.C_cap).sum()) * w.R * 32.0
+    finally:
+        loop.A = A_dev
     tot = max_over_ranks(sum(times), ws_)
-    h2d = (h_logits.numel() * h_logits.element_size() + h_A.numel() * h_A.element_size()
-           + h_H.numel() * h_H.element_size())
+    h2d = (h_logits.numel() * h_logits.element_size() + h_H.numel() * h_H.element_size()
+           + sectors / steps)
     return {"value": round(ws_ * steps / tot, 2), "unit": "steps/s",
             "ms_per_step": round(tot / steps * 1e3, 3),
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(h_res.numel() * 4),
-            "timing": "host wall clock per step: H2D of inputs from pinned memory, the step's C-ABI "
-                      "calls, D2H of accept/next/seq_len/draft, synchronize"}
+            "attention_rows": "in pinned host memory, read in place by the drafting (32-byte sectors at the "
+                              "candidate keys counted in h2d_bytes_per_step)",
+            "timing": "host wall clock per step: H2D of logits and new hidden rows from pinned memory, the "
+                      "step's C-ABI calls, D2H of accept/next/seq_len/draft, synchronize"}
 
 
 def _finite(x):

@@ -20,12 +20,15 @@
  *
  * Fused forms: pldp_draft_step runs 1-3 in one launch (scanning the contexts, or
  * with the incremental token index of pldp_index_build); pldp_verify_greedy_draft
- * runs 4 for the current step and then 1-3 for the next step.  Offline:
+ * and pldp_verify_sample_draft run 4 (greedy or by sampling) for the current step
+ * and then 1-3 for the next step.  Offline:
  * pldp_rank_hidden_avg (App. B.2) and pldp_identify_heads / pldp_top_heads
  * (Sec. 4.2.1).
  *
  * Conventions shared by every call
- *  - Every pointer argument is a DEVICE pointer owned by the caller; the
+ *  - Every pointer argument is a DEVICE pointer owned by the caller (the
+ *    attention rows A of the ranking calls may also be device-addressable
+ *    page-locked host memory, read in place); the
  *    library allocates nothing and keeps no state between calls, except the
  *    caller-provided verification workspace described at pldp_verify_greedy,
  *    the caller-provided token index that the indexed drafting calls keep up
@@ -172,7 +175,11 @@ PLDP_API pldp_status pldp_rank_hidden_avg(const void* H, pldp_dtype dtype, int64
  * induction head at query t-1 attends to is the token it copies).
  *
  *  A          dtype; for sequence b and row r the attention probabilities of
- *             query t-1 over keys: A + b*seq_stride + r*row_stride + key.
+ *             query t-1 over keys: A + b*seq_stride + r*row_stride + key.  A may
+ *             also be page-locked host memory that device code can address (a
+ *             cudaHostAlloc allocation under unified addressing): the kernels read
+ *             only the selected rows' values at the candidate keys, so rows kept
+ *             on the host need not be copied to the device whole.
  *  R          rows per sequence (>= 1); row_stride >= T_cap; seq_stride >=
  *             R * row_stride.
  *  row_idx    int32 [n_sel] device, or NULL for all R rows: the selected
@@ -231,7 +238,8 @@ PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
  *  H .. best_h_score     as pldp_rank_hidden (H = NULL skips hidden ranking;
  *                        H rows must be 16-byte aligned).  h_scores and
  *                        best_h_score may be NULL.
- *  A .. best_a_score     as pldp_rank_attention (A = NULL skips it); a_scores
+ *  A .. best_a_score     as pldp_rank_attention (A = NULL skips it; A may be
+ *                        device-addressable page-locked host memory); a_scores
  *                        and best_a_score may be NULL.
  *  draft_from            0: draft after best_h, 1: after best_a (that ranking
  *                        must be given).
@@ -447,6 +455,56 @@ PLDP_API pldp_status pldp_verify_sample(const void* logits, pldp_dtype dtype, in
 
 /* Bytes of workspace pldp_verify_sample needs (0 if invalid). */
 PLDP_API size_t pldp_verify_sample_workspace_size(int B, int K, int V, pldp_dtype dtype);
+
+/*
+ * Sampling verification of the current step followed by the drafting of the
+ * next one, in one call -- pldp_verify_sample then pldp_draft_step (with the
+ * token index) on the context it has just extended, with the same results and
+ * status bits as those two calls in turn.  Sec. 4.4 at temperature T > 0 (the
+ * paper's sampled runs use T = 1, Table 2), then Eq. 1-3 and Sec. 4.3; the paper
+ * has no fused form.  Three launches: the per-piece stats pass over the logits,
+ * one warp per row that draws, then one CTA per sequence that accepts, appends
+ * and drafts the next step.
+ *
+ *  logits, dtype, V   this step's logits [B, K+1, V], as pldp_verify_sample.
+ *  temperature        T > 0, finite (else PLDP_ERR_INVALID_ARG).
+ *  uniforms           float [B, K+1], as pldp_verify_sample (clamped into [0, 1)).
+ *  draft, draft_len   this step's draft [B, K] and lengths [B]; they may be the
+ *                     same buffers as next.draft and next.draft_len.
+ *  sampled            int32 [B, K+1] out or NULL: every draw y_i.
+ *  accept_len, next_token, kv_keep_len   as pldp_verify_greedy.
+ *  workspace          device scratch of pldp_verify_sample_draft_workspace_size(
+ *                     B, K, V, dtype) bytes, 16-byte aligned (no zeroing needed).
+ *                     Calls that may run concurrently need separate workspaces.
+ *  next               the next step's pldp_draft_step arguments, as for
+ *                     pldp_verify_greedy_draft (next.index required, next.V == V,
+ *                     next.B and next.K are the verification's B and K, next.ids /
+ *                     next.seq_len are appended to, next.status receives both
+ *                     calls' bits, next.workspace is not used).
+ * K + 1 <= 12288.  The draws are those of pldp_verify_sample on the same inputs.
+ */
+typedef struct pldp_verify_sample_draft_args {
+    const void* logits;
+    pldp_dtype dtype;
+    int V;
+    float temperature;
+    const float* uniforms;
+    const int32_t* draft;
+    const int32_t* draft_len;
+    int32_t* sampled;
+    int32_t* accept_len;
+    int32_t* next_token;
+    int32_t* kv_keep_len;
+    void* workspace;
+    size_t workspace_bytes;
+    pldp_draft_step_args next;
+} pldp_verify_sample_draft_args;
+
+/* `args` is a HOST pointer to the argument block, read before the call returns. */
+PLDP_API pldp_status pldp_verify_sample_draft(const pldp_verify_sample_draft_args* args, void* stream);
+
+/* Bytes of workspace pldp_verify_sample_draft needs (0 if invalid). */
+PLDP_API size_t pldp_verify_sample_draft_workspace_size(int B, int K, int V, pldp_dtype dtype);
 
 /*
  * Greedy verification without a caller workspace.  The paper has no counterpart:

@@ -15,8 +15,9 @@ PLD+ (arXiv 2412.01447), per decode step and per sequence:
   * ``pldp_verify_greedy``   -- Sec. 4.4: greedy accept against the target argmax;
   * ``pldp_verify_sample``   -- Sec. 4.4 with sampling, from caller uniforms.
 The fused calls: ``pldp_draft_step`` (the first four in one launch, optionally
-with the token index of ``pldp_index_build``) and ``pldp_verify_greedy_draft``
-(verification, then the next step's draft).  Also ``pldp_rank_hidden_avg``
+with the token index of ``pldp_index_build``), ``pldp_verify_greedy_draft`` and
+``pldp_verify_sample_draft`` (verification, greedy or by sampling, then the next
+step's draft).  Also ``pldp_rank_hidden_avg``
 (App. B.2) and ``pldp_identify_heads`` / ``pldp_top_heads`` (Sec. 4.2.1).
 
 Device buffers are passed as raw pointers, so the binding checks what the C
@@ -45,6 +46,7 @@ __all__ = [
     "pldp_draft_step", "pldp_draft_step_args", "pldp_draft_workspace_size",
     "pldp_index_size", "pldp_index_build",
     "pldp_verify_greedy_draft", "pldp_verify_draft_args",
+    "pldp_verify_sample_draft", "pldp_verify_sample_draft_args", "pldp_verify_sample_draft_workspace_size",
     "pldp_rank_hidden_avg", "pldp_identify_heads", "pldp_top_heads",
     "pldp_version", "pldp_last_error",
 ]
@@ -97,6 +99,17 @@ class pldp_draft_step_args(ctypes.Structure):
         ("draft_len", ctypes.c_void_p), ("status", ctypes.c_void_p),
         ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
         ("index", ctypes.c_void_p), ("index_bytes", ctypes.c_size_t), ("V", ctypes.c_int),
+    ]
+
+
+class pldp_verify_sample_draft_args(ctypes.Structure):
+    """Mirror of the C argument block of pldp_verify_sample_draft (include/pldp.h)."""
+    _fields_ = [
+        ("logits", ctypes.c_void_p), ("dtype", ctypes.c_int), ("V", ctypes.c_int),
+        ("temperature", ctypes.c_float), ("uniforms", ctypes.c_void_p),
+        ("draft", ctypes.c_void_p), ("draft_len", ctypes.c_void_p), ("sampled", ctypes.c_void_p),
+        ("accept_len", ctypes.c_void_p), ("next_token", ctypes.c_void_p), ("kv_keep_len", ctypes.c_void_p),
+        ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t), ("next", pldp_draft_step_args),
     ]
 
 
@@ -153,6 +166,10 @@ def _load():
             lib.pldp_draft_step.restype = ctypes.c_int
             lib.pldp_verify_greedy_draft.argtypes = [ctypes.POINTER(pldp_verify_draft_args), P]
             lib.pldp_verify_greedy_draft.restype = ctypes.c_int
+            lib.pldp_verify_sample_draft.argtypes = [ctypes.POINTER(pldp_verify_sample_draft_args), P]
+            lib.pldp_verify_sample_draft.restype = ctypes.c_int
+            lib.pldp_verify_sample_draft_workspace_size.argtypes = [i32, i32, i32, i32]
+            lib.pldp_verify_sample_draft_workspace_size.restype = sz
             lib.pldp_draft_workspace_size.argtypes = [i32]
             lib.pldp_draft_workspace_size.restype = sz
             lib.pldp_index_size.argtypes = [i32, i32]
@@ -201,6 +218,14 @@ def _dev(t, name, dtype=None, allow_none=False):
 
 
 _WORD = (torch.int32, getattr(torch, "uint32", torch.int32))
+
+
+def _dev_or_pinned(t, name):
+    """A CUDA tensor, or a page-locked (pinned) host tensor, which the device reads in
+    place through unified addressing."""
+    if isinstance(t, torch.Tensor) and not t.is_cuda and t.is_pinned():
+        return ctypes.c_void_p(t.data_ptr())
+    return _dev(t, name)
 
 
 def _dense(t, name, dtype=None, allow_none=False, n=None):
@@ -328,14 +353,16 @@ def pldp_top_heads(counts, k, row_idx, stream=None):
 def pldp_rank_attention(A, seq_len, cand_pos, cand_count, best_pos, row_idx=None, agg=PLDP_AGG_MAX,
                         scores=None, best_score=None, status=None, stream=None):
     """Eq. 2.  A: [B, R, T_cap] float32/bfloat16, attention of query t-1 for each of R
-    (layer, head) rows (unit inner stride); row_idx int32 [n_sel] device or None (all)."""
+    (layer, head) rows (unit inner stride), on the device or in pinned host memory (read
+    in place: only the selected rows' values at the candidate keys cross the link);
+    row_idx int32 [n_sel] device or None (all)."""
     if A.dim() != 3 or A.stride(2) != 1:
         raise ValueError("A must be [B, R, T_cap] with unit inner stride")
     B, R, T_cap = A.shape
     C_cap = cand_pos.shape[1]
     n_sel = R if row_idx is None else row_idx.numel()
     _check("pldp_rank_attention", _load().pldp_rank_attention(
-        _dev(A, "A"), _code(A.dtype), R, A.stride(1), A.stride(0),
+        _dev_or_pinned(A, "A"), _code(A.dtype), R, A.stride(1), A.stride(0),
         _dense(row_idx, "row_idx", torch.int32, allow_none=True), n_sel, int(agg),
         _dense(seq_len, "seq_len", torch.int32, n=B), B, T_cap, _dense(cand_pos, "cand_pos", torch.int32, n=B * C_cap),
         _dense(cand_count, "cand_count", torch.int32, n=B), C_cap,
@@ -390,7 +417,7 @@ def _draft_args(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_
             raise ValueError("A must be [B, R, T_cap] with unit inner stride")
         if A.shape[0] < B or A.shape[2] < T:
             raise ValueError(f"A must cover [B, T_cap] = [{B}, {T}] positions")
-        a.A, a.a_dtype, a.R = _dev(A, "A"), _code(A.dtype), A.shape[1]
+        a.A, a.a_dtype, a.R = _dev_or_pinned(A, "A"), _code(A.dtype), A.shape[1]
         a.a_row_stride, a.a_seq_stride = A.stride(1), A.stride(0)
         a.row_idx = _dense(row_idx, "row_idx", torch.int32, allow_none=True)
         a.n_sel = A.shape[1] if row_idx is None else row_idx.numel()
@@ -457,6 +484,44 @@ def pldp_verify_greedy_draft(logits, draft, draft_len, accept_len, next_token, w
     a.workspace = _dense(workspace, "workspace")
     a.workspace_bytes = workspace.numel() * workspace.element_size()
     _check("pldp_verify_greedy_draft", _load().pldp_verify_greedy_draft(ctypes.byref(a), _stream(stream)))
+
+
+def pldp_verify_sample_draft_workspace_size(B, K, V, dtype=torch.bfloat16) -> int:
+    return int(_load().pldp_verify_sample_draft_workspace_size(B, K, V, _code(dtype)))
+
+
+def pldp_verify_sample_draft(logits, uniforms, draft, draft_len, accept_len, next_token, workspace, ids, seq_len,
+                             ngram_min, ngram_max, cand_pos, cand_count, match_len, next_draft, next_draft_len,
+                             index, temperature=1.0, sampled=None, kv_keep_len=None, stream=None, **kw):
+    """Sampling verification of this step (as pldp_verify_sample at ``temperature``
+    with ``uniforms`` [B, K+1], appending to ids and seq_len) followed by the next
+    step's drafting with the token index (as pldp_draft_step on the extended
+    context), in one call.  workspace: uint8 CUDA tensor of
+    pldp_verify_sample_draft_workspace_size(B, K, V, dtype) bytes.  Other arguments
+    as pldp_verify_greedy_draft."""
+    B, K1, V = logits.shape
+    K = K1 - 1
+    if draft.shape != (B, K) or next_draft.shape != (B, K):
+        raise ValueError("draft and next_draft must be [B, K] with K = logits.shape[1] - 1")
+    if uniforms.shape != (B, K1):
+        raise ValueError("uniforms must be [B, K+1]")
+    if not isinstance(ids, torch.Tensor) or ids.dim() != 2 or ids.shape[0] != B:
+        raise ValueError("ids must be [B, T_cap] with B = logits.shape[0]")
+    a = pldp_verify_sample_draft_args()
+    a.next = _draft_args(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_len, K, next_draft,
+                         next_draft_len, None, index=index, V=V, **kw)
+    a.logits, a.dtype, a.V = _dense(logits, "logits"), _code(logits.dtype), V
+    a.temperature = float(temperature)
+    a.uniforms = _dense(uniforms, "uniforms", torch.float32, n=B * K1)
+    a.draft = _dense(draft, "draft", torch.int32, n=B * K)
+    a.draft_len = _dense(draft_len, "draft_len", torch.int32, n=B)
+    a.sampled = _dense(sampled, "sampled", torch.int32, allow_none=True, n=B * K1)
+    a.accept_len = _dense(accept_len, "accept_len", torch.int32, n=B)
+    a.next_token = _dense(next_token, "next_token", torch.int32, n=B)
+    a.kv_keep_len = _dense(kv_keep_len, "kv_keep_len", torch.int32, allow_none=True, n=B)
+    a.workspace = _dense(workspace, "workspace")
+    a.workspace_bytes = workspace.numel() * workspace.element_size()
+    _check("pldp_verify_sample_draft", _load().pldp_verify_sample_draft(ctypes.byref(a), _stream(stream)))
 
 
 def pldp_index_size(B, V) -> int:

@@ -73,3 +73,36 @@ def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
         raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")
     os.replace(tmp, LIB)
     return LIB
+
+
+def build_variant(name: str, srcs, extra_flags=(), force: bool = False) -> str:
+    """Builds a separate shared library ``_build/<name>/lib<name>.so`` from some of
+    the sources with extra compiler flags (a test build of selected kernels, e.g.
+    with a test-only macro defined).  The product library is not touched."""
+    out_dir = os.path.join(BUILD_DIR, name)
+    out = os.path.join(out_dir, f"lib{name}.so")
+    paths = [os.path.join(CSRC, x) for x in srcs]
+    deps = paths + glob.glob(os.path.join(CSRC, "*.cuh")) + glob.glob(os.path.join(INCLUDE, "*.h")) + [
+        os.path.abspath(__file__)]
+    if not force and os.path.exists(out) and all(os.path.getmtime(p) <= os.path.getmtime(out) for p in deps):
+        return out
+    os.makedirs(out_dir, exist_ok=True)
+    cc = nvcc()
+
+    def compile_one(src):
+        obj = os.path.join(out_dir, os.path.basename(src)[:-3] + ".o")
+        r = subprocess.run([cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", src, "-o", obj], capture_output=True,
+                           text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed on {os.path.basename(src)}:\n{r.stdout}\n{r.stderr}")
+        return obj
+
+    with cf.ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 1)) as ex:
+        objs = list(ex.map(compile_one, paths))
+    tmp = out + f".tmp{os.getpid()}"
+    r = subprocess.run([cc, *ARCH, "-shared", "-Xcompiler", "-fPIC", "-o", tmp, *objs], capture_output=True,
+                       text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, out)
+    return out

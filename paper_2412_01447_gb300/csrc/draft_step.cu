@@ -1,13 +1,14 @@
 // pldp_draft_step: the drafting half of a PLD+ step -- candidate search (Eq. 1
 // with the longest-suffix n-gram rule), ranking by hidden states (Eq. 3) and/or
 // by attentions (Eq. 2), and draft extraction (Sec. 4.3) -- in one launch; and
-// pldp_verify_greedy_draft: greedy verification (Sec. 4.4) followed by the next
-// step's drafting.  Three kernels:
+// pldp_verify_greedy_draft / pldp_verify_sample_draft: greedy or sampling
+// verification (Sec. 4.4) followed by the next step's drafting.  Three kernels:
 //  * draft_step_kernel scans the contexts (below);
 //  * draft_index_kernel looks the occurrences up in the incremental token index
 //    (further down), one CTA per sequence;
-//  * verify_draft_kernel runs the finish of greedy verification and then the
-//    indexed drafting in the same CTA.
+//  * verify_draft_kernel runs the finish of verification (on the greedy pass's
+//    row keys, or on the draws of sampling) and then the indexed drafting in the
+//    same CTA.
 //
 // The scanning kernel: a flat grid of (chunk, sequence) CTAs.  Each CTA
 //  1. streams its chunk of the context with 16-byte loads and, for every
@@ -1018,7 +1019,8 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
 // Verification of the current step -- the finish of greedy verification: the
 // accepted length, the bonus token and the append (Sec. 4.4) -- and then, in the
 // same CTA, the next step's drafting with the token index.  One CTA per
-// sequence, launched behind the verification's argmax pass.  The draft step
+// sequence, launched behind the verification's argmax pass (greedy: the targets
+// are the row keys) or behind the draws of sampling verification (va.row_draws).  The draft step
 // starts from the context the finish has just written: its length is known
 // without a read, and the appended ids are read through L2.
 template <typename TH, bool IVEC>
@@ -1033,8 +1035,9 @@ __global__ void __launch_bounds__(kThreads, 1) verify_draft_kernel(const VerifyA
     if (threadIdx.x < 32) {
         const int lane = static_cast<int>(threadIdx.x);
         FinishOut fo;
-        const int64_t L1 = finish_sequence(va, b, lane, KeyTokens{va.row_keys + static_cast<int64_t>(b) * (va.K + 1)},
-                                           &fo);
+        const int64_t r0 = static_cast<int64_t>(b) * (va.K + 1);
+        const RowTokens src{va.row_draws ? nullptr : va.row_keys + r0, va.row_draws ? va.row_draws + r0 : nullptr};
+        const int64_t L1 = finish_sequence(va, b, lane, src, &fo);
         if (lane == 0) L_after = L1;
         // The drafting's first reads come from what the finish holds: the ids appended
         // since the index was brought up to date (il .. t-1) and the suffix x_t, x_{t-1},
@@ -1251,7 +1254,7 @@ pldp_status launch_verify_draft_t(const VerifyArgs& va, const DraftParams& p, co
                                   cudaStream_t s) {
     const cudaError_t e = launch_pdl(verify_draft_kernel<TH, IVEC>, dim3(static_cast<unsigned>(B)), dim3(kThreads), 0,
                                      s, 0, va, p, ix);
-    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "verify_greedy_draft: launch failed: %s", cudaGetErrorString(e));
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "verify_draft: launch failed: %s", cudaGetErrorString(e));
     return PLDP_OK;
 }
 
@@ -1311,6 +1314,47 @@ extern "C" PLDP_API pldp_status pldp_verify_greedy_draft(const pldp_verify_draft
                                 a->kv_keep_len, n.status);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const pldp_status sp = launch_verify_pass(a->logits, a->dtype, va, a->workspace, s, "verify_greedy_draft");
+    if (sp != PLDP_OK) return sp;
+    if (!n.H) return launch_verify_draft<NoHidden>(va, p, ixv, B, ivec, s);
+    if (n.h_dtype == PLDP_BF16) return launch_verify_draft<__nv_bfloat16>(va, p, ixv, B, ivec, s);
+    return launch_verify_draft<float>(va, p, ixv, B, ivec, s);
+}
+
+extern "C" PLDP_API size_t pldp_verify_sample_draft_workspace_size(int B, int K, int V, pldp_dtype dtype) {
+    return sample_draft_workspace_size(B, K, V, dtype);
+}
+
+extern "C" PLDP_API pldp_status pldp_verify_sample_draft(const pldp_verify_sample_draft_args* a, void* stream) {
+    if (!a) return fail(PLDP_ERR_INVALID_ARG, "verify_sample_draft: null argument block");
+    const pldp_draft_step_args& n = a->next;
+    if (!n.index) return fail(PLDP_ERR_INVALID_ARG, "verify_sample_draft: the next draft needs a token index");
+    if (a->V < 1) return fail(PLDP_ERR_INVALID_ARG, "verify_sample_draft: V < 1");
+    if (n.V != a->V) return fail(PLDP_ERR_INVALID_ARG, "verify_sample_draft: the index's V differs from the logits'");
+    if (a->dtype != PLDP_F32 && a->dtype != PLDP_BF16)
+        return fail(PLDP_ERR_UNSUPPORTED, "verify_sample_draft: unsupported dtype %d", (int)a->dtype);
+    if (!(a->temperature > 0.f) || isinf(a->temperature))
+        return fail(PLDP_ERR_INVALID_ARG, "verify_sample_draft: temperature must be positive and finite");
+    if (n.T_cap > INT32_MAX) return fail(PLDP_ERR_INVALID_ARG, "verify_sample_draft: bad T_cap");
+    if (n.K >= 1 && static_cast<int64_t>(n.K) + 1 > 12288)
+        return fail(PLDP_ERR_UNSUPPORTED, "verify_sample_draft: K > 12287");
+    DraftParams p;
+    IndexView ixv = {};
+    bool has_ix = false, ivec = false, empty = false;
+    const pldp_status st = prepare_draft(&n, "verify_sample_draft", p, ixv, has_ix, ivec, empty);
+    if (st != PLDP_OK || empty) return st;
+    const int B = n.B, K = n.K;
+    if (!a->logits || !a->uniforms || !a->draft || !a->draft_len || !a->accept_len || !a->next_token)
+        return fail(PLDP_ERR_INVALID_ARG, "verify_sample_draft: null pointer");
+    const size_t need = sample_draft_workspace_size(B, K, a->V, a->dtype);
+    if (!a->workspace || a->workspace_bytes < need || !aligned16(a->workspace))
+        return fail(PLDP_ERR_INVALID_ARG, "verify_sample_draft: workspace needs %zu bytes, 16-byte aligned", need);
+    // verification appends to the context the next draft reads: next.ids and next.seq_len
+    VerifyArgs va = verify_args(B, K, a->V, a->draft, a->draft_len, a->sampled, a->accept_len, a->next_token,
+                                const_cast<int32_t*>(n.ids), n.ids_stride, const_cast<int32_t*>(n.seq_len), n.T_cap,
+                                a->kv_keep_len, n.status);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const pldp_status sp = launch_sample_draws(a->logits, a->dtype, va, a->temperature, a->uniforms, a->workspace, s,
+                                               "verify_sample_draft");
     if (sp != PLDP_OK) return sp;
     if (!n.H) return launch_verify_draft<NoHidden>(va, p, ixv, B, ivec, s);
     if (n.h_dtype == PLDP_BF16) return launch_verify_draft<__nv_bfloat16>(va, p, ixv, B, ivec, s);

@@ -1,7 +1,7 @@
-// Greedy verification pieces shared by pldp_verify_greedy (verify.cu) and the
-// fused verification + next draft (draft_step.cu): the argument block, the
-// per-sequence finish (accept, bonus, append; Sec. 4.4) and the launch of the
-// streaming argmax pass.
+// Verification pieces shared by pldp_verify_greedy (verify.cu), pldp_verify_sample
+// (sample.cu) and the fused verification + next draft calls (draft_step.cu): the
+// argument block, the per-sequence finish (accept, bonus, append; Sec. 4.4), the
+// launch of the streaming argmax pass and that of the sampling draws.
 #pragma once
 
 #include "pldp_internal.cuh"
@@ -20,13 +20,14 @@ struct VerifyArgs {
     int64_t T_cap;
     int32_t* kv_keep_len;
     uint32_t* status;
-    unsigned long long* row_keys;   // [B*(K+1)], zero between calls
+    unsigned long long* row_keys;   // [B*(K+1)], zero between calls (greedy)
+    const int32_t* row_draws;       // [B*(K+1)] the draws of sampling verification, or null (greedy)
     int B, K, V;
 };
 
 // Where the finish reads the K+1 target tokens of a sequence: the greedy row keys
-// (argmax packed in the low word; the keys are returned to zero afterwards) or
-// the draws of sampling verification, staged in shared memory.
+// (argmax packed in the low word; the keys are returned to zero afterwards), the
+// draws of sampling verification staged in shared memory, or either (RowTokens).
 struct KeyTokens {
     unsigned long long* keys;   // [K+1] of this sequence
     __device__ __forceinline__ int at(int i) const { return static_cast<int>(key_index(__ldcg(keys + i))); }
@@ -38,6 +39,20 @@ struct SharedTokens {
     const int32_t* tok;          // shared memory, [K+1]
     __device__ __forceinline__ int at(int i) const { return tok[i]; }
     __device__ __forceinline__ void release(int, int) const {}
+};
+
+// Either of the two, chosen per call: the draws when they are given (written by
+// the previous kernel, read through L2), else the greedy row keys.
+struct RowTokens {
+    unsigned long long* keys;    // [K+1] of this sequence (greedy)
+    const int32_t* draws;        // [K+1] of this sequence (sampling), or null
+    __device__ __forceinline__ int at(int i) const {
+        return draws ? __ldcg(draws + i) : static_cast<int>(key_index(__ldcg(keys + i)));
+    }
+    __device__ __forceinline__ void release(int K1, int lane) const {
+        if (!draws)
+            for (int i = lane; i < K1; i += 32) keys[i] = 0ull;
+    }
 };
 
 // What the finish decided, for a caller that continues with the extended context.
@@ -128,6 +143,15 @@ VerifyArgs verify_args(int B, int K, int V, const int32_t* draft, const int32_t*
                        int32_t* argmax, int32_t* accept_len, int32_t* next_token, int32_t* ids,
                        int64_t ids_stride, int32_t* seq_len, int64_t T_cap, int32_t* kv_keep_len,
                        uint32_t* status);
+
+// Sampling verification's draws for the fused sampling + next draft call: launches
+// the stats pass and one warp per row that draws (Sec. 4.4 at temperature T, from
+// the caller's uniforms), leaving the draws in the workspace and setting
+// a.row_draws.  The workspace holds the per-piece stats, then the draws
+// (sample_draft_workspace_size bytes, 16-byte aligned, no zeroing needed).
+size_t sample_draft_workspace_size(int B, int K, int V, pldp_dtype dtype);
+pldp_status launch_sample_draws(const void* logits, pldp_dtype dtype, VerifyArgs& a, float temperature,
+                                const float* uniforms, void* workspace, cudaStream_t s, const char* what);
 
 // Launches the streaming argmax pass over logits [B, K+1, V] that leaves each
 // row's key in `scratch` (pldp_verify_workspace_size bytes, zero between calls)

@@ -359,13 +359,27 @@ __global__ void __launch_bounds__(32 * kFinishWarps, 1) sample_finish_kernel(con
     if (warp == 0) finish_sequence(a.v, b, lane, SharedTokens{draws});
 }
 
+// Draws only, for the fused sampling + next draft call: one warp per row, each
+// draw to draws[row]; the accept/bonus/append and the drafting follow in the
+// next kernel.
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads) sample_draw_kernel(const T* __restrict__ logits, SampleArgs a,
+                                                                int32_t* __restrict__ draws) {
+    pdl_enter();
+    const int64_t r = static_cast<int64_t>(blockIdx.x) * kWarps + (threadIdx.x >> 5);   // warp-uniform
+    const int64_t rows = static_cast<int64_t>(a.v.B) * (a.v.K + 1);
+    if (r >= rows) return;
+    const int y = sample_row<T, VEC>(logits, a, r, threadIdx.x & 31);
+    if ((threadIdx.x & 31) == 0) draws[r] = y;
+}
+
 int sample_pieces(int V, size_t es) {
     const int64_t P = kPieceBytes / static_cast<int64_t>(es);
     return static_cast<int>((V + P - 1) / P);
 }
 
 template <typename T, bool VEC>
-pldp_status launch_sample_t(const void* logits, SampleArgs a, cudaStream_t s) {
+pldp_status launch_stats_t(const void* logits, const SampleArgs& a, cudaStream_t s, const char* what) {
     const int64_t rows = static_cast<int64_t>(a.v.B) * (a.v.K + 1);
     const int64_t units = rows * a.npieces;
     const void* fn = reinterpret_cast<const void*>(&sample_stats_kernel<T, VEC>);
@@ -373,10 +387,30 @@ pldp_status launch_sample_t(const void* logits, SampleArgs a, cudaStream_t s) {
     const int64_t need = (units + kWarps - 1) / kWarps;
     if (blocks > need) blocks = need;
     if (blocks < 1) blocks = 1;
-    cudaError_t e = launch_pdl(sample_stats_kernel<T, VEC>, dim3(static_cast<unsigned>(blocks)), dim3(kThreads), 0,
-                               s, 0, static_cast<const T*>(logits), static_cast<int64_t>(a.v.V), rows, a.npieces,
-                               a.P, a.c, blocks * kWarps, const_cast<float2*>(a.stats));
-    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "verify_sample: launch failed: %s", cudaGetErrorString(e));
+    const cudaError_t e = launch_pdl(sample_stats_kernel<T, VEC>, dim3(static_cast<unsigned>(blocks)), dim3(kThreads),
+                                     0, s, 0, static_cast<const T*>(logits), static_cast<int64_t>(a.v.V), rows,
+                                     a.npieces, a.P, a.c, blocks * kWarps, const_cast<float2*>(a.stats));
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
+    return PLDP_OK;
+}
+
+template <typename T, bool VEC>
+pldp_status launch_draws_t(const void* logits, const SampleArgs& a, int32_t* draws, cudaStream_t s,
+                           const char* what) {
+    const pldp_status st = launch_stats_t<T, VEC>(logits, a, s, what);
+    if (st != PLDP_OK) return st;
+    const int64_t rows = static_cast<int64_t>(a.v.B) * (a.v.K + 1);
+    const cudaError_t e = launch_pdl(sample_draw_kernel<T, VEC>, dim3(static_cast<unsigned>((rows + kWarps - 1) / kWarps)),
+                                     dim3(kThreads), 0, s, 0, static_cast<const T*>(logits), a, draws);
+    if (e != cudaSuccess) return fail(PLDP_ERR_CUDA, "%s: launch failed: %s", what, cudaGetErrorString(e));
+    return PLDP_OK;
+}
+
+template <typename T, bool VEC>
+pldp_status launch_sample_t(const void* logits, SampleArgs a, cudaStream_t s) {
+    const pldp_status st = launch_stats_t<T, VEC>(logits, a, s, "verify_sample");
+    if (st != PLDP_OK) return st;
+    cudaError_t e;
     const size_t smem = static_cast<size_t>(a.v.K + 1) * sizeof(int32_t);
     if (smem > 48 * 1024) {
         e = cudaFuncSetAttribute(sample_finish_kernel<T, VEC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -391,6 +425,40 @@ pldp_status launch_sample_t(const void* logits, SampleArgs a, cudaStream_t s) {
 }
 
 }  // namespace
+}  // namespace pldp
+
+namespace pldp {
+
+size_t sample_draft_workspace_size(int B, int K, int V, pldp_dtype dtype) {
+    if (B < 0 || K < 1 || V < 1 || (dtype != PLDP_F32 && dtype != PLDP_BF16)) return 0;
+    const size_t es = dtype == PLDP_F32 ? 4 : 2;
+    const size_t rows = static_cast<size_t>(B) * (K + 1);
+    const size_t stats = (rows * sample_pieces(V, es) * sizeof(float2) + 255) / 256 * 256;
+    return stats + (rows * sizeof(int32_t) + 255) / 256 * 256;
+}
+
+pldp_status launch_sample_draws(const void* logits, pldp_dtype dtype, VerifyArgs& v, float temperature,
+                                const float* uniforms, void* workspace, cudaStream_t s, const char* what) {
+    const size_t es = dtype == PLDP_F32 ? 4 : 2;
+    const size_t rows = static_cast<size_t>(v.B) * (v.K + 1);
+    SampleArgs a = {};
+    a.v = v;
+    a.uniforms = uniforms;
+    a.stats = static_cast<const float2*>(workspace);
+    a.c = 1.4426950408889634f / temperature;                      // log2(e) / T
+    a.npieces = sample_pieces(v.V, es);
+    a.P = static_cast<int>(kPieceBytes / static_cast<int64_t>(es));
+    int32_t* draws = reinterpret_cast<int32_t*>(static_cast<char*>(workspace) +
+                                                (rows * a.npieces * sizeof(float2) + 255) / 256 * 256);
+    v.row_draws = draws;
+    const bool vec = aligned16(logits) && (static_cast<size_t>(v.V) * es) % 16 == 0;
+    if (dtype == PLDP_BF16)
+        return vec ? launch_draws_t<__nv_bfloat16, true>(logits, a, draws, s, what)
+                   : launch_draws_t<__nv_bfloat16, false>(logits, a, draws, s, what);
+    return vec ? launch_draws_t<float, true>(logits, a, draws, s, what)
+               : launch_draws_t<float, false>(logits, a, draws, s, what);
+}
+
 }  // namespace pldp
 
 using namespace pldp;

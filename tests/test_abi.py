@@ -146,13 +146,15 @@ def test_draft_step_args_layout_matches_header(tmp_path):
         assert getattr(pk.pldp_draft_step_args, n).offset == off, n
 
 
-def test_verify_draft_args_layout_matches_header(tmp_path):
-    """The Python mirror of pldp_verify_draft_args (with its nested draft block) has the
-    C layout (gcc offsetof)."""
-    names = [f for f, _ in pk.pldp_verify_draft_args._fields_]
+@pytest.mark.parametrize("struct", ["pldp_verify_draft_args", "pldp_verify_sample_draft_args"])
+def test_verify_draft_args_layout_matches_header(tmp_path, struct):
+    """The Python mirrors of the fused verification + next draft argument blocks (with
+    their nested draft block) have the C layout (gcc offsetof)."""
+    cls = getattr(pk, struct)
+    names = [f for f, _ in cls._fields_]
     src = ['#include <stdio.h>', '#include <stddef.h>', f'#include "{HEADER}"', "int main(void) {",
-           'printf("%zu\\n", sizeof(pldp_verify_draft_args));']
-    src += [f'printf("%zu\\n", offsetof(pldp_verify_draft_args, {n}));' for n in names]
+           f'printf("%zu\\n", sizeof({struct}));']
+    src += [f'printf("%zu\\n", offsetof({struct}, {n}));' for n in names]
     src += ["return 0; }"]
     c = tmp_path / "layout2.c"
     c.write_text("\n".join(src))
@@ -160,9 +162,9 @@ def test_verify_draft_args_layout_matches_header(tmp_path):
     import subprocess
     subprocess.check_call(["gcc", str(c), "-o", str(exe)])
     out = [int(x) for x in subprocess.check_output([str(exe)]).split()]
-    assert out[0] == ctypes.sizeof(pk.pldp_verify_draft_args)
+    assert out[0] == ctypes.sizeof(cls)
     for n, off in zip(names, out[1:]):
-        assert getattr(pk.pldp_verify_draft_args, n).offset == off, n
+        assert getattr(cls, n).offset == off, n
 
 
 def test_verify_draft_host_checks(so):
@@ -207,6 +209,49 @@ def test_verify_draft_host_checks(so):
     assert call(a) == pk.PLDP_ERR_INVALID_ARG and "workspace" in pk.pldp_last_error()
     a = block(); a.next.B = 0
     assert call(a) == pk.PLDP_OK
+
+
+def test_verify_sample_draft_host_checks(so):
+    """pldp_verify_sample_draft refuses, before any launch: a null block, a missing
+    index, a bad temperature, missing uniforms, the draft step's own argument errors
+    and a short workspace; B == 0 is a no-op."""
+    lib = pk._load()
+    P = ctypes.c_void_p
+
+    def block():
+        a = pk.pldp_verify_sample_draft_args()
+        n = a.next
+        n.ids, n.ids_stride, n.seq_len, n.B, n.T_cap = P(256), 64, P(256), 2, 64
+        n.ngram_min, n.ngram_max, n.cand_pos, n.C_cap = 1, 3, P(256), 8
+        n.cand_count, n.match_len = P(256), P(256)
+        n.H, n.h_dtype, n.d, n.h_seq_stride, n.threshold, n.best_h = P(256), 1, 64, 64 * 64, float("-inf"), P(256)
+        n.draft_from, n.K, n.draft, n.draft_len = 0, 4, P(256), P(256)
+        n.index, n.index_bytes, n.V = P(256), pk.pldp_index_size(2, 100), 100
+        a.logits, a.dtype, a.V, a.temperature, a.uniforms = P(256), 1, 100, 1.0, P(256)
+        a.draft, a.draft_len, a.accept_len, a.next_token = P(256), P(256), P(256), P(256)
+        a.workspace, a.workspace_bytes = P(256), pk.pldp_verify_sample_draft_workspace_size(2, 4, 100)
+        return a
+
+    def call(a):
+        return lib.pldp_verify_sample_draft(ctypes.byref(a), None)
+
+    assert lib.pldp_verify_sample_draft(None, None) == pk.PLDP_ERR_INVALID_ARG
+    a = block(); a.next.index = None
+    assert call(a) == pk.PLDP_ERR_INVALID_ARG and "index" in pk.pldp_last_error()
+    for T in (0.0, -1.0, float("inf"), float("nan")):
+        a = block(); a.temperature = T
+        assert call(a) == pk.PLDP_ERR_INVALID_ARG and "temperature" in pk.pldp_last_error()
+    a = block(); a.uniforms = None
+    assert call(a) == pk.PLDP_ERR_INVALID_ARG and "null" in pk.pldp_last_error()
+    a = block(); a.dtype = 7
+    assert call(a) == pk.PLDP_ERR_UNSUPPORTED
+    a = block(); a.next.ngram_max = 0
+    assert call(a) == pk.PLDP_ERR_INVALID_ARG and "verify_sample_draft" in pk.pldp_last_error()
+    a = block(); a.workspace_bytes = pk.pldp_verify_sample_draft_workspace_size(2, 4, 100) - 16
+    assert call(a) == pk.PLDP_ERR_INVALID_ARG and "workspace" in pk.pldp_last_error()
+    a = block(); a.next.B = 0
+    assert call(a) == pk.PLDP_OK
+    assert pk.pldp_verify_sample_draft_workspace_size(2, 4, 100) >= pk.pldp_verify_sample_workspace_size(2, 4, 100)
 
 
 def test_binding_checks_element_counts_and_shapes():
