@@ -1023,17 +1023,32 @@ __global__ void __launch_bounds__(kThreads, 1) draft_index_kernel(const DraftPar
 // are the row keys) or behind the draws of sampling verification (va.row_draws).  The draft step
 // starts from the context the finish has just written: its length is known
 // without a read, and the appended ids are read through L2.
+constexpr int kOldWin = 32;                        // old-context tokens read before the wait (a lane each)
+
 template <typename TH, bool IVEC>
 __global__ void __launch_bounds__(kThreads, 1) verify_draft_kernel(const VerifyArgs va, const DraftParams p,
                                                                     const IndexView ix) {
     __shared__ StepShared sh;
     __shared__ IndexShared is;
     __shared__ long long L_after;
-    pdl_enter();                                                  // the pass's row keys are final
+    __shared__ int32_t oldwin[kOldWin];                          // x_{Lw}, ..., x_{Lw + kOldWin - 1}
     const int b = blockIdx.x;
-    const int64_t il = ix.ilen[b];                                // does not depend on the verification
+    // Read before the wait, since the argmax pass does not write them (its
+    // predecessors, which did, completed before it started): the indexed length
+    // and the last kOldWin tokens of the context as it was before this step's
+    // append -- the drafting's appended ids and suffix reach back into them.
+    const int64_t il = ix.ilen[b];
+    const int64_t L_old = va.seq_len ? static_cast<int64_t>(va.seq_len[b]) : -1;
+    const int64_t Lw = L_old - kOldWin;
+    const int32_t* row_b = p.ids + static_cast<int64_t>(b) * p.ids_stride;
+    if (threadIdx.x < kOldWin) {
+        const int64_t q = Lw + threadIdx.x;
+        oldwin[threadIdx.x] = (L_old >= 1 && L_old <= p.T_cap && q >= 0) ? __ldcg(row_b + q) : 0;
+    }
+    pdl_enter();                                                  // the pass's row keys are final
     if (threadIdx.x < 32) {
         const int lane = static_cast<int>(threadIdx.x);
+        __syncwarp();                                             // oldwin written by this warp
         FinishOut fo;
         const int64_t r0 = static_cast<int64_t>(b) * (va.K + 1);
         const RowTokens src{va.row_draws ? nullptr : va.row_keys + r0, va.row_draws ? va.row_draws + r0 : nullptr};
@@ -1049,6 +1064,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_draft_kernel(const VerifyA
             const int32_t* dr = va.draft + static_cast<int64_t>(b) * va.K;
             auto tok = [&](int64_t q) -> int32_t {
                 if (q >= L0) return q - L0 < fo.n ? dr[q - L0] : fo.bonus;
+                if (L0 == L_old && q >= Lw) return oldwin[q - Lw];     // read before the wait
                 return __ldcg(row + q);
             };
             const bool usable = il >= 0 && il <= t;
