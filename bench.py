@@ -369,6 +369,8 @@ def bench_config(w, args, ws_):
     return {"workload": workload_name(w),
             "batch_per_gpu": w.B, "context": w.T, "vocab": w.V, "K": w.K, "d": w.d,
             "attention_rows": w.R, "C_cap": w.C_cap,
+            "attention_layout": ("key-major: the R values of a key side by side ([B, T_cap, R] in memory)"
+                                 if w.attn_layout == "key" else "head-major: each row's keys side by side"),
             "l2": ("flushed before every step: 256 MB write then 256 MB read (cold, clean L2)"
                    if args.flush == "write-read" else
                    "flushed before every step: 256 MB write (cold L2 holding dirty lines)")
@@ -702,6 +704,7 @@ def time_identify_heads(pk, loop, w, flush_l2, peak, calls=16, warm=2):
     before each; algorithmic bytes: every row over keys < t plus the ids scanned."""
     dev = loop.device
     loop.step_inputs(0)                                   # attention rows for the current lengths
+    A_rows = loop.A.contiguous()                          # identification reads whole rows: head-major
     pos = (loop.seq_len - 1).to(torch.int32)
     R = w.R
     counts = torch.zeros(R, dtype=torch.int32, device=dev)
@@ -714,7 +717,7 @@ def time_identify_heads(pk, loop, w, flush_l2, peak, calls=16, warm=2):
         counts.zero_()
         if i >= warm:
             ev[i - warm][0].record(s)
-        pk.pldp_identify_heads(loop.ids, pos, loop.A, counts)
+        pk.pldp_identify_heads(loop.ids, pos, A_rows, counts)
         pk.pldp_top_heads(counts, k, top)
         if i >= warm:
             ev[i - warm][1].record(s)
@@ -851,6 +854,7 @@ def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
     best_h, best_a = torch.zeros(B, **i32), torch.zeros(B, **i32)
     draft, dlen = torch.zeros((B, w.K), **i32), torch.zeros(B, **i32)
     dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=dev)
+    A_head = loop.A.contiguous()              # the same rows with each row's keys side by side
     out = {}
     for V in (256, 64):
         g = torch.Generator(device=dev).manual_seed(w.seed + V)
@@ -859,15 +863,18 @@ def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
         torch.cuda.synchronize()
         n_list = float(cnt.clamp(0, C).sum().item())
         calls = [("rank_hidden", lambda: pk.pldp_rank_hidden(loop.H, L, cand, cnt, best_h)),
-                 ("rank_attention", lambda: pk.pldp_rank_attention(loop.A, L, cand, cnt, best_a))]
+                 ("rank_attention", lambda: pk.pldp_rank_attention(loop.A, L, cand, cnt, best_a)),
+                 ("rank_attention_head_major", lambda: pk.pldp_rank_attention(A_head, L, cand, cnt, best_a))]
         times = {}
         for c in calls:
             times.update(_time_calls([c], flush_l2, iters, warm))
-        by = {"rank_hidden": (n_list + B) * w.d * 2.0, "rank_attention": n_list * w.R * 2.0}
+        by = {"rank_hidden": (n_list + B) * w.d * 2.0, "rank_attention": n_list * w.R * 2.0,
+              "rank_attention_head_major": n_list * w.R * 2.0}
         rec = {"vocab": V, "ngram": [1, 1], "mean_candidates_listed": round(n_list / B, 1),
                **{k: _call_stats(v, by[k], peak) for k, v in times.items()}}
-        rec["rank_attention"]["sector_bytes"] = n_list * w.R * 32.0
-        rec["rank_attention"]["sector_gbs"] = round(n_list * w.R * 32.0 / (rec["rank_attention"]["us"] * 1e-6) / 1e9, 1)
+        hm = rec["rank_attention_head_major"]
+        hm["sector_bytes"] = n_list * w.R * 32.0
+        hm["sector_gbs"] = round(hm["sector_bytes"] / (hm["us"] * 1e-6) / 1e9, 1)
         if V == 256:      # at most 256 occurrences per sequence: the launch's own scoring path
             t = _time_calls([("draft_step", lambda: pk.pldp_draft_step(
                 ids, L, 1, 1, cand, cnt, ml, w.K, draft, dlen, dws, H=loop.H, best_h=best_h, A=loop.A,
@@ -876,7 +883,10 @@ def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
             rec["draft_step"] = _call_stats(t["draft_step"], by_d, peak)
         out[f"vocab{V}"] = rec
         del ids
+    del A_head
     out.update({"batch": B, "context": T, "d": w.d, "attention_rows": w.R, "C_cap": C,
+                "attention_layout": "rank_attention: key-major (the loop's layout); rank_attention_head_major: "
+                                    "the same values with each row's keys side by side",
                 "timing": "CUDA events around each call, L2 flushed before each; hidden rows and attention "
                           "values are the decode loop's own tensors"})
     return out
@@ -902,7 +912,7 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     B, K1 = w.B, w.K + 1
     A_dev = loop.A
     h_logits = torch.empty(loop.logits.shape, dtype=loop.logits.dtype, pin_memory=True)
-    h_A = torch.empty(A_dev.shape, dtype=A_dev.dtype, pin_memory=True)
+    h_A = torch.empty_strided(A_dev.shape, A_dev.stride(), dtype=A_dev.dtype, pin_memory=True)   # same layout
     h_H = torch.empty((B, K1, w.d), dtype=loop.H.dtype, pin_memory=True)
     d_H = torch.empty((B, K1, w.d), dtype=loop.H.dtype, device=dev)
     res = torch.empty((B, 3 + w.K), dtype=torch.int32, device=dev)
@@ -912,6 +922,9 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     times = []
     sectors = 0.0
     steps = K_steps
+    # bytes that cross the link per ranked candidate: its R values, one 32-byte sector
+    # each (rows with contiguous keys) or together (key-major)
+    per_cand = (w.R * 32.0 if A_dev.stride(2) == 1 else float(-(-w.R * A_dev.element_size() // 32) * 32))
     try:
         for s in range(W_steps + steps):
             loop.A = A_dev
@@ -933,7 +946,7 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
             torch.cuda.synchronize()
             if s >= W_steps:
                 times.append(time.perf_counter() - t0)
-                sectors += float(path.cnt.clamp(0, w.C_cap).sum()) * w.R * 32.0
+                sectors += float(path.cnt.clamp(0, w.C_cap).sum()) * per_cand
     finally:
         loop.A = A_dev
     tot = max_over_ranks(sum(times), ws_)
@@ -942,8 +955,8 @@ def run_e2e(pk, loop, path, K_steps, W_steps, ws_):
     return {"value": round(ws_ * steps / tot, 2), "unit": "steps/s",
             "ms_per_step": round(tot / steps * 1e3, 3),
             "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(h_res.numel() * 4),
-            "attention_rows": "in pinned host memory, read in place by the drafting (32-byte sectors at the "
-                              "candidate keys counted in h2d_bytes_per_step)",
+            "attention_rows": "in pinned host memory, read in place by the drafting (the 32-byte sectors "
+                              "holding the candidate keys' values counted in h2d_bytes_per_step)",
             "timing": "host wall clock per step: H2D of logits and new hidden rows from pinned memory, the "
                       "step's C-ABI calls, D2H of accept/next/seq_len/draft, synchronize"}
 

@@ -175,13 +175,21 @@ PLDP_API pldp_status pldp_rank_hidden_avg(const void* H, pldp_dtype dtype, int64
  * induction head at query t-1 attends to is the token it copies).
  *
  *  A          dtype; for sequence b and row r the attention probabilities of
- *             query t-1 over keys: A + b*seq_stride + r*row_stride + key.  A may
- *             also be page-locked host memory that device code can address (a
- *             cudaHostAlloc allocation under unified addressing): the kernels read
- *             only the selected rows' values at the candidate keys, so rows kept
- *             on the host need not be copied to the device whole.
- *  R          rows per sequence (>= 1); row_stride >= T_cap; seq_stride >=
- *             R * row_stride.
+ *             query t-1 over keys:
+ *               A + b*seq_stride + r*row_stride + key*key_stride.
+ *             Rows with contiguous keys (key_stride = 1, row_stride >= T_cap) are
+ *             the natural layout of one head's probabilities; the key-major layout
+ *             (row_stride = 1, key_stride >= R) puts the R values of one key side
+ *             by side, so each candidate's values are one contiguous read instead
+ *             of R scattered 32-byte sectors.  A may also be page-locked host
+ *             memory that device code can address (a cudaHostAlloc allocation
+ *             under unified addressing): the kernels read only the selected rows'
+ *             values at the candidate keys, so rows kept on the host need not be
+ *             copied to the device whole.
+ *  R          rows per sequence (>= 1).
+ *  row_stride, key_stride   >= 1 (key_stride 0 is read as 1); the rows must not
+ *             overlap: row_stride >= T_cap * key_stride or key_stride >= R *
+ *             row_stride.  seq_stride >= (R-1)*row_stride + (T_cap-1)*key_stride + 1.
  *  row_idx    int32 [n_sel] device, or NULL for all R rows: the selected
  *             (layer, head) rows L* x G*.  Entries outside [0, R) are ignored
  *             and set ROW_INDEX.
@@ -192,7 +200,7 @@ PLDP_API pldp_status pldp_rank_hidden_avg(const void* H, pldp_dtype dtype, int64
  * MAX is exact; SUM accumulates in fp32 in a fixed order.
  */
 PLDP_API pldp_status pldp_rank_attention(const void* A, pldp_dtype dtype, int R,
-                                         int64_t row_stride, int64_t seq_stride,
+                                         int64_t row_stride, int64_t key_stride, int64_t seq_stride,
                                          const int32_t* row_idx, int n_sel, pldp_agg agg,
                                          const int32_t* seq_len, int B, int64_t T_cap,
                                          const int32_t* cand_pos, const int32_t* cand_count,
@@ -238,7 +246,8 @@ PLDP_API pldp_status pldp_extract_draft(const int32_t* ids, int64_t ids_stride,
  *  H .. best_h_score     as pldp_rank_hidden (H = NULL skips hidden ranking;
  *                        H rows must be 16-byte aligned).  h_scores and
  *                        best_h_score may be NULL.
- *  A .. best_a_score     as pldp_rank_attention (A = NULL skips it; A may be
+ *  A .. best_a_score     as pldp_rank_attention (A = NULL skips it; either
+ *                        layout, a_key_stride as its key_stride; A may be
  *                        device-addressable page-locked host memory); a_scores
  *                        and best_a_score may be NULL.
  *  draft_from            0: draft after best_h, 1: after best_a (that ranking
@@ -289,6 +298,7 @@ typedef struct pldp_draft_step_args {
     pldp_dtype a_dtype;
     int R;
     int64_t a_row_stride;
+    int64_t a_key_stride;   /* elements between keys of a row; 0 is read as 1 */
     int64_t a_seq_stride;
     const int32_t* row_idx;
     int n_sel;

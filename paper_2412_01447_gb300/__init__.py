@@ -92,7 +92,8 @@ class pldp_draft_step_args(ctypes.Structure):
         ("h_seq_stride", ctypes.c_int64), ("threshold", ctypes.c_float), ("h_scores", ctypes.c_void_p),
         ("best_h", ctypes.c_void_p), ("best_h_score", ctypes.c_void_p),
         ("A", ctypes.c_void_p), ("a_dtype", ctypes.c_int), ("R", ctypes.c_int),
-        ("a_row_stride", ctypes.c_int64), ("a_seq_stride", ctypes.c_int64), ("row_idx", ctypes.c_void_p),
+        ("a_row_stride", ctypes.c_int64), ("a_key_stride", ctypes.c_int64), ("a_seq_stride", ctypes.c_int64),
+        ("row_idx", ctypes.c_void_p),
         ("n_sel", ctypes.c_int), ("agg", ctypes.c_int), ("a_scores", ctypes.c_void_p),
         ("best_a", ctypes.c_void_p), ("best_a_score", ctypes.c_void_p),
         ("draft_from", ctypes.c_int), ("K", ctypes.c_int), ("draft", ctypes.c_void_p),
@@ -154,7 +155,7 @@ def _load():
             lib.pldp_rank_hidden_avg.argtypes = [P, i32, i64, i64, i32, P, i32, i64, P, P, i32, f32, P, P,
                                                  P, P, P]
             lib.pldp_rank_hidden_avg.restype = ctypes.c_int
-            lib.pldp_rank_attention.argtypes = [P, i32, i32, i64, i64, P, i32, i32, P, i32, i64, P,
+            lib.pldp_rank_attention.argtypes = [P, i32, i32, i64, i64, i64, P, i32, i32, P, i32, i64, P,
                                                 P, i32, P, P, P, P, P]
             lib.pldp_extract_draft.argtypes = [P, i64, P, i64, P, i32, i32, P, P, P]
             lib.pldp_verify_greedy.argtypes = [P, i32, i32, i32, i32, P, P, P, P, P, P, i64, P, i64,
@@ -353,16 +354,17 @@ def pldp_top_heads(counts, k, row_idx, stream=None):
 def pldp_rank_attention(A, seq_len, cand_pos, cand_count, best_pos, row_idx=None, agg=PLDP_AGG_MAX,
                         scores=None, best_score=None, status=None, stream=None):
     """Eq. 2.  A: [B, R, T_cap] float32/bfloat16, attention of query t-1 for each of R
-    (layer, head) rows (unit inner stride), on the device or in pinned host memory (read
-    in place: only the selected rows' values at the candidate keys cross the link);
-    row_idx int32 [n_sel] device or None (all)."""
-    if A.dim() != 3 or A.stride(2) != 1:
-        raise ValueError("A must be [B, R, T_cap] with unit inner stride")
+    (layer, head) rows, with contiguous keys (each row dense) or key-major (the R values
+    of a key dense: e.g. a [B, T_cap, R] tensor transposed to [B, R, T_cap]), on the
+    device or in pinned host memory (read in place: only the selected rows' values at the
+    candidate keys cross the link); row_idx int32 [n_sel] device or None (all)."""
+    if A.dim() != 3:
+        raise ValueError("A must be [B, R, T_cap]")
     B, R, T_cap = A.shape
     C_cap = cand_pos.shape[1]
     n_sel = R if row_idx is None else row_idx.numel()
     _check("pldp_rank_attention", _load().pldp_rank_attention(
-        _dev_or_pinned(A, "A"), _code(A.dtype), R, A.stride(1), A.stride(0),
+        _dev_or_pinned(A, "A"), _code(A.dtype), R, A.stride(1), A.stride(2), A.stride(0),
         _dense(row_idx, "row_idx", torch.int32, allow_none=True), n_sel, int(agg),
         _dense(seq_len, "seq_len", torch.int32, n=B), B, T_cap, _dense(cand_pos, "cand_pos", torch.int32, n=B * C_cap),
         _dense(cand_count, "cand_count", torch.int32, n=B), C_cap,
@@ -413,12 +415,12 @@ def _draft_args(ids, seq_len, ngram_min, ngram_max, cand_pos, cand_count, match_
         a.best_h = _dense(best_h, "best_h", torch.int32, n=B)
         a.best_h_score = _dense(best_h_score, "best_h_score", torch.float32, allow_none=True, n=B)
     if A is not None:
-        if A.dim() != 3 or A.stride(2) != 1:
-            raise ValueError("A must be [B, R, T_cap] with unit inner stride")
+        if A.dim() != 3:
+            raise ValueError("A must be [B, R, T_cap]")
         if A.shape[0] < B or A.shape[2] < T:
             raise ValueError(f"A must cover [B, T_cap] = [{B}, {T}] positions")
         a.A, a.a_dtype, a.R = _dev_or_pinned(A, "A"), _code(A.dtype), A.shape[1]
-        a.a_row_stride, a.a_seq_stride = A.stride(1), A.stride(0)
+        a.a_row_stride, a.a_key_stride, a.a_seq_stride = A.stride(1), A.stride(2), A.stride(0)
         a.row_idx = _dense(row_idx, "row_idx", torch.int32, allow_none=True)
         a.n_sel = A.shape[1] if row_idx is None else row_idx.numel()
         a.agg = int(agg)

@@ -83,6 +83,7 @@ struct DraftParams {
     bool a_bf16;
     int R;
     int64_t a_row_stride;
+    int64_t a_key_stride;
     int64_t a_seq_stride;
     const int32_t* row_idx;
     int n_sel;
@@ -198,7 +199,7 @@ __device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int
         const bool rv = r >= 0 && r < p.R;
 #pragma unroll
         for (int h = 0; h < NB; ++h)
-            av[h] = (rv && a_ok[h]) ? load_attn(ab, static_cast<int64_t>(r) * p.a_row_stride + j[h], p.a_bf16) : NAN;
+            av[h] = (rv && a_ok[h]) ? load_attn(ab, static_cast<int64_t>(r) * p.a_row_stride + j[h] * p.a_key_stride, p.a_bf16) : NAN;
     }
     if constexpr (HAS_H) {
         if (any_h) {
@@ -245,7 +246,7 @@ __device__ __forceinline__ void cta_score(const DraftParams& p, int b, const int
             float v[NB];
 #pragma unroll
             for (int h = 0; h < NB; ++h)
-                v[h] = (rv && a_ok[h]) ? load_attn(ab, static_cast<int64_t>(r) * p.a_row_stride + j[h], p.a_bf16) : NAN;
+                v[h] = (rv && a_ok[h]) ? load_attn(ab, static_cast<int64_t>(r) * p.a_row_stride + j[h] * p.a_key_stride, p.a_bf16) : NAN;
 #pragma unroll
             for (int h = 0; h < NB; ++h)
                 if (v[h] == v[h]) acc[h] = is_max ? fmaxf(acc[h], v[h]) : acc[h] + v[h];
@@ -1198,9 +1199,9 @@ pldp_status prepare_draft(const pldp_draft_step_args* a, const char* what, Draft
         if (a->agg != PLDP_AGG_MAX && a->agg != PLDP_AGG_SUM)
             return fail(PLDP_ERR_INVALID_ARG, "%s: unknown aggregation %d", what, (int)a->agg);
         if (a->R < 1) return fail(PLDP_ERR_INVALID_ARG, "%s: R < 1", what);
-        if (a->a_row_stride < a->T_cap) return fail(PLDP_ERR_INVALID_ARG, "%s: a_row_stride < T_cap", what);
-        if (a->a_seq_stride < static_cast<int64_t>(a->R) * a->a_row_stride)
-            return fail(PLDP_ERR_INVALID_ARG, "%s: a_seq_stride < R*a_row_stride", what);
+        if (const char* why = attention_layout_error(a->R, a->T_cap, a->a_row_stride,
+                                                     a->a_key_stride == 0 ? 1 : a->a_key_stride, a->a_seq_stride))
+            return fail(PLDP_ERR_INVALID_ARG, "%s: attention layout: %s", what, why);
         sel = a->row_idx ? a->n_sel : a->R;
         if (sel < 1 || sel > kMaxSelRows)
             return fail(PLDP_ERR_INVALID_ARG, "%s: need 1 <= n_sel <= %d", what, kMaxSelRows);
@@ -1248,6 +1249,7 @@ pldp_status prepare_draft(const pldp_draft_step_args* a, const char* what, Draft
     p.a_bf16 = a->a_dtype == PLDP_BF16;
     p.R = a->R;
     p.a_row_stride = a->a_row_stride;
+    p.a_key_stride = a->a_key_stride == 0 ? 1 : a->a_key_stride;
     p.a_seq_stride = a->a_seq_stride;
     p.row_idx = a->row_idx;
     p.n_sel = sel;

@@ -334,7 +334,8 @@ __device__ __forceinline__ float load_attn(const void* base, int64_t idx, bool a
 // the scattered values are in flight.  Lane sums run in the order of the CTA path.
 template <bool CANDS_SHARED>
 __device__ __forceinline__ void attention_rank_warp(const void* ab, bool a_bf16, const int64_t* rows_sh, int n_sel,
-                                                    int64_t t, const int32_t* __restrict__ cands, int S, int rank,
+                                                    int64_t key_stride, int64_t t, const int32_t* __restrict__ cands,
+                                                    int S, int rank,
                                                     const int32_t* jpre, bool is_max, float* __restrict__ scores_row,
                                                     RankShared& sh, const Batch& bt) {
     const int lane = threadIdx.x & 31;
@@ -360,7 +361,8 @@ __device__ __forceinline__ void attention_rank_warp(const void* ab, bool a_bf16,
                 const int r = r0 + 32 * u;
                 const int64_t off = (r < n_sel) ? rows_sh[r] : -1;
 #pragma unroll
-                for (int c = 0; c < 2; ++c) v[c][u] = (ok[c] && off >= 0) ? load_attn(ab, off + j[c], a_bf16) : NAN;
+                for (int c = 0; c < 2; ++c)
+                    v[c][u] = (ok[c] && off >= 0) ? load_attn(ab, off + j[c] * key_stride, a_bf16) : NAN;
             }
 #pragma unroll
             for (int c = 0; c < 2; ++c)
@@ -394,12 +396,13 @@ __device__ __forceinline__ void attention_rank_warp(const void* ab, bool a_bf16,
 }
 
 // Eq. 2 for this CTA's candidates.  `rows_sh` (shared) holds the element offset
-// of each selected row, or -1 for an invalid one.  Same conventions as
+// of each selected row, or -1 for an invalid one; key j of a row is key_stride
+// elements after key j - 1.  Same conventions as
 // hidden_rank_cta; every candidate in [0, t) is eligible.  With CANDS_SHARED
 // the candidate list is in shared memory (else global, read through L2).
 template <bool CANDS_SHARED = false>
 __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
-                                                   const int64_t* rows_sh, int n_sel, int64_t t,
+                                                   const int64_t* rows_sh, int n_sel, int64_t key_stride, int64_t t,
                                                    const int32_t* __restrict__ cands, int n, int S,
                                                    int rank, const int32_t* jpre, bool is_max,
                                                    float* __restrict__ scores_row, RankShared& sh,
@@ -407,8 +410,8 @@ __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
     const int lane = threadIdx.x & 31, warp = wg.warp();
     const Batch bt = batch_shape(n, S, rank, wg);
     if (bt.G == 1) {                                      // one warp per candidate: no barriers
-        attention_rank_warp<CANDS_SHARED>(ab, a_bf16, rows_sh, n_sel, t, cands, S, rank, jpre, is_max, scores_row,
-                                          sh, bt);
+        attention_rank_warp<CANDS_SHARED>(ab, a_bf16, rows_sh, n_sel, key_stride, t, cands, S, rank, jpre, is_max,
+                                          scores_row, sh, bt);
         wg.sync();
         return;
     }
@@ -429,7 +432,7 @@ __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
                 for (int u = 0; u < U; ++u) {
                     const int r = r0 + step * u;
                     const int64_t off = (r < n_sel) ? rows_sh[r] : -1;
-                    v[u] = (off >= 0) ? load_attn(ab, off + j, a_bf16) : NAN;
+                    v[u] = (off >= 0) ? load_attn(ab, off + j * key_stride, a_bf16) : NAN;
                 }
 #pragma unroll
                 for (int u = 0; u < U; ++u)
@@ -459,6 +462,20 @@ __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
         }
         wg.sync();
     }
+}
+
+// Host: the attention layout rules of the ranking calls (A + b*seq_stride +
+// r*row_stride + key*key_stride, rows that do not overlap).  Returns null when the
+// layout is valid, else what is wrong.
+inline const char* attention_layout_error(int R, int64_t T_cap, int64_t row_stride, int64_t key_stride,
+                                          int64_t seq_stride) {
+    if (row_stride < 1 || key_stride < 1) return "row and key strides must be >= 1";
+    const bool head_major = row_stride >= T_cap * key_stride;
+    const bool key_major = key_stride >= static_cast<int64_t>(R) * row_stride;
+    if (!head_major && !key_major) return "rows overlap: need row_stride >= T_cap*key_stride or key_stride >= R*row_stride";
+    const int64_t extent = static_cast<int64_t>(R - 1) * row_stride + (T_cap > 0 ? T_cap - 1 : 0) * key_stride + 1;
+    if (seq_stride < extent) return "seq_stride shorter than one sequence's rows";
+    return nullptr;
 }
 
 // Stages the element offsets of the selected attention rows; returns (in every

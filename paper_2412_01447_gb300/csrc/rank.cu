@@ -304,7 +304,7 @@ rank_hidden_avg_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride, i
 
 template <bool CLUSTER>
 __global__ void __launch_bounds__(kThreads)
-rank_attention_kernel(const void* __restrict__ A, bool a_bf16, int R, int64_t row_stride,
+rank_attention_kernel(const void* __restrict__ A, bool a_bf16, int R, int64_t row_stride, int64_t key_stride,
                       int64_t seq_stride, const int32_t* __restrict__ row_idx, int n_sel, int agg,
                       const int32_t* __restrict__ seq_len, int64_t T_cap,
                       const int32_t* __restrict__ cand_pos, const int32_t* __restrict__ cand_count,
@@ -338,7 +338,7 @@ rank_attention_kernel(const void* __restrict__ A, bool a_bf16, int R, int64_t ro
     if (rank == 0 && tid == 0 && bad && status) atomicOr(status + b, PLDP_ST_ROW_INDEX);
     const size_t es = a_bf16 ? 2 : 4;
     const void* ab = static_cast<const char*>(A) + static_cast<int64_t>(b) * seq_stride * es;
-    attention_rank_cta(ab, a_bf16, rows_sh, n_sel, t, cand_pos + static_cast<int64_t>(b) * C_cap, n, S,
+    attention_rank_cta(ab, a_bf16, rows_sh, n_sel, key_stride, t, cand_pos + static_cast<int64_t>(b) * C_cap, n, S,
                        rank, sh.jpre, agg == PLDP_AGG_MAX,
                        scores ? scores + static_cast<int64_t>(b) * C_cap : nullptr, sh);
     store_best<CLUSTER>(sh, mine, b, best_pos, best_score, status, PLDP_ST_TIMEOUT);
@@ -393,15 +393,15 @@ cudaError_t launch_hidden(int B, int S, size_t smem, void* stream, const T* h, i
 }
 
 cudaError_t launch_attention(int B, int S, size_t smem, void* stream, const void* a, bool a_bf16,
-                             int R, int64_t row_stride, int64_t seq_stride, const int32_t* row_idx,
+                             int R, int64_t row_stride, int64_t key_stride, int64_t seq_stride, const int32_t* row_idx,
                              int sel, int agg, const int32_t* seq_len, int64_t T_cap,
                              const int32_t* cand_pos, const int32_t* cand_count, int C_cap,
                              float* scores, int32_t* best_pos, float* best_score, uint32_t* status) {
     if (S > 1)
-        return launch_rank(rank_attention_kernel<true>, B, S, smem, stream, a, a_bf16, R, row_stride,
+        return launch_rank(rank_attention_kernel<true>, B, S, smem, stream, a, a_bf16, R, row_stride, key_stride,
                            seq_stride, row_idx, sel, agg, seq_len, T_cap, cand_pos, cand_count, C_cap,
                            scores, best_pos, best_score, status);
-    return launch_rank(rank_attention_kernel<false>, B, S, smem, stream, a, a_bf16, R, row_stride,
+    return launch_rank(rank_attention_kernel<false>, B, S, smem, stream, a, a_bf16, R, row_stride, key_stride,
                        seq_stride, row_idx, sel, agg, seq_len, T_cap, cand_pos, cand_count, C_cap,
                        scores, best_pos, best_score, status);
 }
@@ -519,7 +519,7 @@ extern "C" PLDP_API pldp_status pldp_rank_hidden(const void* H, pldp_dtype dtype
 }
 
 extern "C" PLDP_API pldp_status pldp_rank_attention(const void* A, pldp_dtype dtype, int R,
-                                                    int64_t row_stride, int64_t seq_stride,
+                                                    int64_t row_stride, int64_t key_stride, int64_t seq_stride,
                                                     const int32_t* row_idx, int n_sel, pldp_agg agg,
                                                     const int32_t* seq_len, int B, int64_t T_cap,
                                                     const int32_t* cand_pos,
@@ -534,9 +534,9 @@ extern "C" PLDP_API pldp_status pldp_rank_attention(const void* A, pldp_dtype dt
         return fail(PLDP_ERR_INVALID_ARG, "rank_attention: unknown aggregation %d", (int)agg);
     if (R < 1) return fail(PLDP_ERR_INVALID_ARG, "rank_attention: R < 1");
     if (T_cap < 0 || T_cap > INT32_MAX) return fail(PLDP_ERR_INVALID_ARG, "rank_attention: bad T_cap");
-    if (row_stride < T_cap) return fail(PLDP_ERR_INVALID_ARG, "rank_attention: row_stride < T_cap");
-    if (seq_stride < static_cast<int64_t>(R) * row_stride)
-        return fail(PLDP_ERR_INVALID_ARG, "rank_attention: seq_stride < R*row_stride");
+    if (key_stride == 0) key_stride = 1;
+    if (const char* why = attention_layout_error(R, T_cap, row_stride, key_stride, seq_stride))
+        return fail(PLDP_ERR_INVALID_ARG, "rank_attention: %s", why);
     const int sel = row_idx ? n_sel : R;
     if (sel < 1 || sel > kMaxSelRows)
         return fail(PLDP_ERR_INVALID_ARG, "rank_attention: need 1 <= n_sel <= %d", kMaxSelRows);
@@ -548,7 +548,7 @@ extern "C" PLDP_API pldp_status pldp_rank_attention(const void* A, pldp_dtype dt
     const size_t smem = static_cast<size_t>(sel) * sizeof(int64_t);
     const int S = pick_split(B, C_cap, reinterpret_cast<const void*>(&rank_attention_kernel<true>), smem);
     cudaError_t e;
-    e = launch_attention(B, S, smem, stream, A, dtype == PLDP_BF16, R, row_stride, seq_stride, row_idx,
+    e = launch_attention(B, S, smem, stream, A, dtype == PLDP_BF16, R, row_stride, key_stride, seq_stride, row_idx,
                          sel, static_cast<int>(agg), seq_len, T_cap, cand_pos, cand_count, C_cap,
                          scores, best_pos, best_score, status);
     if (e != cudaSuccess)

@@ -82,12 +82,18 @@ def test_host_argument_checks(so):
     assert lib.pldp_identify_heads(*bad) == 1 and "row_stride" in pk.pldp_last_error()
     assert lib.pldp_top_heads(ctypes.c_void_p(256), 4, 5, ctypes.c_void_p(256), null) == 1
     assert lib.pldp_top_heads(ctypes.c_void_p(256), 9000, 5, ctypes.c_void_p(256), null) == 1
-    # rank_attention: bad aggregation, n_sel out of range
-    a = [null, 1, 4, 8, 32, null, 4, 0, null, 1, 8, null, null, 4, null, null, null, null, null]
-    bad = list(a); bad[7] = 5
+    # rank_attention: bad aggregation, n_sel out of range, overlapping or short layouts
+    a = [null, 1, 4, 8, 1, 32, null, 4, 0, null, 1, 8, null, null, 4, null, null, null, null, null]
+    bad = list(a); bad[8] = 5
     assert lib.pldp_rank_attention(*bad) == 1
-    bad = list(a); bad[5] = ctypes.c_void_p(16); bad[6] = 0
+    bad = list(a); bad[6] = ctypes.c_void_p(16); bad[7] = 0
     assert lib.pldp_rank_attention(*bad) == 1
+    bad = list(a); bad[3], bad[4] = 2, 2                  # rows of 8 keys 2 apart, 2 apart: they overlap
+    assert lib.pldp_rank_attention(*bad) == 1 and "overlap" in pk.pldp_last_error()
+    bad = list(a); bad[5] = 31                            # one element short of the 4 rows of 8 keys
+    assert lib.pldp_rank_attention(*bad) == 1 and "seq_stride" in pk.pldp_last_error()
+    ok = list(a); ok[3], ok[4], ok[5] = 1, 4, 32          # key-major: the 4 values of a key side by side
+    assert lib.pldp_rank_attention(*ok) == 1 and "null" in pk.pldp_last_error()   # layout passes; no buffers
     # extract_draft: K < 1
     assert lib.pldp_extract_draft(null, 8, null, 8, null, 1, 0, null, null, null) == 1
     # verify_greedy: K < 1, ids without seq_len, workspace too small

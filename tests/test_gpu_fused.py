@@ -61,6 +61,8 @@ def test_draft_step_random(lib, T, V, B, mode):
         lens[3] = T + 3                       # invalid length
     H = torch.randn((B, T, d), generator=gen, device=DEV).to(torch.bfloat16) if mode != "attention" else None
     A = torch.rand((B, R, T), generator=gen, device=DEV).to(torch.bfloat16) if mode != "hidden" else None
+    if A is not None and T % 3 == 0:                  # key-major: the R values of a key side by side
+        A = A.transpose(1, 2).contiguous().transpose(1, 2)
     buf = Buffers(B, K, 8, C, DEV)
     draft_from = "attention" if mode == "attention" else "hidden"
     gpu_step(buf, i32(ids), i32(lens), None, H=H, A=A, draft_from=draft_from, append=False, fused=True)

@@ -1,7 +1,8 @@
 """Attention rows kept in pinned host memory: the rankings read them in place
 (only the selected rows' values at the candidate keys cross the link) and give
 exactly the results of the same rows on the device, for the separate Eq. 2
-ranking and for the one-launch drafting with the token index."""
+ranking and for the one-launch drafting with the token index, in both memory
+orders (each row's keys side by side, or the R values of each key)."""
 import numpy as np
 import pytest
 import torch
@@ -13,11 +14,15 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda"
 
 
-def test_rank_attention_reads_host_rows_in_place(lib):
+@pytest.mark.parametrize("layout", ["head", "key"])
+def test_rank_attention_reads_host_rows_in_place(lib, layout):
     rng = np.random.default_rng(4)
     B, R, T, C = 12, 32, 3000, 64
     A = torch.rand((B, R, T), device=DEV).to(torch.bfloat16)
-    A_host = A.cpu().pin_memory()
+    if layout == "key":
+        A = A.transpose(1, 2).contiguous().transpose(1, 2)
+    A_host = torch.empty_strided(A.shape, A.stride(), dtype=A.dtype, pin_memory=True)
+    A_host.copy_(A)
     lens = torch.as_tensor(rng.integers(2, T + 1, size=B).astype(np.int32), device=DEV)
     cands = torch.as_tensor(np.sort(rng.choice(T - 1, (B, C)), axis=1).astype(np.int32), device=DEV)
     cnt = torch.as_tensor(rng.integers(0, C + 1, size=B).astype(np.int32), device=DEV)
@@ -38,10 +43,11 @@ def test_draft_step_reads_host_rows_in_place(lib):
     ids = torch.as_tensor(rng.integers(0, V, size=(B, T)).astype(np.int32), device=DEV)
     L = torch.as_tensor(rng.integers(2, T + 1, size=B).astype(np.int32), device=DEV)
     H = torch.randn((B, T, d), device=DEV).to(torch.bfloat16)
-    A = torch.rand((B, R, T), device=DEV).to(torch.bfloat16)
-    A_host = A.cpu().pin_memory()
+    A = torch.rand((B, T, R), device=DEV).to(torch.bfloat16).transpose(1, 2)      # key-major
+    A_host = torch.empty_strided(A.shape, A.stride(), dtype=A.dtype, pin_memory=True)
+    A_host.copy_(A)
     out = []
-    for src in (A, A_host):
+    for src in (A, A_host, A.contiguous()):                                      # ... and head-major
         index = torch.empty(pk.pldp_index_size(B, V), dtype=torch.uint8, device=DEV)
         pk.pldp_index_build(ids, L, V, index)
         buf = Buffers(B, K, V, 64, DEV)
@@ -51,4 +57,5 @@ def test_draft_step_reads_host_rows_in_place(lib):
         out.append(snapshot(buf))
     for k in ("cand", "cnt", "best_h", "best_a", "scores_a", "bscore_a", "draft", "dlen", "status"):
         assert np.array_equal(out[0][k], out[1][k], equal_nan=True), k
+        assert np.array_equal(out[0][k], out[2][k], equal_nan=True), k
     assert (out[0]["cnt"] > 0).sum() > B // 2

@@ -46,7 +46,8 @@ def test_identify_heads_matches_oracle(lib, T, dtype, V, max_suffix):
 
 
 def test_identify_recovers_planted_heads(lib):
-    w = wl.CONFIGS["attention_b32_ctx8k"].replace(B=32, prompt_len=3000, out_len=1000, V=8000)
+    w = wl.CONFIGS["attention_b32_ctx8k"].replace(B=32, prompt_len=3000, out_len=1000, V=8000,
+                                                  attn_layout="head")   # identification reads whole rows
     tok, src = wl.token_streams(w, w.T, 99)
     rng = np.random.default_rng(100)
     obs_b, obs_p = [], []

@@ -140,10 +140,13 @@ def test_rank_hidden_tie_goes_to_smaller_position(lib):
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("agg", [0, 1])
 @pytest.mark.parametrize("rows", [None, [3, 0, 7, 15], [2, -1, 99, 5]])
-def test_rank_attention(lib, dtype, agg, rows):
+@pytest.mark.parametrize("layout", ["head", "key"])
+def test_rank_attention(lib, dtype, agg, rows, layout):
     rng = np.random.default_rng(3 + agg)
     B, R, T, C_cap = 10, 16, 777, 96
     A = torch.rand((B, R, T), device=DEV).to(dtype)
+    if layout == "key":                                  # the same values, the R of a key side by side
+        A = A.transpose(1, 2).contiguous().transpose(1, 2)
     A[:, :, 5] = A[:, :, 9]                           # ties between columns 5 and 9
     lens = rng.integers(0, T + 1, size=B)
     lens[:3] = [0, 1, T]

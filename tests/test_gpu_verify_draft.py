@@ -142,6 +142,8 @@ def _verify_draft_case(T, V, B, mode, shared, K, C, ngram, dt):
     lens[4] = 0                               # empty: verification refuses it (SEQ_LEN), drafting finds nothing
     H = torch.randn((B, T_cap, d), generator=gen, device=DEV).to(dt) if mode != "attention" else None
     A = torch.rand((B, R, T_cap), generator=gen, device=DEV).to(dt) if mode != "hidden" else None
+    if A is not None and T % 3 == 0:                  # key-major: the R values of a key side by side
+        A = A.transpose(1, 2).contiguous().transpose(1, 2)
     draft_from = "attention" if mode == "attention" else "hidden"
     ids_a, L_a = i32(ids), i32(lens)
     ids_b, L_b = ids_a.clone(), L_a.clone()

@@ -24,7 +24,8 @@ Recipe (every config):
     is the true continuation at the measured step.
   * attention rows of query t-1 (R = layers x heads): softmax over keys 0..t-1
     of N(0, 1) logits, +6 at the source of x_t in ``planted_heads`` heads of
-    every layer; keys >= t are 0.
+    every layer; keys >= t are 0.  Held key-major by default (the R values of one
+    key side by side, [B, T_cap, R] in memory, seen as [B, R, T_cap]).
   * target logits: N(0, 1); a planted row gets its chosen token set to
     (row max + 1), which makes that token the unique argmax.
   * bf16 tensors come from torch's bf16 generators (round-to-nearest-even casts
@@ -64,6 +65,8 @@ class Workload:
     heads: int = 0
     planted_heads: int = 0
     planted_logit: float = 6.0
+    attn_layout: str = "key"         # memory order of the attention rows: "key" (the R values of a key
+                                     # side by side) or "head" (each row's keys side by side)
     accept: str = "uniform"          # "fixed:<n>", "uniform" (U{0..K}) or "ground_truth"
     steps: int = 1
     seed: int = 1000
@@ -203,13 +206,21 @@ def induction_rows(w: Workload) -> np.ndarray:
     return np.asarray(rows, np.int32)
 
 
+def empty_attention(w: Workload, T_cap: int, device) -> torch.Tensor:
+    """An uninitialised [B, R, T_cap] bf16 attention tensor in the workload's memory
+    order: key-major storage [B, T_cap, R] viewed as [B, R, T_cap], or head-major."""
+    if w.attn_layout == "key":
+        return torch.empty((w.B, T_cap, w.R), dtype=torch.bfloat16, device=device).transpose(1, 2)
+    return torch.empty((w.B, w.R, T_cap), dtype=torch.bfloat16, device=device)
+
+
 def gen_attention(w: Workload, seq_len: torch.Tensor, src_of_last: torch.Tensor, T_cap: int,
                   device, gen: torch.Generator, out: Optional[torch.Tensor] = None,
                   chunk: int = 8) -> torch.Tensor:
     """Attention rows of query t-1: [B, R, T_cap] bf16.  ``seq_len`` and
     ``src_of_last`` (the source of x_t, -1 if none) are device tensors [B]."""
     B, R = w.B, w.R
-    A = out if out is not None else torch.empty((B, R, T_cap), dtype=torch.bfloat16, device=device)
+    A = out if out is not None else empty_attention(w, T_cap, device)
     planted = torch.zeros(R, dtype=torch.bool, device=device)
     planted[torch.from_numpy(induction_rows(w).astype(np.int64)).to(device)] = True
     keys = torch.arange(T_cap, device=device)
@@ -317,7 +328,7 @@ class DecodeLoop:
         self.gen = torch.Generator(device=device)
         self.gen.manual_seed(self.seed)
         self.H = gen_hidden(w, src, self.T_cap, device, self.gen) if (with_hidden and w.d) else None
-        self.A = (torch.empty((w.B, w.R, self.T_cap), dtype=torch.bfloat16, device=device)
+        self.A = (empty_attention(w, self.T_cap, device)
                   if (with_attention and w.R) else None)
         self.logits = torch.empty((w.B, w.K + 1, w.V), dtype=torch_dtype(w.logits_dtype),
                                   device=device)
