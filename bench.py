@@ -72,8 +72,10 @@ def parse():
                          "pldp_verify_greedy_draft call (which verifies a step and drafts the next)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sample", action="store_true",
-                    help="skip the separate timings on the loop's tensors (rank stress, sampling verification, "
-                         "averaged ranking, head identification)")
+                    help="skip the separate timings of sampling verification (alone and with the next draft), "
+                         "averaged ranking and head identification on the loop's tensors")
+    ap.add_argument("--no-rank-stress", action="store_true",
+                    help="skip the candidate-heavy ranking timings")
     ap.add_argument("--no-configs", action="store_true",
                     help="skip the per-call timing of the four single-step workloads")
     ap.add_argument("--ref-seqs", type=int, default=2, help="sequences per oracle step (reference arm)")
@@ -530,8 +532,9 @@ def run_ours(args, ws_, rank, local):
         out["two_call_variant"] = two_call
     if path.index is not None:
         out["draft_scan_variant"] = time_scan_variant(pk, loop, w, flush_l2)
-    if not args.no_sample:
+    if not args.no_rank_stress:
         out["rank_stress"] = time_rank_stress(pk, loop, w, flush_l2, peak)
+    if not args.no_sample:
         out["sampling_verify"] = time_sampling_verify(pk, loop, w, flush_l2, peak)
         if path.vd:
             out["sampling_verify_draft"] = time_sample_draft_loop(pk, loop, path, w, flush_l2, peak)
@@ -841,9 +844,9 @@ def time_single_step_configs(pk, flush_l2, peak, iters=32, warm=3):
 def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
     """Candidate-heavy ranking, reported apart from the headline: the decode loop's
     batch, context and artifacts (bf16 hidden rows of width d, R attention rows) with
-    contexts drawn from a small vocabulary and Eq. 1's unigram match (n-gram 1..1),
-    so that x_t has hundreds of earlier occurrences and the rankings have bytes to
-    move.  Each call timed with CUDA events, L2 flushed before each; the candidate
+    contexts drawn from a small vocabulary (context / 128 and context / 512 tokens)
+    and Eq. 1's unigram match (n-gram 1..1), so that x_t has about 128 and 512
+    earlier occurrences and the rankings have bytes to move.  Each call timed with CUDA events, L2 flushed before each; the candidate
     lists come from one untimed pldp_find_candidates call."""
     dev = loop.device
     B, T, C = w.B, w.T, w.C_cap
@@ -856,7 +859,7 @@ def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
     dws = torch.zeros(pk.pldp_draft_workspace_size(B), dtype=torch.uint8, device=dev)
     A_head = loop.A.contiguous()              # the same rows with each row's keys side by side
     out = {}
-    for V in (256, 64):
+    for V in (max(2, T // 128), max(2, T // 512)):     # about 128 and 512 earlier occurrences of x_t
         g = torch.Generator(device=dev).manual_seed(w.seed + V)
         ids = torch.randint(0, V, (B, T_cap), generator=g, device=dev, dtype=torch.int32)
         pk.pldp_find_candidates(ids, L, 1, 1, cand, cnt, ml)
@@ -875,13 +878,14 @@ def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
         hm = rec["rank_attention_head_major"]
         hm["sector_bytes"] = n_list * w.R * 32.0
         hm["sector_gbs"] = round(hm["sector_bytes"] / (hm["us"] * 1e-6) / 1e9, 1)
-        if V == 256:      # at most 256 occurrences per sequence: the launch's own scoring path
+        if V == max(2, T // 128):      # at most 256 occurrences per sequence: the launch's own scoring path
             t = _time_calls([("draft_step", lambda: pk.pldp_draft_step(
                 ids, L, 1, 1, cand, cnt, ml, w.K, draft, dlen, dws, H=loop.H, best_h=best_h, A=loop.A,
                 best_a=best_a, draft_from="hidden"))], flush_l2, iters, warm)
             by_d = 4.0 * B * T + by["rank_hidden"] + by["rank_attention"] + 4.0 * B * w.K
             rec["draft_step"] = _call_stats(t["draft_step"], by_d, peak)
         out[f"vocab{V}"] = rec
+        rec["label"] = f"~{T // V} occurrences per sequence"
         del ids
     del A_head
     out.update({"batch": B, "context": T, "d": w.d, "attention_rows": w.R, "C_cap": C,
