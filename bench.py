@@ -536,12 +536,13 @@ def run_ours(args, ws_, rank, local):
         out["rank_stress"] = time_rank_stress(pk, loop, w, flush_l2, peak)
     if not args.no_sample:
         out["sampling_verify"] = time_sampling_verify(pk, loop, w, flush_l2, peak)
-        if path.vd:
-            out["sampling_verify_draft"] = time_sample_draft_loop(pk, loop, path, w, flush_l2, peak)
         out["rank_hidden_avg"] = time_rank_hidden_avg(pk, loop, path, w, flush_l2, peak)
         out["identify_heads"] = time_identify_heads(pk, loop, w, flush_l2, peak)
+        if path.vd:       # last: sampling leaves contexts that no longer follow the ground truth
+            out["sampling_verify_draft"] = time_sample_draft_loop(pk, loop, path, w, flush_l2, peak)
     if not args.no_configs:
-        out["configs"] = time_single_step_configs(pk, flush_l2, peak)
+        out["configs"] = time_single_step_configs(pk, flush_l2, peak, oracle_timing=(
+            rank == 0 and ws_ == 1 and not args.no_cpu_baseline))
     if not args.no_e2e:
         out["e2e"] = run_e2e(pk, loop, path, K_steps, W_steps, ws_)
     if rank == 0 and ws_ == 1 and not args.no_cpu_baseline:
@@ -765,15 +766,67 @@ def _call_stats(us, by, peak):
 SINGLE_STEP = ("one_step_b1_ctx512", "hidden_b8_ctx4k", "hidden_b64_ctx16k", "attention_b32_ctx8k")
 
 
-def time_single_step_configs(pk, flush_l2, peak, iters=32, warm=3):
+def oracle_single_step(orc, inp, w):
+    """The oracle's whole step on a single-step workload's inputs (host copies), timed
+    on one host core: candidate search, the workload's ranking, draft, greedy
+    verification with append.  The hidden / attention host arrays hold only the rows
+    the oracle's ranking reads (zero pages elsewhere), as in the CPU baseline."""
+    ids, L = _host(inp["ids"]).copy(), _host(inp["seq_len"]).copy()
+    lg = _host(inp["logits"])
+    cand, cnt, _, _ = orc.find_candidates(ids, L, w.ngram_min, w.ngram_max, w.C_cap)
+    Hs, As = sparse_rows(inp["H"], inp["A"], L, cand, cnt)
+    t0 = time.perf_counter()
+    cand, cnt, _, _ = orc.find_candidates(ids, L, w.ngram_min, w.ngram_max, w.C_cap)
+    if Hs is not None:
+        _, best, _ = orc.rank_hidden(Hs, L, cand, cnt)
+    else:
+        _, best, _ = orc.rank_attention(As, L, cand, cnt)
+    draft, dl = orc.extract_draft(ids, L, best, w.K)
+    orc.verify_greedy(lg, draft, dl, ids=ids, seq_len=L, kv_keep=True)
+    return (time.perf_counter() - t0) * 1e6
+
+
+def sparse_rows(H, A, L, cand, cnt):
+    """Host copies of H [B, T_cap, d] and A [B, R, T_cap] (device tensors or None) that
+    hold, per sequence, H_{t-1}, each listed candidate's H_{j-1} and A[:, j]; every
+    other row is a zero page that is never touched."""
+    B = len(L)
+    bh, rh, ba, ja = [], [], [], []
+    for b in range(B):
+        t = int(L[b]) - 1
+        if t < 1:
+            continue
+        js = cand[b, :max(0, min(int(cnt[b]), cand.shape[1]))].astype(np.int64)
+        js = js[(js >= 0) & (js < t)]
+        rows = np.unique(np.concatenate([js[js >= 1] - 1, [t - 1]]))
+        bh += [b] * rows.size
+        rh += rows.tolist()
+        ba += [b] * js.size
+        ja += js.tolist()
+    Hs = As = None
+    if H is not None:
+        Hs = np.zeros(tuple(H.shape), np.uint16 if H.dtype == torch.bfloat16 else np.float32)
+        if bh:
+            bi, ri = np.asarray(bh), np.asarray(rh)
+            Hs[bi, ri] = _host(H[torch.as_tensor(bi, device=H.device), torch.as_tensor(ri, device=H.device)])
+    if A is not None:
+        As = np.zeros(tuple(A.shape), np.uint16 if A.dtype == torch.bfloat16 else np.float32)
+        if ba:
+            bi, ji = np.asarray(ba), np.asarray(ja)
+            As[bi, :, ji] = _host(A[torch.as_tensor(bi, device=A.device), :, torch.as_tensor(ji, device=A.device)])
+    return Hs, As
+
+
+def time_single_step_configs(pk, flush_l2, peak, iters=32, warm=3, oracle_timing=False):
     """The four single-step workloads: one decode step each (the state restored before
     every iteration), timed per C-ABI call and for the whole step with CUDA events,
     L2 flushed before each step.  Two forms of the step: the five separate calls
     (candidate search, the workload's ranking, draft, greedy verification with append)
     and the fused drafting launch + verification.  Algorithmic bytes per call are the
     per-unit figures: 4 B per context position scanned, (|P| + 1) * d * s of hidden
-    rows, |P| * R * 2 B of attention values (32 B sectors in practice), K * 4 B of
-    draft, (K + 1) * V * s of logits."""
+    rows, |P| * R * 2 B of attention values, K * 4 B of draft, (K + 1) * V * s of
+    logits.  With oracle_timing the oracle's step on the same inputs is timed too
+    (one host core)."""
     dev = torch.device("cuda", torch.cuda.current_device())
     out = {}
     for name in SINGLE_STEP:
@@ -831,8 +884,11 @@ def time_single_step_configs(pk, flush_l2, peak, iters=32, warm=3):
             step = np.sum([np.asarray(v) for v in times.values()], axis=0)
             tot = sum(by[k] for k in times)
             rec[form]["step"] = _call_stats(step, tot, peak)
-        if A is not None:
-            rec["separate_calls"]["rank_attention"]["sector_bytes"] = n_list * w.R * 32.0
+        if oracle_timing:
+            import oracle
+            reset()
+            torch.cuda.synchronize()
+            rec["oracle_us_per_step"] = round(oracle_single_step(oracle, inp, w), 1)
         out[name] = rec
         del inp, H, A, logits, ids, L, ids0, L0
         torch.cuda.empty_cache()

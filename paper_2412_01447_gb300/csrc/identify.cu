@@ -7,11 +7,12 @@
 // G* x L*.
 //
 // pldp_identify_heads: a (group of kRowsPerCta rows, observation) grid of CTAs.
-//  1. The context before x_p is scanned for x_p (by every CTA of the observation:
-//     4 bytes per position against 2 R bytes of attention); every occurrence j gets its
-//     overlap ov(j) (the length of the common suffix of x[..j] and x[..p]) and
-//     r* = argmax ov, the smaller j on ties, from a CTA-wide max of packed keys
-//     (ov << 32 | ~j).
+//  1. The context before x_p is scanned for x_p, each cluster of up to 8 CTAs of
+//     the observation splitting it into consecutive parts (4 bytes per position
+//     against 2 R bytes of attention); every occurrence j gets its overlap ov(j)
+//     (the length of the common suffix of x[..j] and x[..p]) and r* = argmax ov,
+//     the smaller j on ties, from a max of packed keys (ov << 32 | ~j) over the
+//     CTA and then over the cluster's distributed shared memory.
 //  2. The R rows of query p-1 are reduced to their first maximum, one warp per
 //     row (16-byte streaming loads where rows allow, packed (value, ~key)
 //     maxima), and a row whose maximum is at r* adds one to counts[r].  The rows
@@ -28,6 +29,7 @@ constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxTopRows = 8192;   // counts staged in shared memory by pldp_top_heads
 constexpr int kRowsPerCta = 8;      // attention rows per CTA (one per warp)
+constexpr int kIdentCluster = 8;    // CTAs of one observation that share its copy-source scan
 
 // The first maximum of elements [0, n) of one attention row, by one warp, as a
 // packed (value, ~key) key.  Each lane keeps a running (max, first key) over its
@@ -105,6 +107,7 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
                       int64_t row_stride, int64_t seq_stride, unsigned* __restrict__ counts,
                       int32_t* __restrict__ r_star, uint32_t* __restrict__ status) {
     __shared__ unsigned long long wkey[kWarps];
+    __shared__ unsigned long long cta_key;                        // this CTA's best occurrence key
     pdl_enter();
     const int b = blockIdx.y;                                     // the CTAs of one observation are adjacent:
     const int r0 = blockIdx.x * kRowsPerCta;                      // its ids are read once from DRAM, then L2
@@ -131,21 +134,26 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
         const int r = r0 + warp + i * kWarps;
         rk[i] = r < r1 ? row_first_max<VEC>(ab + static_cast<int64_t>(r) * row_stride * es, a_bf16, p, lane) : 0ull;
     }
-    // 1. the copy source r*: positions [0, p) in tiles, eight loads in flight per thread
+    // 1. the copy source r*: the cluster's CTAs (those of one observation) scan
+    //    consecutive parts of [0, p) in tiles, eight loads in flight per thread, and
+    //    meet over distributed shared memory
+    cg::cluster_group cluster = cg::this_cluster();
+    const int64_t cs = static_cast<int64_t>(cluster.num_blocks()), crank = cluster.block_rank();
     unsigned long long best = 0;
     constexpr int U = 8;
     if constexpr (IVEC) {
         const int4* x4 = reinterpret_cast<const int4*>(x);
         const int64_t nq = (p + 3) / 4;                             // int4 units covering [0, p)
-        for (int64_t q0 = tid; q0 < nq; q0 += static_cast<int64_t>(kThreads) * U) {
+        const int64_t q_lo = nq * crank / cs, q_hi = nq * (crank + 1) / cs;
+        for (int64_t q0 = q_lo + tid; q0 < q_hi; q0 += static_cast<int64_t>(kThreads) * U) {
             int4 v[U];
 #pragma unroll
             for (int u = 0; u < U; ++u)
-                if (q0 + u * kThreads < nq) v[u] = __ldg(x4 + q0 + u * kThreads);
+                if (q0 + u * kThreads < q_hi) v[u] = __ldg(x4 + q0 + u * kThreads);
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const int64_t q = q0 + u * kThreads;
-                if (q >= nq) continue;
+                if (q >= q_hi) continue;
                 const int32_t e[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {
@@ -158,15 +166,16 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
             }
         }
     } else {
-        for (int64_t j0 = tid; j0 < p; j0 += static_cast<int64_t>(kThreads) * U) {
+        const int64_t j_lo = p * crank / cs, j_hi = p * (crank + 1) / cs;
+        for (int64_t j0 = j_lo + tid; j0 < j_hi; j0 += static_cast<int64_t>(kThreads) * U) {
             int32_t v[U];
 #pragma unroll
             for (int u = 0; u < U; ++u)
-                if (j0 + u * kThreads < p) v[u] = __ldg(x + j0 + u * kThreads);
+                if (j0 + u * kThreads < j_hi) v[u] = __ldg(x + j0 + u * kThreads);
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const int64_t j = j0 + u * kThreads;
-                if (j < p && v[u] == xp) {
+                if (j < j_hi && v[u] == xp) {
                     const unsigned long long key = occurrence_key(x, j, p, max_suffix);
                     best = key > best ? key : best;
                 }
@@ -176,9 +185,23 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
     best = warp_max_u64(best);
     if (lane == 0) wkey[warp] = best;
     __syncthreads();
-    best = 0;
+    if (tid == 0) {
+        unsigned long long k = 0;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) best = wkey[w] > best ? wkey[w] : best;
+        for (int w = 0; w < kWarps; ++w) k = wkey[w] > k ? wkey[w] : k;
+        cta_key = k;
+    }
+    cluster.sync();                                               // every CTA's part is in
+    if (tid == 0) {
+        unsigned long long k = 0;
+        for (int c = 0; c < static_cast<int>(cs); ++c) {
+            const unsigned long long o = *cluster.map_shared_rank(&cta_key, c);
+            k = o > k ? o : k;
+        }
+        wkey[0] = k;
+    }
+    cluster.sync();                                               // read before any CTA of the cluster leaves
+    best = wkey[0];
     const int64_t rs = best ? static_cast<int64_t>(0xFFFFFFFFu - static_cast<uint32_t>(best & 0xFFFFFFFFull)) : -1;
     if (tid == 0 && blockIdx.x == 0 && r_star) r_star[b] = static_cast<int32_t>(rs);
     if (rs < 0) return;
@@ -234,10 +257,14 @@ extern "C" PLDP_API pldp_status pldp_identify_heads(const int32_t* ids, int64_t 
     const bool bf16 = dtype == PLDP_BF16;
     const bool ivec = aligned16(ids) && ids_stride % 4 == 0;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const dim3 grid(static_cast<unsigned>((R + kRowsPerCta - 1) / kRowsPerCta), static_cast<unsigned>(B));
+    // the CTAs of an observation in clusters of up to kIdentCluster (the grid padded to a
+    // whole number of them; padding CTAs hold no rows and only scan)
+    const int groups = (R + kRowsPerCta - 1) / kRowsPerCta;
+    const int cs = groups < kIdentCluster ? groups : kIdentCluster;
+    const dim3 grid(static_cast<unsigned>((groups + cs - 1) / cs * cs), static_cast<unsigned>(B));
     cudaError_t e;
 #define PLDP_IDENTIFY_LAUNCH(V, I)                                                                          \
-    launch_pdl(identify_heads_kernel<V, I>, grid, dim3(kThreads), 0, s, 0, ids, ids_stride, pos, T_cap, max_suffix, \
+    launch_pdl(identify_heads_kernel<V, I>, grid, dim3(kThreads), 0, s, cs, ids, ids_stride, pos, T_cap, max_suffix, \
                A, bf16, R, row_stride, seq_stride, static_cast<unsigned*>(counts), r_star, status)
     if (vec)
         e = ivec ? PLDP_IDENTIFY_LAUNCH(true, true) : PLDP_IDENTIFY_LAUNCH(true, false);

@@ -65,3 +65,23 @@ def test_reference_arm_line_has_the_contract_keys(monkeypatch):
     e = out["e2e"]
     assert e["value"] == out["value"] and e["unit"] == out["unit"]
     assert e["h2d_bytes_per_step"] == 0 and e["d2h_bytes_per_step"] == 0
+
+
+def test_oracle_single_step_on_sparse_rows_matches_dense():
+    """The configs' oracle timing runs the oracle on host arrays holding only the rows
+    its ranking reads; its rankings there equal those on the whole tensors."""
+    import numpy as np
+    import torch
+    import oracle
+    w = wl.CONFIGS["attention_b32_ctx8k"].replace(B=3, prompt_len=300, out_len=100, V=50, d=64)
+    inp = wl.single_step(w, device="cpu")
+    ids, L = inp["ids"].numpy(), inp["seq_len"].numpy()
+    cand, cnt, _, _ = oracle.find_candidates(ids, L, w.ngram_min, w.ngram_max, w.C_cap)
+    Hs, As = bench.sparse_rows(inp["H"], inp["A"], L, cand, cnt)
+    dense_h = inp["H"].contiguous().view(torch.int16).numpy().view(np.uint16)
+    dense_a = inp["A"].contiguous().view(torch.int16).numpy().view(np.uint16)
+    for rank, full, sparse in ((oracle.rank_hidden, dense_h, Hs), (oracle.rank_attention, dense_a, As)):
+        s_f, b_f, _ = rank(full, L, cand, cnt)
+        s_s, b_s, _ = rank(sparse, L, cand, cnt)
+        assert np.array_equal(s_f, s_s, equal_nan=True) and np.array_equal(b_f, b_s)
+    assert bench.oracle_single_step(oracle, inp, w) > 0
