@@ -60,6 +60,6 @@ extern "C" {
 
 PLDP_API const char* pldp_last_error(void) { return pldp::g_last_error; }
 
-PLDP_API int pldp_version(void) { return 100; }  // 0.1.0
+PLDP_API int pldp_version(void) { return 200; }  // 0.2.0: attention key stride, fused sampling call
 
 }  // extern "C"

@@ -41,7 +41,7 @@ def test_no_stray_exports(so):
 
 
 def test_version_and_workspace_are_host_only():
-    assert pk.pldp_version() == 100
+    assert pk.pldp_version() == 200
     assert pk.pldp_verify_workspace_size(0, 1, 1) == 0 + 0
     n = pk.pldp_verify_workspace_size(128, 12, 128256)
     assert n >= 128 * 13 * 8 and n % 256 == 0                  # one 64-bit key per logits row
