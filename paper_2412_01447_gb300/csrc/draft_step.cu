@@ -1035,16 +1035,19 @@ __global__ void __launch_bounds__(kThreads, 1) verify_draft_kernel(const VerifyA
     __shared__ int32_t oldwin[kOldWin];                          // x_{Lw}, ..., x_{Lw + kOldWin - 1}
     const int b = blockIdx.x;
     // Read before the wait, since the argmax pass does not write them (its
-    // predecessors, which did, completed before it started): the indexed length
-    // and the last kOldWin tokens of the context as it was before this step's
-    // append -- the drafting's appended ids and suffix reach back into them.
+    // predecessors, which did, completed before it started): the indexed length,
+    // the last kOldWin tokens of the context as it was before this step's append --
+    // the drafting's appended ids and suffix reach back into them -- and the
+    // finish's draft, draft length and context length.
     const int64_t il = ix.ilen[b];
     const int64_t L_old = va.seq_len ? static_cast<int64_t>(va.seq_len[b]) : -1;
     const int64_t Lw = L_old - kOldWin;
     const int32_t* row_b = p.ids + static_cast<int64_t>(b) * p.ids_stride;
+    FinishIn fin = {};
     if (threadIdx.x < kOldWin) {
         const int64_t q = Lw + threadIdx.x;
         oldwin[threadIdx.x] = (L_old >= 1 && L_old <= p.T_cap && q >= 0) ? __ldcg(row_b + q) : 0;
+        fin = finish_inputs(va, b, static_cast<int>(threadIdx.x));    // the draft: not written by the pass
     }
     pdl_enter();                                                  // the pass's row keys are final
     if (threadIdx.x < 32) {
@@ -1053,7 +1056,7 @@ __global__ void __launch_bounds__(kThreads, 1) verify_draft_kernel(const VerifyA
         FinishOut fo;
         const int64_t r0 = static_cast<int64_t>(b) * (va.K + 1);
         const RowTokens src{va.row_draws ? nullptr : va.row_keys + r0, va.row_draws ? va.row_draws + r0 : nullptr};
-        const int64_t L1 = finish_sequence(va, b, lane, src, &fo);
+        const int64_t L1 = finish_sequence(va, b, lane, src, &fo, &fin);
         if (lane == 0) L_after = L1;
         // The drafting's first reads come from what the finish holds: the ids appended
         // since the index was brought up to date (il .. t-1) and the suffix x_t, x_{t-1},

@@ -62,20 +62,36 @@ struct FinishOut {
     bool appended;  // draft[0..n-1] and bonus were written at positions L .. L+n
 };
 
+// The finish's inputs that do not depend on the target tokens (the draft length,
+// the context length and lane i's draft token i), for a caller that reads them
+// before the tokens are final.
+struct FinishIn {
+    int d_in;
+    int64_t L;
+    int tok_first;
+};
+
+__device__ __forceinline__ FinishIn finish_inputs(const VerifyArgs& a, int64_t b, int lane) {
+    return FinishIn{a.draft_len[b], a.seq_len ? static_cast<int64_t>(a.seq_len[b]) : 0,
+                    lane < a.K ? a.draft[b * a.K + lane] : 0};
+}
+
 // Accept/bonus/append for sequence b, by one warp, once its K+1 target tokens are
-// final.  Everything it reads is requested up front (one round trip when K < 32).
+// final.  Everything it reads is requested up front (one round trip when K < 32);
+// `in` (optional) holds the inputs that were read earlier.
 // Sec. 4.4: n = first i < d with draft_i != target_i (else d), bonus = target_n.
 // Returns (in every lane) the context length after the call: L + n + 1 when the
 // tokens were appended, L when they were not (capacity, no ids), -1 when seq_len
 // is absent or out of range.
 template <typename Src>
 __device__ int64_t finish_sequence(const VerifyArgs& a, int64_t b, int lane, const Src& src,
-                                   FinishOut* out = nullptr) {
+                                   FinishOut* out = nullptr, const FinishIn* in = nullptr) {
     const int K1 = a.K + 1;
-    const int d_in = a.draft_len[b];
-    const int64_t L = a.seq_len ? a.seq_len[b] : 0;
+    const FinishIn fi = in ? *in : finish_inputs(a, b, lane);
+    const int d_in = fi.d_in;
+    const int64_t L = fi.L;
     const int t_first = lane < K1 ? src.at(lane) : 0;
-    const int tok_first = lane < a.K ? a.draft[b * a.K + lane] : 0;
+    const int tok_first = fi.tok_first;
     uint32_t st = 0;
     int d = d_in;
     if (d < 0 || d > a.K) {

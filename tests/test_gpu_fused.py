@@ -71,13 +71,16 @@ def test_draft_step_random(lib, T, V, B, mode):
 
 
 @pytest.mark.parametrize("agg", [0, 1])
-def test_draft_step_rows_threshold_long_draft(lib, agg):
+@pytest.mark.parametrize("layout", ["head", "key"])
+def test_draft_step_rows_threshold_long_draft(lib, agg, layout):
     rng = np.random.default_rng(9 + agg)
     B, T, C, K, d, R = 10, 9000, 40, 70, 512, 16
     ids = rng.integers(0, 4, size=(B, T)).astype(np.int32)      # many candidates: overflow
     lens = rng.integers(2, T + 1, size=B)
     H = torch.randn((B, T, d), device=DEV, dtype=torch.float32)
     A = torch.rand((B, R, T), device=DEV, dtype=torch.float32)
+    if layout == "key":                                          # the R values of a key side by side
+        A = A.transpose(1, 2).contiguous().transpose(1, 2)
     rows = [5, -2, 0, 15, 40, 3]                                  # two invalid rows
     buf = Buffers(B, K, 8, C, DEV)
     gpu_step(buf, i32(ids), i32(lens), None, ngram=(2, 4), H=H, A=A, row_idx=rows, agg=agg,
