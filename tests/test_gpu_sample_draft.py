@@ -172,3 +172,55 @@ def test_sample_draft_decode_loop(lib):
         _same_index(ix_a, ix_b, B, V)
         _oracle_step(g, pre, 1.0, ids_b, L_b, loop.H, loop.A, ng, C, K, "hidden")
     assert (host(L_b) > w.T).all()
+
+
+def test_sample_draft_graph_capture_replays(lib):
+    """One pldp_verify_sample_draft call captured in a CUDA graph and replayed step
+    after step gives the eager call's results, the token index kept up to date by the
+    replays (the uniforms and logits are rewritten in place before each replay)."""
+    w = wl.CONFIGS["decode_loop_b128_ctx32k"].replace(B=16, prompt_len=3000, out_len=1000, V=32000, d=1024)
+    ng = (w.ngram_min, w.ngram_max)
+    B, K, C, V = w.B, w.K, w.C_cap, w.V
+    loops = [wl.DecodeLoop(w, steps=6, device=DEV) for _ in range(2)]
+    bufs = [Buffers(B, K, V, C, DEV) for _ in range(2)]
+    idx = [torch.empty(pk.pldp_index_size(B, V), dtype=torch.uint8, device=DEV) for _ in range(2)]
+    wss = [torch.empty(pk.pldp_verify_sample_draft_workspace_size(B, K, V), dtype=torch.uint8, device=DEV)
+           for _ in range(2)]
+    us = [torch.zeros((B, K + 1), dtype=torch.float32, device=DEV) for _ in range(2)]
+
+    def call(i, stream=None):
+        lp, buf = loops[i], bufs[i]
+        pk.pldp_verify_sample_draft(lp.logits, us[i], buf.draft, buf.dlen, buf.acc, buf.nxt, wss[i], lp.ids,
+                                    lp.seq_len, ng[0], ng[1], buf.cand, buf.cnt, buf.ml, buf.draft, buf.dlen, idx[i],
+                                    temperature=1.0, sampled=buf.argmax, kv_keep_len=buf.kv, stream=stream,
+                                    **_kw(buf, lp.H, lp.A, "hidden"))
+
+    for i in range(2):
+        lp, buf = loops[i], bufs[i]
+        pk.pldp_index_build(lp.ids, lp.seq_len, V, idx[i])
+        lp.step_inputs(0)
+        _draft(buf, lp.ids, lp.seq_len, idx[i], V, lp.H, lp.A, ng, "hidden")
+    # the stats pass's launch shape is looked up once, on an uncaptured call
+    tmp = torch.zeros(B, dtype=torch.int32, device=DEV)
+    pk.pldp_verify_sample(loops[0].logits, us[0], bufs[0].draft, bufs[0].dlen, tmp, tmp.clone(),
+                          torch.empty(pk.pldp_verify_sample_workspace_size(B, K, V), dtype=torch.uint8, device=DEV))
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream()
+    stream.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        call(1, stream=torch.cuda.current_stream())
+    gen = torch.Generator(device=DEV).manual_seed(4)
+    for s in range(6):
+        u = torch.rand((B, K + 1), generator=gen, device=DEV)
+        for i in range(2):
+            loops[i].step_inputs(s)
+            us[i].copy_(u)
+        call(0)
+        graph.replay()
+        torch.cuda.synchronize()
+        ga, gb = _snap(bufs[0]), _snap(bufs[1])
+        for k in ("cnt", "ml", "best_h", "best_a", "draft", "dlen", "acc", "nxt", "argmax", "kv", "status"):
+            assert np.array_equal(ga[k], gb[k]), (s, k)
+        assert torch.equal(loops[0].ids, loops[1].ids) and torch.equal(loops[0].seq_len, loops[1].seq_len)
+        assert torch.equal(idx[0][:4 * B], idx[1][:4 * B])
