@@ -10,14 +10,18 @@
 //  1. The context before x_p is scanned for x_p, each cluster of up to 8 CTAs of
 //     the observation splitting it into consecutive parts (4 bytes per position
 //     against 2 R bytes of attention); every occurrence j gets its overlap ov(j)
-//     (the length of the common suffix of x[..j] and x[..p]) and r* = argmax ov,
-//     the smaller j on ties, from a max of packed keys (ov << 32 | ~j) over the
-//     CTA and then over the cluster's distributed shared memory.
+//     (the length of the common suffix of x[..j] and x[..p], measured by the whole
+//     warp, 32 offsets per round trip) and r* = argmax ov, the smaller j on ties,
+//     from a max of packed keys (ov << 32 | ~j) over the CTA and then over the
+//     cluster: each CTA writes its key into every peer's shared memory and arrives
+//     on the cluster barrier.
 //  2. The R rows of query p-1 are reduced to their first maximum, one warp per
 //     row (16-byte streaming loads where rows allow, packed (value, ~key)
-//     maxima), and a row whose maximum is at r* adds one to counts[r].  The rows
-//     are read first (they do not depend on r*, and they are the bandwidth); the
-//     latency-bound scan of step 1 follows.
+//     maxima).  Only then does the CTA wait on the cluster barrier -- its peers'
+//     keys arrived long before -- and a row whose maximum is at r* adds one to
+//     counts[r].  The short latency-bound scan thus comes first and the rows
+//     (the bandwidth) after it, and no CTA waits at its end for a slower peer or
+//     stays resident for peers that still read its shared memory.
 // pldp_top_heads: one CTA ranks the counts and writes the k rows with the most
 // (ties to the smaller row index) -- the row_idx of pldp_rank_attention.
 #include "pldp_internal.cuh"
@@ -91,23 +95,49 @@ __device__ __forceinline__ unsigned long long row_first_max(const void* row, boo
                 : row_first_max_elem(static_cast<const float*>(row), n, lane);
 }
 
-// Packed (ov, ~j) key of occurrence j of x_p (x_j = x_p known), or 0.
-__device__ __forceinline__ unsigned long long occurrence_key(const int32_t* __restrict__ x, int64_t j, int64_t p,
-                                                             int max_suffix) {
-    int k = 1;                                                      // x_j = x_p itself
-    while (k < max_suffix && j - k >= 0 && __ldg(x + j - k) == __ldg(x + p - k)) ++k;
-    return (static_cast<unsigned long long>(k) << 32) |
+// Packed (ov, ~j) key of occurrence j of x_p (x_j = x_p known), by the whole warp
+// (j, p warp-uniform): lane k of a round compares x_{j-k} with x_{p-k}, so the
+// common suffix is measured 32 tokens per round trip instead of one, and ov is
+// the first offset that differs (or max_suffix, or j + 1 at the context start).
+__device__ __forceinline__ unsigned long long warp_occurrence_key(const int32_t* __restrict__ x, int64_t j,
+                                                                  int64_t p, int max_suffix, int lane) {
+    int ov = max_suffix;
+    for (int k0 = 0; k0 < max_suffix; k0 += 32) {
+        const int k = k0 + lane;
+        const bool same = k < max_suffix && j - k >= 0 && __ldg(x + j - k) == __ldg(x + p - k);
+        const unsigned diff = __ballot_sync(0xFFFFFFFFu, !same);
+        if (diff) {                                                 // warp-uniform
+            ov = k0 + __ffs(diff) - 1;
+            break;
+        }
+    }
+    return (static_cast<unsigned long long>(ov) << 32) |
            static_cast<unsigned long long>(0xFFFFFFFFu - static_cast<uint32_t>(j));
 }
 
+// The occurrences a warp found in one tile, walked by the whole warp one at a time:
+// lane L's bit i of `hits` stands for position pos_of(L, i).  Every lane runs every
+// iteration (the loop condition is a ballot).
+template <typename PosOf>
+__device__ __forceinline__ void walk_hits(uint32_t hits, const int32_t* __restrict__ x, int64_t p, int max_suffix,
+                                          int lane, unsigned long long& best, PosOf pos_of) {
+    for (unsigned who = __ballot_sync(0xFFFFFFFFu, hits != 0); who; who = __ballot_sync(0xFFFFFFFFu, hits != 0)) {
+        const int L = __ffs(who) - 1;
+        const int bit = __shfl_sync(0xFFFFFFFFu, __ffs(hits) - 1, L);
+        const unsigned long long key = warp_occurrence_key(x, pos_of(L, bit), p, max_suffix, lane);
+        best = key > best ? key : best;
+        if (lane == L) hits &= hits - 1;
+    }
+}
+
 template <bool VEC, bool IVEC>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 4)   // 64 registers: 4 CTAs per SM
 identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const int32_t* __restrict__ pos,
                       int64_t T_cap, int max_suffix, const void* __restrict__ A, bool a_bf16, int R,
                       int64_t row_stride, int64_t seq_stride, unsigned* __restrict__ counts,
                       int32_t* __restrict__ r_star, uint32_t* __restrict__ status) {
     __shared__ unsigned long long wkey[kWarps];
-    __shared__ unsigned long long cta_key;                        // this CTA's best occurrence key
+    __shared__ unsigned long long peer_key[kIdentCluster];        // the best occurrence key of each CTA of the cluster
     pdl_enter();
     const int b = blockIdx.y;                                     // the CTAs of one observation are adjacent:
     const int r0 = blockIdx.x * kRowsPerCta;                      // its ids are read once from DRAM, then L2
@@ -122,8 +152,73 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
     }
     const int32_t* x = ids + static_cast<int64_t>(b) * ids_stride;
     const int32_t xp = __ldg(x + p);
-    // 2 (first: it does not depend on r*, and it is the bandwidth). The first maximum of
-    // each of this CTA's rows, two rows per warp.
+    // every CTA of the cluster must be running before any writes into its shared memory
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+    // 1. the copy source r*: the cluster's CTAs (those of one observation) scan
+    //    consecutive parts of [0, p) in tiles, several loads in flight per thread, and
+    //    meet over distributed shared memory
+    cg::cluster_group cluster = cg::this_cluster();
+    const int64_t cs = static_cast<int64_t>(cluster.num_blocks()), crank = cluster.block_rank();
+    unsigned long long best = 0;
+    constexpr int U = IVEC ? 4 : 8;                         // loads in flight per thread
+    // Tiles are walked per warp (the loop bounds are warp-uniform) so that each
+    // warp's occurrences can be measured by all its lanes together.
+    const int64_t wbase = static_cast<int64_t>(warp) * 32;
+    if constexpr (IVEC) {
+        static_assert(U * 4 <= 32, "one hit bit per position of a tile");
+        const int4* x4 = reinterpret_cast<const int4*>(x);
+        const int64_t nq = (p + 3) / 4;                             // int4 units covering [0, p)
+        const int64_t q_lo = nq * crank / cs, q_hi = nq * (crank + 1) / cs;
+        for (int64_t qb = q_lo + wbase; qb < q_hi; qb += static_cast<int64_t>(kThreads) * U) {
+            const int64_t q0 = qb + lane;
+            int4 v[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+                if (q0 + u * kThreads < q_hi) v[u] = __ldg(x4 + q0 + u * kThreads);
+            uint32_t hits = 0;
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int64_t q = q0 + u * kThreads;
+                if (q >= q_hi) continue;
+                const int32_t e[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    if (4 * q + c < p && e[c] == xp) hits |= 1u << (4 * u + c);
+            }
+            walk_hits(hits, x, p, max_suffix, lane, best, [&](int L, int bit) {
+                return 4 * (qb + L + static_cast<int64_t>(bit >> 2) * kThreads) + (bit & 3);
+            });
+        }
+    } else {
+        const int64_t j_lo = p * crank / cs, j_hi = p * (crank + 1) / cs;
+        for (int64_t jb = j_lo + wbase; jb < j_hi; jb += static_cast<int64_t>(kThreads) * U) {
+            const int64_t j0 = jb + lane;
+            int32_t v[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+                if (j0 + u * kThreads < j_hi) v[u] = __ldg(x + j0 + u * kThreads);
+            uint32_t hits = 0;
+#pragma unroll
+            for (int u = 0; u < U; ++u)
+                if (j0 + u * kThreads < j_hi && v[u] == xp) hits |= 1u << u;
+            walk_hits(hits, x, p, max_suffix, lane, best, [&](int L, int bit) {
+                return jb + L + static_cast<int64_t>(bit) * kThreads;
+            });
+        }
+    }
+    best = warp_max_u64(best);
+    if (lane == 0) wkey[warp] = best;
+    asm volatile("barrier.cluster.wait.aligned;" ::: "memory");  // every peer has started
+    __syncthreads();
+    if (tid == 0) {                                               // this CTA's best, into every peer's slot
+        unsigned long long k = 0;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) k = wkey[w] > k ? wkey[w] : k;
+        for (int c = 0; c < static_cast<int>(cs); ++c) *cluster.map_shared_rank(&peer_key[crank], c) = k;
+    }
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    // 2. the first maximum of each of this CTA's rows, one row per warp, while the
+    //    peers' keys come in
     constexpr int RW = kRowsPerCta / kWarps;
     const size_t es = a_bf16 ? 2 : 4;
     const char* ab = static_cast<const char*>(A) + static_cast<int64_t>(b) * seq_stride * es;
@@ -134,74 +229,9 @@ identify_heads_kernel(const int32_t* __restrict__ ids, int64_t ids_stride, const
         const int r = r0 + warp + i * kWarps;
         rk[i] = r < r1 ? row_first_max<VEC>(ab + static_cast<int64_t>(r) * row_stride * es, a_bf16, p, lane) : 0ull;
     }
-    // 1. the copy source r*: the cluster's CTAs (those of one observation) scan
-    //    consecutive parts of [0, p) in tiles, eight loads in flight per thread, and
-    //    meet over distributed shared memory
-    cg::cluster_group cluster = cg::this_cluster();
-    const int64_t cs = static_cast<int64_t>(cluster.num_blocks()), crank = cluster.block_rank();
-    unsigned long long best = 0;
-    constexpr int U = 8;
-    if constexpr (IVEC) {
-        const int4* x4 = reinterpret_cast<const int4*>(x);
-        const int64_t nq = (p + 3) / 4;                             // int4 units covering [0, p)
-        const int64_t q_lo = nq * crank / cs, q_hi = nq * (crank + 1) / cs;
-        for (int64_t q0 = q_lo + tid; q0 < q_hi; q0 += static_cast<int64_t>(kThreads) * U) {
-            int4 v[U];
-#pragma unroll
-            for (int u = 0; u < U; ++u)
-                if (q0 + u * kThreads < q_hi) v[u] = __ldg(x4 + q0 + u * kThreads);
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const int64_t q = q0 + u * kThreads;
-                if (q >= q_hi) continue;
-                const int32_t e[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    const int64_t j = 4 * q + c;
-                    if (j < p && e[c] == xp) {
-                        const unsigned long long key = occurrence_key(x, j, p, max_suffix);
-                        best = key > best ? key : best;
-                    }
-                }
-            }
-        }
-    } else {
-        const int64_t j_lo = p * crank / cs, j_hi = p * (crank + 1) / cs;
-        for (int64_t j0 = j_lo + tid; j0 < j_hi; j0 += static_cast<int64_t>(kThreads) * U) {
-            int32_t v[U];
-#pragma unroll
-            for (int u = 0; u < U; ++u)
-                if (j0 + u * kThreads < j_hi) v[u] = __ldg(x + j0 + u * kThreads);
-#pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const int64_t j = j0 + u * kThreads;
-                if (j < j_hi && v[u] == xp) {
-                    const unsigned long long key = occurrence_key(x, j, p, max_suffix);
-                    best = key > best ? key : best;
-                }
-            }
-        }
-    }
-    best = warp_max_u64(best);
-    if (lane == 0) wkey[warp] = best;
-    __syncthreads();
-    if (tid == 0) {
-        unsigned long long k = 0;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) k = wkey[w] > k ? wkey[w] : k;
-        cta_key = k;
-    }
-    cluster.sync();                                               // every CTA's part is in
-    if (tid == 0) {
-        unsigned long long k = 0;
-        for (int c = 0; c < static_cast<int>(cs); ++c) {
-            const unsigned long long o = *cluster.map_shared_rank(&cta_key, c);
-            k = o > k ? o : k;
-        }
-        wkey[0] = k;
-    }
-    cluster.sync();                                               // read before any CTA of the cluster leaves
-    best = wkey[0];
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");   // every peer's key is in
+    best = 0;
+    for (int c = 0; c < static_cast<int>(cs); ++c) best = peer_key[c] > best ? peer_key[c] : best;
     const int64_t rs = best ? static_cast<int64_t>(0xFFFFFFFFu - static_cast<uint32_t>(best & 0xFFFFFFFFull)) : -1;
     if (tid == 0 && blockIdx.x == 0 && r_star) r_star[b] = static_cast<int32_t>(rs);
     if (rs < 0) return;
