@@ -53,6 +53,7 @@ constexpr int kScoreUnroll = 2;                                // 16-byte row lo
 constexpr int kScoreBatch = 2;                                 // occurrences scored per pass (scan kernel)
 constexpr int kMaxScoreBatch = 4;                              // ... and at most (the indexed kernel)
 constexpr int kSpeculate = kMaxScoreBatch;                     // occurrences scored before their suffix match
+constexpr int kPrefetchOcc = 32;                                // occurrences whose rows are prefetched otherwise
 constexpr size_t kMaxQueryBytes = 196608;
 constexpr int kMaxSelRows = 8192;
 constexpr int64_t kMaxPositions = int64_t(1) << 27;            // (j << 4) | m fits 31 bits
@@ -794,6 +795,24 @@ __device__ __forceinline__ void index_draft(const DraftParams& p, const IndexVie
     float* hsc = (HAS_H && p.h_scores) ? p.h_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
     float* asc = (has_a && p.a_scores) ? p.a_scores + static_cast<int64_t>(b) * p.C_cap : nullptr;
     const int nocc = indexed ? is.nocc : 0;
+    // More occurrences than are scored at once: the suffix matches come first, and
+    // meanwhile the rows of (up to kPrefetchOcc of) the occurrences head for L2 --
+    // H_{j-1} with one bulk prefetch, the attention values at key j when the
+    // selected rows of a key are side by side -- so that the candidates' scoring,
+    // a round trip later, finds them there.
+    if (indexed && nocc > kSpeculate && tid < nocc && tid < kPrefetchOcc) {
+        const int64_t j = is.occ[tid];
+        if (HAS_H && j >= 1 && j < t)
+            prefetch_l2_bulk(static_cast<const char*>(p.H) + (static_cast<int64_t>(b) * p.h_seq_stride + (j - 1) * p.d) * h_es,
+                             static_cast<uint32_t>(p.d * h_es));
+        if (has_a && p.a_row_stride == 1 && !p.row_idx && j >= 0 && j < t) {
+            const size_t a_es = p.a_bf16 ? 2 : 4;
+            const char* run = static_cast<const char*>(p.A) + (static_cast<int64_t>(b) * p.a_seq_stride + j * p.a_key_stride) * a_es;
+            const char* end = run + static_cast<int64_t>(p.R) * a_es;          // every address inside the run
+            for (const char* a = run; a < end; a += 128) asm volatile("prefetch.global.L2 [%0];" ::"l"(a));
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(end - 1));
+        }
+    }
 
     // Warp 0: the choices of both rankings (best keys hk, ak), the draft (Sec. 4.3)
     // with draft_tok(i, j*) giving token j* + 1 + i, and the per-sequence outputs.
