@@ -85,8 +85,12 @@ __device__ __forceinline__ void prefetch_first(RankShared& sh, const int32_t* ca
     }
 }
 
+// 72 registers: the compiler's own choice for 256 threads was 64 with spills of the
+// per-warp candidate stream (8 loads in flight per lane); without them, at 3 CTAs per
+// SM, Eq. 3 on 510 candidates per sequence measured 116.6 -> 109.5 us (128 candidates:
+// 42.8 -> 43.3 us), alternated on one box.
 template <typename T, bool VEC, bool CLUSTER>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __maxnreg__(72)
 rank_hidden_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride,
                    const int32_t* __restrict__ seq_len, int64_t T_cap,
                    const int32_t* __restrict__ cand_pos, const int32_t* __restrict__ cand_count,
