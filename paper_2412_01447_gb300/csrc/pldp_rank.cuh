@@ -395,6 +395,77 @@ __device__ __forceinline__ void attention_rank_warp(const void* ab, bool a_bf16,
     if (lane == 0 && best > sh.slot_key[bt.slot]) sh.slot_key[bt.slot] = best;
 }
 
+// Eq. 2 under MAX with one warp per candidate when the selected rows of a key are
+// one dense run of nv 16-byte vectors (all R rows in order, row stride 1: the
+// key-major layout; nv a power of two, at most 32 * kDenseLoads): the warp reads
+// whole vectors -- up to kDenseLoads per lane in flight, 32 * kDenseLoads vectors,
+// i.e. several candidates' runs at once when they are short -- instead of one value
+// per lane.  A lane's vectors belong to one candidate per load; the max over the
+// nv lanes (nv <= 32) or the nv / 32 loads and the warp (nv > 32) of a candidate is
+// exact, so the scores are those of the value-per-lane path bit for bit.
+constexpr int kDenseLoads = 4;
+
+template <typename T, bool CANDS_SHARED>
+__device__ __forceinline__ void attention_rank_warp_dense(const T* ab, int nv, int64_t key_stride, int64_t t,
+                                                          const int32_t* __restrict__ cands, int S, int rank,
+                                                          const int32_t* jpre, float* __restrict__ scores_row,
+                                                          RankShared& sh, const Batch& bt) {
+    constexpr int VW = 16 / static_cast<int>(sizeof(T));
+    const int lane = threadIdx.x & 31;
+    const int P = bt.P;
+    const int lpc = nv < 32 ? nv : 32;                    // lanes per candidate and load
+    const int cpl = 32 / lpc;                             // candidates per load
+    const int vpl = nv / lpc;                             // loads per lane per candidate (<= kDenseLoads)
+    const int ng = kDenseLoads / vpl;                     // load groups (one candidate per lane each)
+    unsigned long long best = 0;
+    for (int i0 = 0; bt.slot + i0 * P < bt.n_local; i0 += ng * cpl) {   // warp-uniform
+        uint4 x[kDenseLoads];
+        int32_t jl[kDenseLoads];                          // this lane's candidate position in load u, or -1
+#pragma unroll
+        for (int u = 0; u < kDenseLoads; ++u) {
+            const int g = u / vpl;                        // runtime divisor: a shift (vpl a power of two)
+            const int k = bt.slot + (i0 + g * cpl + lane / lpc) * P;
+            int32_t j = -1;
+            if (k < bt.n_local) {
+                const int64_t jj = cand_at<CANDS_SHARED>(cands, jpre, k, rank + S * k, P);
+                if (jj >= 0 && jj < t) j = static_cast<int32_t>(jj);
+            }
+            jl[u] = j;
+            if (j >= 0)
+                x[u] = *reinterpret_cast<const uint4*>(
+                    ab + j * key_stride + static_cast<int64_t>((u - g * vpl) * lpc + lane % lpc) * VW);
+        }
+        float m[kDenseLoads];
+#pragma unroll
+        for (int u = 0; u < kDenseLoads; ++u) m[u] = jl[u] >= 0 ? vmax(x[u], T()) : -INFINITY;
+        // fold each group's vpl loads into its first (registers only: the indices are fixed)
+#pragma unroll
+        for (int st = 1; st < kDenseLoads; st <<= 1)
+#pragma unroll
+            for (int u = 0; u + st < kDenseLoads; u += 2 * st)
+                if (st < vpl) m[u] = fmaxf(m[u], m[u + st]);
+        // then over the candidate's lanes; lane q * lpc writes candidate i0 + g * cpl + q
+#pragma unroll
+        for (int u = 0; u < kDenseLoads; ++u) {
+            if (u % vpl != 0) continue;                   // warp-uniform
+            float v = m[u];
+            for (int o = lpc / 2; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+            const int k = bt.slot + (i0 + (u / vpl) * cpl + lane / lpc) * P;
+            if (lane % lpc == 0 && k < bt.n_local) {
+                const int32_t j = jl[u];
+                const float sc = j >= 0 ? v : -INFINITY;
+                if (scores_row) scores_row[rank + S * k] = sc;
+                if (j >= 0) {
+                    const unsigned long long key = pack_key(sc, static_cast<uint32_t>(j));
+                    best = key > best ? key : best;
+                }
+            }
+        }
+    }
+    best = warp_max_u64(best);
+    if (lane == 0 && best > sh.slot_key[bt.slot]) sh.slot_key[bt.slot] = best;
+}
+
 // Eq. 2 for this CTA's candidates.  `rows_sh` (shared) holds the element offset
 // of each selected row, or -1 for an invalid one; key j of a row is key_stride
 // elements after key j - 1.  Same conventions as
@@ -406,9 +477,20 @@ __device__ __forceinline__ void attention_rank_cta(const void* ab, bool a_bf16,
                                                    const int32_t* __restrict__ cands, int n, int S,
                                                    int rank, const int32_t* jpre, bool is_max,
                                                    float* __restrict__ scores_row, RankShared& sh,
-                                                   const WarpGroup& wg = whole_cta()) {
+                                                   const WarpGroup& wg = whole_cta(), int dense_nv = 0) {
     const int lane = threadIdx.x & 31, warp = wg.warp();
     const Batch bt = batch_shape(n, S, rank, wg);
+    if (bt.G == 1 && dense_nv > 0 && is_max) {            // one warp per candidate, whole vectors
+        if (a_bf16)
+            attention_rank_warp_dense<__nv_bfloat16, CANDS_SHARED>(static_cast<const __nv_bfloat16*>(ab), dense_nv,
+                                                                   key_stride, t, cands, S, rank, jpre, scores_row,
+                                                                   sh, bt);
+        else
+            attention_rank_warp_dense<float, CANDS_SHARED>(static_cast<const float*>(ab), dense_nv, key_stride, t,
+                                                           cands, S, rank, jpre, scores_row, sh, bt);
+        wg.sync();
+        return;
+    }
     if (bt.G == 1) {                                      // one warp per candidate: no barriers
         attention_rank_warp<CANDS_SHARED>(ab, a_bf16, rows_sh, n_sel, key_stride, t, cands, S, rank, jpre, is_max,
                                           scores_row, sh, bt);

@@ -306,10 +306,12 @@ rank_hidden_avg_kernel(const T* __restrict__ H, int64_t d, int64_t seq_stride, i
     store_best<CLUSTER>(sh, mine, b, best_pos, best_score, status, PLDP_ST_TIMEOUT);
 }
 
-template <bool CLUSTER>
+// DENSE: all R rows in order, each key's values one run of dense_nv 16-byte vectors
+// (checked on the host), ranked under MAX with whole-vector loads.
+template <bool CLUSTER, bool DENSE>
 __global__ void __launch_bounds__(kThreads)
 rank_attention_kernel(const void* __restrict__ A, bool a_bf16, int R, int64_t row_stride, int64_t key_stride,
-                      int64_t seq_stride, const int32_t* __restrict__ row_idx, int n_sel, int agg,
+                      int64_t seq_stride, const int32_t* __restrict__ row_idx, int n_sel, int agg, int dense_nv,
                       const int32_t* __restrict__ seq_len, int64_t T_cap,
                       const int32_t* __restrict__ cand_pos, const int32_t* __restrict__ cand_count,
                       int C_cap, float* __restrict__ scores, int32_t* __restrict__ best_pos,
@@ -344,7 +346,8 @@ rank_attention_kernel(const void* __restrict__ A, bool a_bf16, int R, int64_t ro
     const void* ab = static_cast<const char*>(A) + static_cast<int64_t>(b) * seq_stride * es;
     attention_rank_cta(ab, a_bf16, rows_sh, n_sel, key_stride, t, cand_pos + static_cast<int64_t>(b) * C_cap, n, S,
                        rank, sh.jpre, agg == PLDP_AGG_MAX,
-                       scores ? scores + static_cast<int64_t>(b) * C_cap : nullptr, sh);
+                       scores ? scores + static_cast<int64_t>(b) * C_cap : nullptr, sh, whole_cta(),
+                       DENSE ? dense_nv : 0);
     store_best<CLUSTER>(sh, mine, b, best_pos, best_score, status, PLDP_ST_TIMEOUT);
 }
 
@@ -396,18 +399,32 @@ cudaError_t launch_hidden(int B, int S, size_t smem, void* stream, const T* h, i
                        best_score, status);
 }
 
+template <bool DENSE>
 cudaError_t launch_attention(int B, int S, size_t smem, void* stream, const void* a, bool a_bf16,
                              int R, int64_t row_stride, int64_t key_stride, int64_t seq_stride, const int32_t* row_idx,
-                             int sel, int agg, const int32_t* seq_len, int64_t T_cap,
+                             int sel, int agg, int dense_nv, const int32_t* seq_len, int64_t T_cap,
                              const int32_t* cand_pos, const int32_t* cand_count, int C_cap,
                              float* scores, int32_t* best_pos, float* best_score, uint32_t* status) {
     if (S > 1)
-        return launch_rank(rank_attention_kernel<true>, B, S, smem, stream, a, a_bf16, R, row_stride, key_stride,
-                           seq_stride, row_idx, sel, agg, seq_len, T_cap, cand_pos, cand_count, C_cap,
-                           scores, best_pos, best_score, status);
-    return launch_rank(rank_attention_kernel<false>, B, S, smem, stream, a, a_bf16, R, row_stride, key_stride,
-                       seq_stride, row_idx, sel, agg, seq_len, T_cap, cand_pos, cand_count, C_cap,
+        return launch_rank(rank_attention_kernel<true, DENSE>, B, S, smem, stream, a, a_bf16, R, row_stride,
+                           key_stride, seq_stride, row_idx, sel, agg, dense_nv, seq_len, T_cap, cand_pos, cand_count,
+                           C_cap, scores, best_pos, best_score, status);
+    return launch_rank(rank_attention_kernel<false, DENSE>, B, S, smem, stream, a, a_bf16, R, row_stride, key_stride,
+                       seq_stride, row_idx, sel, agg, dense_nv, seq_len, T_cap, cand_pos, cand_count, C_cap,
                        scores, best_pos, best_score, status);
+}
+
+// Vectors per key of the dense form of Eq. 2 (all rows in order, row stride 1, every
+// run 16-byte aligned, a power of two of vectors up to 32 * kDenseLoads), or 0.
+int dense_vectors(const void* A, size_t es, int R, int64_t row_stride, int64_t key_stride, int64_t seq_stride,
+                  const int32_t* row_idx, pldp_agg agg) {
+    if (agg != PLDP_AGG_MAX || row_idx || row_stride != 1 || !aligned16(A)) return 0;
+    if ((key_stride * static_cast<int64_t>(es)) % 16 || (seq_stride * static_cast<int64_t>(es)) % 16) return 0;
+    const int64_t bytes = static_cast<int64_t>(R) * static_cast<int64_t>(es);
+    if (bytes % 16) return 0;
+    const int64_t nv = bytes / 16;
+    if (nv > 32 * kDenseLoads || (nv & (nv - 1))) return 0;
+    return static_cast<int>(nv);
 }
 
 template <typename T, bool VEC>
@@ -550,11 +567,19 @@ extern "C" PLDP_API pldp_status pldp_rank_attention(const void* A, pldp_dtype dt
         return fail(PLDP_ERR_INVALID_ARG, "rank_attention: null pointer");
 
     const size_t smem = static_cast<size_t>(sel) * sizeof(int64_t);
-    const int S = pick_split(B, C_cap, reinterpret_cast<const void*>(&rank_attention_kernel<true>), smem);
+    const int nv = dense_vectors(A, dtype == PLDP_F32 ? 4 : 2, R, row_stride, key_stride, seq_stride, row_idx, agg);
     cudaError_t e;
-    e = launch_attention(B, S, smem, stream, A, dtype == PLDP_BF16, R, row_stride, key_stride, seq_stride, row_idx,
-                         sel, static_cast<int>(agg), seq_len, T_cap, cand_pos, cand_count, C_cap,
-                         scores, best_pos, best_score, status);
+    if (nv > 0) {
+        const int S = pick_split(B, C_cap, reinterpret_cast<const void*>(&rank_attention_kernel<true, true>), smem);
+        e = launch_attention<true>(B, S, smem, stream, A, dtype == PLDP_BF16, R, row_stride, key_stride, seq_stride,
+                                   row_idx, sel, static_cast<int>(agg), nv, seq_len, T_cap, cand_pos, cand_count, C_cap,
+                                   scores, best_pos, best_score, status);
+    } else {
+        const int S = pick_split(B, C_cap, reinterpret_cast<const void*>(&rank_attention_kernel<true, false>), smem);
+        e = launch_attention<false>(B, S, smem, stream, A, dtype == PLDP_BF16, R, row_stride, key_stride, seq_stride,
+                                    row_idx, sel, static_cast<int>(agg), 0, seq_len, T_cap, cand_pos, cand_count,
+                                    C_cap, scores, best_pos, best_score, status);
+    }
     if (e != cudaSuccess)
         return fail(PLDP_ERR_CUDA, "rank_attention: launch failed: %s", cudaGetErrorString(e));
     return PLDP_OK;

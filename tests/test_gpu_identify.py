@@ -22,9 +22,10 @@ def i32(x):
 @pytest.mark.parametrize("T,dtype", [(256, torch.bfloat16), (301, torch.bfloat16), (200, torch.float32),
                                      (4096, torch.bfloat16)])
 @pytest.mark.parametrize("V,max_suffix", [(3, 64), (20, 2), (200, 64)])
-# R = 20: 3 CTAs of 8 rows per observation, one cluster of 3; R = 72: 9 CTAs in clusters
-# of 8, the grid padded with 7 CTAs that hold no rows but take part in the scan
-@pytest.mark.parametrize("R", [20, 72])
+# R = 5: one CTA per observation (a cluster of one); R = 20: 3 CTAs of 8 rows per
+# observation, one cluster of 3; R = 72: 9 CTAs in clusters of 8, the grid padded with 7
+# CTAs that hold no rows but take part in the scan
+@pytest.mark.parametrize("R", [5, 20, 72])
 def test_identify_heads_matches_oracle(lib, T, dtype, V, max_suffix, R):
     rng = np.random.default_rng(T + V + max_suffix + R)
     B = 24

@@ -16,13 +16,21 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda"
 
 
-@pytest.mark.parametrize("B,T,V,d,R,dtype,C_cap,thr,agg", [
-    (128, 32768, 64, 4096, 128, torch.bfloat16, 1024, float("-inf"), 0),
-    (128, 32768, 256, 4096, 128, torch.bfloat16, 1024, float("-inf"), 1),
-    (24, 9000, 40, 1000, 16, torch.float32, 300, 0.02, 0),
-    (7, 20000, 30, 768, 48, torch.bfloat16, 2048, float("-inf"), 1),
+# key_major: the R values of a key side by side, as the benchmark holds them.  Under MAX
+# with all rows and whole 16-byte runs of a power-of-two count of vectors, Eq. 2 takes
+# the dense whole-vector path: 16 vectors a key (R = 128 bf16, R = 64 f32), 4 (R = 32
+# bf16) and 128 (R = 1024 bf16, several loads per lane); SUM stays on the value path.
+@pytest.mark.parametrize("B,T,V,d,R,dtype,C_cap,thr,agg,key_major", [
+    (128, 32768, 64, 4096, 128, torch.bfloat16, 1024, float("-inf"), 0, True),
+    (128, 32768, 256, 4096, 128, torch.bfloat16, 1024, float("-inf"), 1, False),
+    (24, 9000, 40, 1000, 16, torch.float32, 300, 0.02, 0, False),
+    (7, 20000, 30, 768, 48, torch.bfloat16, 2048, float("-inf"), 1, False),
+    (16, 6000, 12, 256, 32, torch.bfloat16, 1024, float("-inf"), 0, True),
+    (16, 6000, 12, 256, 32, torch.bfloat16, 1024, float("-inf"), 1, True),
+    (8, 4000, 8, 128, 1024, torch.bfloat16, 1024, float("-inf"), 0, True),
+    (12, 5000, 20, 512, 64, torch.float32, 600, float("-inf"), 0, True),
 ])
-def test_candidate_heavy_rankings(lib, B, T, V, d, R, dtype, C_cap, thr, agg):
+def test_candidate_heavy_rankings(lib, B, T, V, d, R, dtype, C_cap, thr, agg, key_major):
     rng = np.random.default_rng(T + V)
     gen = torch.Generator(device=DEV).manual_seed(V)
     ids = rng.integers(0, V, size=(B, T)).astype(np.int32)
@@ -33,7 +41,7 @@ def test_candidate_heavy_rankings(lib, B, T, V, d, R, dtype, C_cap, thr, agg):
     L_g = torch.as_tensor(lens, device=DEV)
     H = torch.randn((B, T, d), generator=gen, device=DEV).to(dtype)
     A = torch.rand((B, R, T), generator=gen, device=DEV).to(dtype)
-    if V == 64:                                          # key-major, as the benchmark holds them
+    if key_major:
         A = A.transpose(1, 2).contiguous().transpose(1, 2)
     buf = Buffers(B, 8, 8, C_cap, DEV)
     lib.pldp_find_candidates(ids_g, L_g, 1, 1, buf.cand, buf.cnt, buf.ml, buf.status)
