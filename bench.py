@@ -934,6 +934,17 @@ def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
         hm = rec["rank_attention_head_major"]
         hm["sector_bytes"] = n_list * w.R * 32.0
         hm["sector_gbs"] = round(hm["sector_bytes"] / (hm["us"] * 1e-6) / 1e9, 1)
+        if V == max(2, T // 512):
+            # Eq. 2 over 1024 rows a key (e.g. 32 layers x 32 heads), key-major: the same
+            # candidates with 2 KB of attention values each, bytes enough to show bandwidth
+            Rw = 1024
+            gw = torch.Generator(device=dev).manual_seed(w.seed + 1024)
+            A_wide = torch.rand((B, T_cap, Rw), generator=gw, device=dev).to(torch.bfloat16).transpose(1, 2)
+            tw = _time_calls([("rank_attention_1024_rows", lambda: pk.pldp_rank_attention(A_wide, L, cand, cnt,
+                                                                                          best_a))],
+                             flush_l2, iters, warm)
+            rec["rank_attention_1024_rows"] = _call_stats(tw["rank_attention_1024_rows"], n_list * Rw * 2.0, peak)
+            del A_wide
         if V == max(2, T // 128):      # at most 256 occurrences per sequence: the launch's own scoring path
             t = _time_calls([("draft_step", lambda: pk.pldp_draft_step(
                 ids, L, 1, 1, cand, cnt, ml, w.K, draft, dlen, dws, H=loop.H, best_h=best_h, A=loop.A,
@@ -946,7 +957,8 @@ def time_rank_stress(pk, loop, w, flush_l2, peak, iters=32, warm=3):
     del A_head
     out.update({"batch": B, "context": T, "d": w.d, "attention_rows": w.R, "C_cap": C,
                 "attention_layout": "rank_attention: key-major (the loop's layout); rank_attention_head_major: "
-                                    "the same values with each row's keys side by side",
+                                    "the same values with each row's keys side by side; rank_attention_1024_rows: "
+                                    "1024 key-major rows of uniform values, the same candidates",
                 "timing": "CUDA events around each call, L2 flushed before each; hidden rows and attention "
                           "values are the decode loop's own tensors"})
     return out

@@ -14,8 +14,9 @@ pytestmark = pytest.mark.gpu
 DEV = "cuda"
 
 
-@pytest.mark.parametrize("layout", ["head", "key"])
-def test_rank_attention_reads_host_rows_in_place(lib, layout):
+# all rows of a key-major layout take the dense whole-vector form of Eq. 2 (MAX)
+@pytest.mark.parametrize("layout,select", [("head", True), ("key", True), ("key", False)])
+def test_rank_attention_reads_host_rows_in_place(lib, layout, select):
     rng = np.random.default_rng(4)
     B, R, T, C = 12, 32, 3000, 64
     A = torch.rand((B, R, T), device=DEV).to(torch.bfloat16)
@@ -26,7 +27,7 @@ def test_rank_attention_reads_host_rows_in_place(lib, layout):
     lens = torch.as_tensor(rng.integers(2, T + 1, size=B).astype(np.int32), device=DEV)
     cands = torch.as_tensor(np.sort(rng.choice(T - 1, (B, C)), axis=1).astype(np.int32), device=DEV)
     cnt = torch.as_tensor(rng.integers(0, C + 1, size=B).astype(np.int32), device=DEV)
-    rows = torch.as_tensor(np.array([3, 7, 1, 30, 12], np.int32), device=DEV)
+    rows = torch.as_tensor(np.array([3, 7, 1, 30, 12], np.int32), device=DEV) if select else None
     out = []
     for src in (A, A_host):
         buf = Buffers(B, 4, 8, C, DEV)
