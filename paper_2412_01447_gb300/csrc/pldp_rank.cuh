@@ -423,7 +423,7 @@ __device__ __forceinline__ void attention_rank_warp_dense(const T* ab, int nv, i
         int32_t jl[kDenseLoads];                          // this lane's candidate position in load u, or -1
 #pragma unroll
         for (int u = 0; u < kDenseLoads; ++u) {
-            const int g = u / vpl;                        // runtime divisor: a shift (vpl a power of two)
+            const int g = u / vpl;                        // the load group (vpl: 1, 2 or 4)
             const int k = bt.slot + (i0 + g * cpl + lane / lpc) * P;
             int32_t j = -1;
             if (k < bt.n_local) {
